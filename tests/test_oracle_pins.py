@@ -1,0 +1,273 @@
+"""Pins of the CPU oracle against things other than itself.
+
+* torch.nn's Transformer decoder (library) for the decoder forward, the
+  block-causal mask of a verification pass, the cross-attention padding mask
+  and the cached encoder K/V (Sec. 3 "Speculative Loop": the target checks the
+  block in one pass);
+* torch.nn.MultiheadAttention's head-averaged weights for the runtime anchor
+  (Sec. 5 "Verification-Attention Correction");
+* brute-force enumeration of every draft block on a tiny vocabulary for the
+  longest-prefix rule (Sec. 3);
+* the lossless invariant: speculative output equals plain greedy decoding
+  (Sec. 1, Sec. 3: identical under exact arithmetic);
+* rollback followed by the same verification reproduces outputs and cache;
+* special cases: no drafts is one greedy step, true drafts are all accepted,
+  wrong drafts are all rejected.
+"""
+import itertools
+
+import numpy as np
+import pytest
+
+import workload as W
+from oracle import Oracle, OracleError, greedy_transcript
+from tests.torch_ref import TorchDecoder
+
+TINY = W.ModelDims(n_layers=2, d_model=64, n_heads=2, d_ffn=256, vocab=97, dtype="fp32",
+                   max_pos=64, max_enc=40, anchor_layer=1)
+ENC_LENS = [23, 40, 7]
+
+
+def _setup(dims=TINY, enc_lens=ENC_LENS, std=0.3, t_max=None, prompt_len=W.PROMPT_LEN):
+    blob = W.make_weights(dims, std=std)
+    t_max = t_max or max(enc_lens)
+    enc = W.make_encoder_states(dims, enc_lens, t_max)
+    o = Oracle(dims, blob)
+    o.encode_cache(enc, enc_lens)
+    prompt = W.make_prompt(dims, len(enc_lens), prompt_len)
+    o.prefill(prompt)
+    return o, blob, enc, prompt
+
+
+@pytest.mark.parametrize("std", [0.02, 0.3])
+def test_verify_rows_match_torch_decoder(std):
+    """Every verify row equals the library decoder's full-sequence logits at the
+    same position: the cache, the block-causal mask and the encoder K/V are right."""
+    o, blob, enc, prompt = _setup(std=std)
+    ref = TorchDecoder(TINY, blob)
+    rng = np.random.default_rng(7)
+    hist = [list(prompt[b]) for b in range(3)]
+    for step in range(4):
+        k = 5
+        draft = rng.integers(0, TINY.vocab, size=(3, k))
+        lens = np.array([5, 2, 0])
+        res = o.verify(draft, lens)
+        for b in range(3):
+            rows = [r for r, (bb, _) in enumerate(res.rows) if bb == b]
+            seq = hist[b] + [int(t) for t in draft[b, :lens[b]]]
+            logits, _ = ref.forward(seq, enc[b], ENC_LENS[b])
+            start = len(hist[b]) - 1          # position of the pending token
+            np.testing.assert_allclose(res.logits[rows], logits[start:start + lens[b] + 1],
+                                       rtol=0, atol=1e-10)
+            hist[b] = hist[b] + [int(t) for t in draft[b, :res.accepted[b]]] + [int(res.bonus[b])]
+
+
+def test_anchor_matches_torch_head_mean_weights():
+    """The anchor profile is torch's head-averaged cross-attention at the anchor
+    layer, read at the row whose argmax is the bonus token; the anchor is its peak."""
+    o, blob, enc, prompt = _setup()
+    ref = TorchDecoder(TINY, blob)
+    rng = np.random.default_rng(3)
+    hist = [list(prompt[b]) for b in range(3)]
+    for step in range(3):
+        draft = rng.integers(0, TINY.vocab, size=(3, 3))
+        res = o.verify(draft, np.array([3, 3, 1]))
+        for b in range(3):
+            seq = hist[b] + [int(t) for t in draft[b, :3]]
+            _, w = ref.forward(seq, enc[b], ENC_LENS[b], anchor_layer=TINY.anchor)
+            row = len(hist[b]) - 1 + int(res.accepted[b])
+            np.testing.assert_allclose(res.anchor_profile[b], w[row], rtol=0, atol=1e-12)
+            assert res.anchor[b] == int(np.argmax(w[row]))
+            hist[b] = hist[b] + [int(t) for t in draft[b, :res.accepted[b]]] + [int(res.bonus[b])]
+
+
+def test_anchor_planted_peak():
+    """Overwriting one frame's anchor-layer keys with a large multiple of the
+    scored row's query (per head) must move the anchor to that frame.  The
+    anchor-layer query is computed before that layer's cross-attention, so the
+    planted keys do not change it."""
+    o, blob, enc, prompt = _setup()
+    snap = o.snapshot()
+    rows = [(b, int(o.pending[b]), int(o.kv_len[b])) for b in range(3)]
+    _, q_anchor = o._forward(rows)
+    o.restore(snap)
+    hd = TINY.head_dim
+    targets = [17, 39, 0]
+    for b, jstar in enumerate(targets):
+        q = q_anchor[b]
+        key = np.concatenate([q[h * hd:(h + 1) * hd] / np.linalg.norm(q[h * hd:(h + 1) * hd])
+                              for h in range(TINY.n_heads)])
+        o.Kx[TINY.anchor][b][jstar] = 80.0 * key
+    res = o.verify(np.zeros((3, 1), dtype=int), np.zeros(3, dtype=int))
+    assert list(res.anchor) == targets
+    for b, jstar in enumerate(targets):
+        assert res.anchor_profile[b][jstar] > 0.99
+
+
+def _greedy_continuation(o, n):
+    snap = o.snapshot()
+    out = []
+    for _ in range(n):
+        out.append(o.ar_step())
+    o.restore(snap)
+    return np.stack(out, axis=1)      # [B, n]
+
+
+def test_accept_brute_force_tiny_vocab():
+    """Accepted length equals the longest prefix of the block that matches the
+    target's greedy continuation, for every draft block over an 8-token vocabulary."""
+    dims = W.ModelDims(n_layers=1, d_model=64, n_heads=1, d_ffn=128, vocab=8, dtype="fp32",
+                       max_pos=32, max_enc=16, anchor_layer=0)
+    o, *_ = _setup(dims, enc_lens=[11, 16], std=0.5, prompt_len=2)
+    for _ in range(2):   # two different states
+        g = _greedy_continuation(o, 4)           # g[:, j] = greedy token j+1 after pending
+        snap = o.snapshot()
+        for k in (1, 2, 3):
+            for block in itertools.product(range(8), repeat=k):
+                for lens_b in range(k + 1):
+                    o.restore(snap)
+                    draft = np.array([block, block[::-1]])
+                    res = o.verify(draft, np.array([lens_b, k]))
+                    for b in range(2):
+                        L = lens_b if b == 0 else k
+                        n = 0
+                        while n < L and draft[b, n] == g[b, n]:
+                            n += 1
+                        assert res.accepted[b] == n
+                        assert res.bonus[b] == g[b, n]
+                        assert res.kv_len[b] == snap[2][b] + 1 + n
+                        assert res.restart[b] == int(n < L)
+        o.restore(snap)
+        o.ar_step()
+
+
+def test_lossless_speculative_equals_greedy():
+    """Speculative decoding with corrupted and slipped drafts returns exactly the
+    plain greedy sequence, which itself equals the library decoder's greedy
+    decoding by full recomputation."""
+    total = [30, 22, 27]
+    o, blob, enc, prompt = _setup()
+    snap = o.snapshot()
+    truth = greedy_transcript(o, prompt, total)
+    ref = TorchDecoder(TINY, blob)
+    for b in range(3):
+        assert list(truth[b, :total[b]]) == ref.greedy(prompt[b], enc[b], ENC_LENS[b], total[b])
+    wl = W.Workload("t", TINY, 3, 5, tuple(t - W.PROMPT_LEN for t in total), tuple(ENC_LENS),
+                    (0.4, 0.2, 0.6), "half", t_max=40)
+    corr = W.make_corruption(wl)
+    o.restore(snap)
+    seq = [list(prompt[b]) for b in range(3)]
+    steps = 0
+    while True:
+        draft, lens = W.make_drafts(truth, total, o.kv_len, wl.k, corr)
+        if np.all(lens < 0):
+            break
+        res = o.verify(draft, lens)
+        steps += 1
+        for b in range(3):
+            if lens[b] >= 0:
+                seq[b] += [int(t) for t in draft[b, :res.accepted[b]]] + [int(res.bonus[b])]
+    for b in range(3):
+        assert seq[b] == list(truth[b, :total[b]])
+    assert steps < max(total) - W.PROMPT_LEN      # drafts were accepted along the way
+
+
+def test_rollback_then_reverify_reproduces_cache():
+    o, *_ = _setup()
+    o.verify(np.array([[1, 2], [3, 4], [5, 6]]), np.array([2, 2, 2]))
+    snap = o.snapshot()
+    draft = np.array([[11, 12, 13], [14, 15, 16], [17, 18, 19]])
+    r1 = o.verify(draft, np.array([3, 1, 2]))
+    s1 = o.snapshot()
+    o.rollback(snap[2], snap[3])
+    r2 = o.verify(draft, np.array([3, 1, 2]))
+    s2 = o.snapshot()
+    for a, b in zip(r1.__dict__.values(), r2.__dict__.values()):
+        if isinstance(a, np.ndarray):
+            assert np.array_equal(a, b)
+    for l in range(TINY.n_layers):
+        assert np.array_equal(s1[0][l], s2[0][l]) and np.array_equal(s1[1][l], s2[1][l])
+    assert np.array_equal(s1[2], s2[2]) and np.array_equal(s1[3], s2[3])
+
+
+def test_special_cases():
+    o, *_ = _setup()
+    snap = o.snapshot()
+    g = _greedy_continuation(o, 5)
+    # no drafts == one greedy step
+    res = o.verify(np.zeros((3, 4), dtype=int), np.zeros(3, dtype=int))
+    assert list(res.bonus) == list(g[:, 0]) and list(res.accepted) == [0, 0, 0]
+    # true continuation: everything accepted, bonus is the next greedy token
+    o.restore(snap)
+    res = o.verify(g[:, :4], np.array([4, 4, 4]))
+    assert list(res.accepted) == [4, 4, 4] and list(res.bonus) == list(g[:, 4])
+    assert list(res.restart) == [0, 0, 0]
+    # every draft wrong at depth 1: nothing accepted
+    o.restore(snap)
+    wrong = (g[:, :4] + 1) % TINY.vocab
+    res = o.verify(wrong, np.array([4, 4, 4]))
+    assert list(res.accepted) == [0, 0, 0] and list(res.bonus) == list(g[:, 0])
+    assert list(res.restart) == [1, 1, 1]
+    # an inactive utterance keeps its state
+    o.restore(snap)
+    res = o.verify(g[:, :2], np.array([2, -1, 0]))
+    assert res.kv_len[1] == snap[2][1] and res.bonus[1] == -1 and res.anchor[1] == -1
+    assert res.accepted[0] == 2 and res.kv_len[0] == snap[2][0] + 3
+    assert res.kv_len[2] == snap[2][2] + 1
+
+
+def test_errors():
+    o, *_ = _setup()
+    with pytest.raises(OracleError):
+        o.verify(np.array([[1], [2], [TINY.vocab]]), np.array([1, 1, 1]))
+    with pytest.raises(OracleError):
+        o.verify(np.array([[1], [2], [3]]), np.array([2, 1, 1]))
+    with pytest.raises(OracleError):
+        o.rollback(o.kv_len + 1, o.pending)
+    o2 = Oracle(TINY, W.make_weights(TINY))
+    with pytest.raises(OracleError):
+        o2.prefill(np.zeros((1, 2), dtype=int))
+    # capacity: P + lens + 1 > max_pos
+    o.rollback(o.kv_len, o.pending)
+    o.kv_len[:] = TINY.max_pos - 2
+    with pytest.raises(OracleError):
+        o.verify(np.ones((3, 2), dtype=int), np.array([2, 0, 0]))
+
+
+def _mut_gelu_tanh(x):
+    return 0.5 * x * (1 + np.tanh(np.sqrt(2 / np.pi) * (x + 0.044715 * x ** 3)))
+
+
+def _mut_ln_unbiased(x, g, b):
+    mu = x.mean(axis=-1, keepdims=True)
+    var = x.var(axis=-1, ddof=1, keepdims=True)
+    return (x - mu) / np.sqrt(var + 1e-5) * g + b
+
+
+def _mut_attention_scale(q, K, V, n_heads):
+    import oracle.decoder as D
+    # scores scaled by 1/head_dim instead of 1/sqrt(head_dim)
+    return D.__dict__["_orig_attention"](q / np.sqrt(K.shape[1] // n_heads), K, V, n_heads)
+
+
+def _mut_head_mean_logits(q, K, n_heads):
+    import oracle.decoder as D
+    n, d = K.shape
+    hd = d // n_heads
+    s = np.einsum("hc,nhc->hn", q.reshape(n_heads, hd), K.reshape(n, n_heads, hd)) / np.sqrt(hd)
+    return D.softmax(s.mean(axis=0))
+
+
+@pytest.mark.parametrize("name,fn", [("gelu", _mut_gelu_tanh), ("layer_norm", _mut_ln_unbiased),
+                                     ("attention", _mut_attention_scale),
+                                     ("head_mean_attention", _mut_head_mean_logits)])
+def test_pins_catch_planted_mistakes(monkeypatch, name, fn):
+    """A plausible mistake planted in the oracle makes the library pins fail."""
+    import oracle.decoder as D
+    monkeypatch.setitem(D.__dict__, "_orig_attention", D.attention)
+    monkeypatch.setattr(D, name, fn)
+    with pytest.raises(AssertionError):
+        if name == "head_mean_attention":
+            test_anchor_matches_torch_head_mean_weights()
+        else:
+            test_verify_rows_match_torch_decoder(0.3)
