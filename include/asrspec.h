@@ -1,0 +1,191 @@
+/*
+ * asrspec.h - C ABI of the GB300 (sm_103a) draft-verify step for single-model
+ * speculative ASR decoding ("Alignment Drift in Single-Model Speculative
+ * Decoding for ASR: Mechanism, Correction, and Cost").
+ *
+ * The step (Sec. 3, "Speculative Loop"): a draft proposes up to K tokens per
+ * utterance; the frozen target scores the pending token and the K drafts in
+ * one decoder pass, accepts the longest prefix that matches its own greedy
+ * output and adds its next prediction (the "bonus" token, so a round advances
+ * 1 + L tokens, App. "Correction and Cost", cost derivation).  Accepted tokens
+ * and their cached states feed the next round (App. "Decoding and
+ * Intervention Protocol", real cached loop).  The runtime correction re-anchors
+ * the next draft round at the peak of the target's head-averaged audio
+ * attention at one decoder layer, recomputed from the existing key cache
+ * without another target pass (Sec. 5 "Verification-Attention Correction",
+ * App. "Runtime anchor construction").
+ *
+ * Model: a Whisper-style pre-LN decoder (Sec. 3 "Models and Protocol"):
+ * learned positional table, per layer LN -> causal self-attention (biases on
+ * q, v and the output; none on k) -> LN -> cross-attention to the encoder
+ * states -> LN -> MLP (erf GELU), final LN, LM head tied to the token
+ * embedding.  Head dimension 64.  LayerNorm eps 1e-5.
+ *
+ * Conventions
+ *  - All calls are asynchronous on the handle's CUDA stream unless host I/O
+ *    is enabled (asr_spec_set_host_io), in which case every call that takes
+ *    or returns arrays synchronises before it returns.
+ *  - Array arguments are device pointers by default; with host I/O enabled
+ *    they are host pointers (pinned or pageable) and the library copies them.
+ *  - The handle owns every device buffer it allocates (weights, caches,
+ *    activations).  The caller owns every argument buffer.
+ *  - Return value: ASR_OK (0) or a negative ASR_E_* code; the message is in
+ *    asr_spec_last_error.  Conditions that depend on device data (a token id
+ *    out of range, lens out of range, context capacity) are found by the
+ *    kernels, which then skip the step without changing any state and set the
+ *    device status word, read by asr_spec_status.  No kernel traps.
+ *  - Arithmetic: bf16 models keep weights, K/V caches and GEMM inputs in
+ *    bf16 and accumulate, normalise and run the residual stream in fp32;
+ *    fp32 models run everything in fp32 (no TF32).
+ */
+#ifndef ASRSPEC_H_
+#define ASRSPEC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ASR_OK 0
+#define ASR_E_INVAL (-1)     /* bad argument: dims, k > max_draft, B > max_batch, null pointer */
+#define ASR_E_STATE (-2)     /* call out of order: prefill before encode_cache, verify before prefill */
+#define ASR_E_CAPACITY (-3)  /* t_max > max_enc, P0 > max_pos */
+#define ASR_E_OOM (-4)       /* device allocation failed */
+#define ASR_E_CUDA (-5)      /* a CUDA runtime call failed */
+#define ASR_E_DEVICE (-6)    /* the device status word is set (see asr_spec_status) */
+
+/* Device status bits returned by asr_spec_status. */
+#define ASR_ST_BAD_TOKEN 1      /* a draft, prompt or rollback token outside [0, vocab) */
+#define ASR_ST_BAD_LENS 2       /* lens[b] outside [-1, k] */
+#define ASR_ST_CAPACITY 4       /* kv_len[b] + lens[b] + 1 > max_pos, or enc_len out of range */
+#define ASR_ST_WAIT_TIMEOUT 8   /* a bounded pipeline wait gave up; results of that call are invalid */
+#define ASR_ST_NOT_READY 16     /* an utterance slot without an encoder cache or prefill */
+
+typedef struct asr_spec* asr_spec_handle;
+
+typedef struct {
+  int32_t n_layers;     /* decoder layers L */
+  int32_t d_model;      /* d, a multiple of 64 */
+  int32_t n_heads;      /* H = d / 64 */
+  int32_t d_ffn;        /* MLP width, a multiple of 64 */
+  int32_t vocab;        /* V */
+  int32_t max_pos;      /* rows of the positional table = decoder context, e.g. 448 */
+  int32_t max_batch;    /* utterance slots B_max */
+  int32_t max_draft;    /* largest draft length k accepted by asr_spec_verify */
+  int32_t max_enc;      /* encoder frames per utterance, e.g. 1500 */
+  int32_t dtype;        /* 0 = fp32, 1 = bf16 */
+  int32_t anchor_layer; /* 0-based layer read by the re-anchoring readout; -1 = floor(3 L / 4) */
+} asr_model_dims;
+
+/* Host fp32 weights, one flat blob in this order (matrices [out][in], row-major):
+ *   tok_emb [V][d], pos_emb [max_pos][d],
+ *   per layer: ln1_g[d] ln1_b[d] wq[d][d] bq[d] wk[d][d] wv[d][d] bv[d] wo[d][d] bo[d]
+ *              ln2_g ln2_b wcq[d][d] bcq[d] wck[d][d] wcv[d][d] bcv[d] wco[d][d] bco[d]
+ *              ln3_g ln3_b w1[F][d] b1[F] w2[d][F] b2[d]
+ *   lnf_g[d], lnf_b[d].
+ * bf16 models round each value to bf16 (nearest, ties to even) on upload. */
+typedef struct {
+  const float* blob;
+  size_t n_floats;
+} asr_weights;
+
+/* Create a handle: validate dims, allocate device weights, caches and
+ * work buffers, upload the weights.  stream: a cudaStream_t (NULL = the
+ * legacy default stream) on which every later call is ordered.  Synchronous.
+ * Errors: ASR_E_INVAL (dims), ASR_E_OOM, ASR_E_CUDA. */
+int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void* stream,
+                    asr_spec_handle* out);
+
+/* Select host (1) or device (0, default) pointers for array arguments. */
+int asr_spec_set_host_io(asr_spec_handle h, int host_io);
+
+/* Build the cross-attention K/V cache of every layer for B utterances, once per
+ * utterance (the encoded audio is reused by every verification step, Sec. 1 and
+ * App. "Runtime anchor construction"): Kx_l = E Wck_l^T, Vx_l = E Wcv_l^T + bcv_l.
+ *   enc_states: [B][t_max][d] in the model dtype (fp32 or bf16); always a device
+ *               pointer; frames t >= enc_lens[b] are ignored.
+ *   enc_lens:   [B] int32, 1 <= enc_lens[b] <= t_max.
+ * Occupies slots 0..B-1 and clears their decoder state (call asr_spec_prefill next).
+ * Errors: ASR_E_INVAL (B, pointers), ASR_E_CAPACITY (t_max > max_enc). */
+int asr_spec_encode_cache(asr_spec_handle h, int32_t B, const void* enc_states, int32_t t_max,
+                          const int32_t* enc_lens);
+
+/* Cache a prompt of P0 tokens per utterance: K/V of prompt[b][0..P0-2] at
+ * positions 0..P0-2; prompt[b][P0-1] becomes the pending token, scored by the
+ * next verify at position P0-1.  prompt: [B][P0] int32.
+ * Errors: ASR_E_STATE (no encoder cache), ASR_E_CAPACITY (P0 > max_pos). */
+int asr_spec_prefill(asr_spec_handle h, const int32_t* prompt, int32_t P0);
+
+/* One verification round (Sec. 3 "Speculative Loop").
+ *   draft [B][k] int32: proposed tokens; entries past lens[b] are ignored.
+ *   lens  [B] int32: valid drafts 0..k, or -1 for an utterance that sits out.
+ * Row i of utterance b is the pending token (i = 0) or draft i, at position
+ * kv_len[b] + i; it attends to the committed cache and to rows 0..i of its own
+ * block.  With g_i the argmax of row i (lowest id on ties):
+ *   accepted[b] = n = the largest n <= lens[b] with draft[b][j-1] == g_{j-1} for all j <= n
+ *   bonus[b]    = g_n;  the new kv_len[b] = old kv_len[b] + 1 + n; pending = bonus
+ *   anchor[b]   = argmax over frames j < enc_len[b] of the head mean of the
+ *                 per-head softmax attention of row n at the anchor layer
+ *                 (lowest frame on ties).
+ * Sitting-out utterances return accepted 0, bonus -1, anchor -1, kv_len unchanged.
+ * Outputs are [B] int32 each.
+ * Errors: ASR_E_INVAL (k outside [0, max_draft]), ASR_E_STATE (no prefill).
+ * Data errors (token id, lens, capacity) skip the whole step and set the
+ * status word. */
+int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens, int32_t k,
+                    int32_t* accepted, int32_t* bonus, int32_t* kv_len, int32_t* anchor);
+
+/* Roll the committed cache back (App. "Decoding and Intervention Protocol":
+ * the cached states of accepted tokens are what the next round reuses):
+ * kv_len[b] <- new_len[b] (which must not exceed the current kv_len[b]) and
+ * pending[b] <- new_pending[b].  Cache rows at and beyond new_len are dead.
+ * new_len[b] = -1 leaves utterance b unchanged.  Both [B] int32.
+ * Invalid values set the status word and change nothing. */
+int asr_spec_rollback(asr_spec_handle h, const int32_t* new_len, const int32_t* new_pending);
+
+/* Read the committed lengths and pending tokens: [B] int32 each. */
+int asr_spec_state(asr_spec_handle h, int32_t* kv_len, int32_t* pending);
+
+/* Test support: the LM-head logits of every row scored by the last verify,
+ * recomputed from its final-LN rows with the same tensor-core arithmetic as the
+ * fused argmax.  out: [R][V] fp32 with R = the number of rows of that call
+ * (sum over active b of lens[b] + 1, in utterance order); returns R (>= 0) or
+ * an error. */
+int asr_spec_debug_logits(asr_spec_handle h, float* out, int32_t max_rows);
+
+/* Synchronise the stream, then return and clear the device status word
+ * (ASR_ST_* bits; 0 = clean).  Negative on a CUDA error. */
+int asr_spec_status(asr_spec_handle h);
+
+/* Message of the last error on this handle (static storage of the handle). */
+const char* asr_spec_last_error(asr_spec_handle h);
+
+/* Free every device buffer of the handle.  NULL is a no-op. */
+void asr_spec_destroy(asr_spec_handle h);
+
+/* ---- Workload utility (not part of the paper's method) -------------------
+ * Synthetic draft source used by benchmarks in place of a trained draft
+ * model: draft i (1-based) of a round at committed length P is
+ * truth[b][P+i] (or truth[b][P+i-1] when shift[b][P] = s > 0 and i >= s),
+ * replaced by repl[b][P][i-1] when that is >= 0.  lens[b] = -1 once
+ * P + 1 >= total_len[b], else min(k, total_len[b] - P - 2).
+ *   truth [B][max_pos], total_len [B], repl [B][max_pos][k_repl], shift [B][max_pos];
+ *   draft_out [B][k], lens_out [B].  Device pointers only. */
+int asr_spec_synth_drafts(asr_spec_handle h, const int32_t* truth, const int32_t* total_len,
+                          const int32_t* repl, int32_t k_repl, const int32_t* shift, int32_t k,
+                          int32_t* draft_out, int32_t* lens_out);
+
+/* ---- Kernel test entry (not part of the paper's method) ------------------
+ * C[m][n] = sum_k A[m][k] * B[n][k] through the tcgen05 tensor-core GEMM
+ * (impl 0) or the SIMT GEMM (impl 1); A, B bf16 row-major device arrays,
+ * C fp32.  K % 64 == 0.  Synchronous. */
+int asr_spec_test_gemm(int32_t impl, const void* A, const void* B, float* C, int32_t M, int32_t N,
+                       int32_t K, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ASRSPEC_H_ */

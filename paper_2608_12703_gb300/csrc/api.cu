@@ -1,0 +1,669 @@
+// C ABI of the draft-verify step: handle, weights upload, per-utterance
+// encoder cache, prefill, verify, rollback.  See include/asrspec.h.
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "kernels.h"
+
+using namespace asrspec;
+
+namespace {
+
+constexpr int NUM_SMS_TARGET = 152;
+
+struct LayerW {
+  void *wqkv, *wo, *wcq, *wco, *w1, *w2;
+  float *bqkv, *bo, *bcq, *bco, *b1, *b2;
+  float *ln1g, *ln1b, *ln2g, *ln2b, *ln3g, *ln3b;
+  CUtensorMap m_wqkv, m_wo, m_wcq, m_wco, m_w1, m_w2;
+};
+
+}  // namespace
+
+struct asr_spec {
+  asr_model_dims dims{};
+  int L = 0, d = 0, H = 0, F = 0, V = 0, maxpos = 0, Bmax = 0, kmax = 0, Tmax = 0, anchor = 0;
+  bool bf16 = true;
+  size_t es = 2;  // element size of weights / caches / GEMM inputs
+  cudaStream_t st = nullptr;
+  int host_io = 0;
+  int state = 0;  // 0 created, 1 encoder cache built, 2 prefilled
+  int B = 0, t_max = 0;
+  std::string err;
+
+  std::vector<void*> allocs;
+  void *w_tok = nullptr, *w_pos = nullptr, *w_cross = nullptr;
+  float *b_cross = nullptr, *lnf_g = nullptr, *lnf_b = nullptr;
+  CUtensorMap m_tok{};
+  std::vector<LayerW> lw;
+
+  void *kself = nullptr, *vself = nullptr, *xkv = nullptr;
+  int *enc_len = nullptr, *kv_len = nullptr, *pending = nullptr, *ready = nullptr;
+
+  int R_max = 0, R_pad = 0;
+  float *x = nullptr, *q = nullptr, *q_anchor = nullptr, *ml = nullptr, *part = nullptr;
+  void *xn = nullptr, *att = nullptr, *hbuf = nullptr, *xf = nullptr;
+  RowPlan plan{};
+  unsigned long long* row_key = nullptr;
+  unsigned long long* frame_key = nullptr;  // [Bmax] keys + [Bmax] int tickets
+  int* anchor_row = nullptr;
+  int *draft_buf = nullptr, *lens_buf = nullptr, *prompt_buf = nullptr, *out4 = nullptr, *misc = nullptr;
+  int* status = nullptr;
+  float* ws = nullptr;
+  size_t ws_floats = 0;
+  int* tickets = nullptr;
+  int n_tickets = 0;
+  std::map<std::pair<int, int>, CUtensorMap> bmaps;  // (buffer id, BN) -> map
+};
+
+namespace {
+
+int fail(asr_spec* h, int code, const std::string& msg) {
+  if (h) h->err = msg;
+  return code;
+}
+
+#define CK(call)                                                                       \
+  do {                                                                                 \
+    cudaError_t e_ = (call);                                                           \
+    if (e_ != cudaSuccess) return fail(h, ASR_E_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+template <typename T>
+int dalloc(asr_spec* h, T** p, size_t bytes) {
+  void* v = nullptr;
+  if (cudaMalloc(&v, bytes) != cudaSuccess) return fail(h, ASR_E_OOM, "cudaMalloc failed");
+  h->allocs.push_back(v);
+  *p = static_cast<T*>(v);
+  return 0;
+}
+
+// Round fp32 -> bf16 (nearest, ties to even), host side.
+uint16_t f2bf_host(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7fffffffu) > 0x7f800000u) return 0x7fc0;
+  u += 0x7fffu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+
+// Upload `n` consecutive fp32 values as the model's storage type.
+int upload(asr_spec* h, void* dst, const float* src, size_t n) {
+  if (!h->bf16) {
+    CK(cudaMemcpy(dst, src, n * 4, cudaMemcpyHostToDevice));
+    return 0;
+  }
+  std::vector<uint16_t> tmp(n);
+  for (size_t i = 0; i < n; ++i) tmp[i] = f2bf_host(src[i]);
+  CK(cudaMemcpy(dst, tmp.data(), n * 2, cudaMemcpyHostToDevice));
+  return 0;
+}
+int upload_f32(asr_spec* h, float* dst, const float* src, size_t n) {
+  CK(cudaMemcpy(dst, src, n * 4, cudaMemcpyHostToDevice));
+  return 0;
+}
+
+const CUtensorMap* bmap(asr_spec* h, int id, const void* buf, int rows, int cols, int bn) {
+  auto key = std::make_pair(id, bn);
+  auto it = h->bmaps.find(key);
+  if (it != h->bmaps.end()) return &it->second;
+  CUtensorMap m;
+  if (!make_tmap_bf16(&m, buf, rows, cols, bn)) return nullptr;
+  return &(h->bmaps[key] = m);
+}
+
+int pick_splits(int tiles, int nkb) {
+  int s = (2 * NUM_SMS_TARGET + tiles / 2) / std::max(tiles, 1);
+  s = std::max(1, std::min(s, nkb / 2));
+  return s;
+}
+
+// One projection over the verify rows: out-features m (weights = A), rows n (activations = B).
+int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, const void* X, int x_id, int N,
+              int mode, const Epi& epi_in) {
+  Epi epi = epi_in;
+  epi.M = M;
+  epi.N = N;
+  if (!h->bf16) {
+    launch_gemm_simt(W, 0, X, 0, M, N, K, mode, epi, h->st);
+    return 0;
+  }
+  TcGemm g{};
+  g.mapA = *mW;
+  g.bn = tc_pick_bn(N);
+  const CUtensorMap* mb = bmap(h, x_id, X, h->R_pad, K, g.bn);
+  if (!mb) return fail(h, ASR_E_CUDA, "tensor map encode failed");
+  g.mapB = *mb;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  const int tiles = ((M + 127) / 128) * ((N + g.bn - 1) / g.bn);
+  g.splits = mode == EPI_ARGMAX || mode == EPI_F32 ? 1 : pick_splits(tiles, K / 64);
+  while (g.splits > 1 && (size_t)g.splits * tiles * 128 * g.bn > h->ws_floats) --g.splits;
+  if (tiles > h->n_tickets && g.splits > 1) g.splits = 1;
+  g.ws = h->ws;
+  g.tickets = h->tickets;
+  launch_gemm_tc(g, mode, epi, h->status, h->st);
+  return 0;
+}
+
+enum BufId { BUF_XN = 1, BUF_ATT = 2, BUF_H = 3, BUF_XF = 4 };
+
+// The decoder layers over the rows laid out by the last plan kernel.
+int run_layers(asr_spec* h, int N) {
+  const int d = h->d;
+  Epi base{};
+  base.n_valid = h->plan.n_rows;
+  base.d = d;
+  base.row_b = h->plan.row_b;
+  base.row_pos = h->plan.row_pos;
+  base.kv_bf16 = h->bf16;
+  base.act_bf16 = h->bf16;
+  base.max_pos = h->maxpos;
+  base.n_heads = h->H;
+  const size_t self_layer = (size_t)h->Bmax * h->H * h->maxpos * 64 * h->es;
+  const size_t cross_half = (size_t)h->Bmax * h->H * h->Tmax * 64 * h->es;
+  launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st);
+  for (int l = 0; l < h->L; ++l) {
+    LayerW& w = h->lw[l];
+    char* ks = static_cast<char*>(h->kself) + l * self_layer;
+    char* vs = static_cast<char*>(h->vself) + l * self_layer;
+    char* kx = static_cast<char*>(h->xkv) + (size_t)l * 2 * cross_half;
+    char* vx = kx + cross_half;
+    // self-attention block
+    launch_layernorm(h->x, w.ln1g, w.ln1b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+    Epi e = base;
+    e.bias = w.bqkv;
+    e.out_f32 = h->q;
+    e.kcache = ks;
+    e.vcache = vs;
+    if (int rc = gemm_rows(h, w.wqkv, &w.m_wqkv, 3 * d, d, h->xn, BUF_XN, N, EPI_QKV, e)) return rc;
+    AttnArgs a{};
+    a.q = h->q;
+    a.kc = ks;
+    a.vc = vs;
+    a.kv_bf16 = h->bf16;
+    a.t_alloc = h->maxpos;
+    a.causal = 1;
+    a.enc_len = h->enc_len;
+    a.kv_len = h->kv_len;
+    a.plan = h->plan;
+    a.B = h->B;
+    a.H = h->H;
+    a.d = d;
+    a.k1 = h->kmax + 1;
+    a.chunk = attn_chunk_len(h->bf16);
+    a.n_chunks = (h->maxpos + a.chunk - 1) / a.chunk;
+    a.part = h->part;
+    a.out = h->att;
+    a.out_bf16 = h->bf16;
+    a.ml_out = nullptr;
+    launch_attention(a, h->st);
+    e = base;
+    e.bias = w.bo;
+    e.x = h->x;
+    if (int rc = gemm_rows(h, w.wo, &w.m_wo, d, d, h->att, BUF_ATT, N, EPI_RESID, e)) return rc;
+    // cross-attention block
+    launch_layernorm(h->x, w.ln2g, w.ln2b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+    float* qc = (l == h->anchor) ? h->q_anchor : h->q;
+    e = base;
+    e.bias = w.bcq;
+    e.out_f32 = qc;
+    if (int rc = gemm_rows(h, w.wcq, &w.m_wcq, d, d, h->xn, BUF_XN, N, EPI_Q, e)) return rc;
+    a.q = qc;
+    a.kc = kx;
+    a.vc = vx;
+    a.t_alloc = h->Tmax;
+    a.causal = 0;
+    a.n_chunks = (h->Tmax + a.chunk - 1) / a.chunk;
+    a.ml_out = (l == h->anchor) ? h->ml : nullptr;
+    launch_attention(a, h->st);
+    e = base;
+    e.bias = w.bco;
+    e.x = h->x;
+    if (int rc = gemm_rows(h, w.wco, &w.m_wco, d, d, h->att, BUF_ATT, N, EPI_RESID, e)) return rc;
+    // MLP block
+    launch_layernorm(h->x, w.ln3g, w.ln3b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+    e = base;
+    e.bias = w.b1;
+    e.act = h->hbuf;
+    if (int rc = gemm_rows(h, w.w1, &w.m_w1, h->F, d, h->xn, BUF_XN, N, EPI_GELU, e)) return rc;
+    e = base;
+    e.bias = w.b2;
+    e.x = h->x;
+    if (int rc = gemm_rows(h, w.w2, &w.m_w2, d, h->F, h->hbuf, BUF_H, N, EPI_RESID, e)) return rc;
+  }
+  return 0;
+}
+
+bool dims_ok(const asr_model_dims& m) {
+  return m.n_layers >= 1 && m.d_model >= 64 && m.d_model % 64 == 0 && m.d_model <= 2048 &&
+         m.n_heads * 64 == m.d_model && m.d_ffn >= 64 && m.d_ffn % 64 == 0 && m.vocab >= 2 && m.max_pos >= 2 &&
+         m.max_batch >= 1 && m.max_batch <= 1024 && m.max_draft >= 0 && m.max_draft <= 31 && m.max_enc >= 1 &&
+         (m.dtype == 0 || m.dtype == 1) && m.anchor_layer >= -1 && m.anchor_layer < m.n_layers;
+}
+
+int copy_in(asr_spec* h, int* dst, const int32_t* src, size_t n) {
+  CK(cudaMemcpyAsync(dst, src, n * 4, h->host_io ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToDevice, h->st));
+  return 0;
+}
+int copy_out(asr_spec* h, int32_t* dst, const int* src, size_t n) {
+  CK(cudaMemcpyAsync(dst, src, n * 4, h->host_io ? cudaMemcpyDeviceToHost : cudaMemcpyDeviceToDevice, h->st));
+  return 0;
+}
+
+}  // namespace
+
+extern "C" {
+
+int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void* stream, asr_spec_handle* out) {
+  if (!dims || !weights || !weights->blob || !out) return ASR_E_INVAL;
+  *out = nullptr;
+  if (!dims_ok(*dims)) return ASR_E_INVAL;
+  asr_spec* h = new asr_spec();
+  h->dims = *dims;
+  h->L = dims->n_layers;
+  h->d = dims->d_model;
+  h->H = dims->n_heads;
+  h->F = dims->d_ffn;
+  h->V = dims->vocab;
+  h->maxpos = dims->max_pos;
+  h->Bmax = dims->max_batch;
+  h->kmax = dims->max_draft;
+  h->Tmax = dims->max_enc;
+  h->anchor = dims->anchor_layer >= 0 ? dims->anchor_layer : (3 * h->L) / 4;
+  h->bf16 = dims->dtype == 1;
+  h->es = h->bf16 ? 2 : 4;
+  h->st = static_cast<cudaStream_t>(stream);
+  const int d = h->d, F = h->F, L = h->L;
+  const size_t per_layer = 8 * (size_t)d * d + 13 * (size_t)d + 2 * (size_t)F * d + F;
+  const size_t expect = (size_t)h->V * d + (size_t)h->maxpos * d + L * per_layer + 2 * (size_t)d;
+  if (weights->n_floats != expect) {
+    delete h;
+    return ASR_E_INVAL;
+  }
+  int rc = 0;
+  auto finish = [&](int code) {
+    if (code) asr_spec_destroy(h);
+    else *out = h;
+    return code;
+  };
+  const float* src = weights->blob;
+  size_t off = 0;
+  auto take = [&](size_t n) {
+    const float* p = src + off;
+    off += n;
+    return p;
+  };
+  const size_t es = h->es;
+  if ((rc = dalloc(h, &h->w_tok, (size_t)h->V * d * es))) return finish(rc);
+  if ((rc = upload(h, h->w_tok, take((size_t)h->V * d), (size_t)h->V * d))) return finish(rc);
+  if ((rc = dalloc(h, &h->w_pos, (size_t)h->maxpos * d * es))) return finish(rc);
+  if ((rc = upload(h, h->w_pos, take((size_t)h->maxpos * d), (size_t)h->maxpos * d))) return finish(rc);
+  if ((rc = dalloc(h, &h->w_cross, (size_t)L * 2 * d * d * es))) return finish(rc);
+  if ((rc = dalloc(h, &h->b_cross, (size_t)L * 2 * d * 4))) return finish(rc);
+  h->lw.resize(L);
+  std::vector<float> tmp;
+  for (int l = 0; l < L; ++l) {
+    LayerW& w = h->lw[l];
+    auto vec = [&](float** dst, size_t n, const float* s) {
+      int r = dalloc(h, dst, n * 4);
+      if (!r) r = upload_f32(h, *dst, s, n);
+      return r;
+    };
+    auto mat = [&](void** dst, size_t n, const float* s) {
+      int r = dalloc(h, dst, n * es);
+      if (!r) r = upload(h, *dst, s, n);
+      return r;
+    };
+    const float* ln1g = take(d);
+    const float* ln1b = take(d);
+    const float* wq = take((size_t)d * d);
+    const float* bq = take(d);
+    const float* wk = take((size_t)d * d);
+    const float* wv = take((size_t)d * d);
+    const float* bv = take(d);
+    const float* wo = take((size_t)d * d);
+    const float* bo = take(d);
+    const float* ln2g = take(d);
+    const float* ln2b = take(d);
+    const float* wcq = take((size_t)d * d);
+    const float* bcq = take(d);
+    const float* wck = take((size_t)d * d);
+    const float* wcv = take((size_t)d * d);
+    const float* bcv = take(d);
+    const float* wco = take((size_t)d * d);
+    const float* bco = take(d);
+    const float* ln3g = take(d);
+    const float* ln3b = take(d);
+    const float* w1 = take((size_t)F * d);
+    const float* b1 = take(F);
+    const float* w2 = take((size_t)d * F);
+    const float* b2 = take(d);
+    // fused [q; k; v] projection, no key bias
+    tmp.assign((size_t)3 * d * d, 0.f);
+    std::memcpy(tmp.data(), wq, (size_t)d * d * 4);
+    std::memcpy(tmp.data() + (size_t)d * d, wk, (size_t)d * d * 4);
+    std::memcpy(tmp.data() + (size_t)2 * d * d, wv, (size_t)d * d * 4);
+    if ((rc = mat(&w.wqkv, (size_t)3 * d * d, tmp.data()))) return finish(rc);
+    std::vector<float> bqkv(3 * d, 0.f);
+    std::memcpy(bqkv.data(), bq, d * 4);
+    std::memcpy(bqkv.data() + 2 * d, bv, d * 4);
+    if ((rc = vec(&w.bqkv, 3 * d, bqkv.data()))) return finish(rc);
+    if ((rc = mat(&w.wo, (size_t)d * d, wo)) || (rc = vec(&w.bo, d, bo))) return finish(rc);
+    if ((rc = mat(&w.wcq, (size_t)d * d, wcq)) || (rc = vec(&w.bcq, d, bcq))) return finish(rc);
+    if ((rc = mat(&w.wco, (size_t)d * d, wco)) || (rc = vec(&w.bco, d, bco))) return finish(rc);
+    if ((rc = mat(&w.w1, (size_t)F * d, w1)) || (rc = vec(&w.b1, F, b1))) return finish(rc);
+    if ((rc = mat(&w.w2, (size_t)d * F, w2)) || (rc = vec(&w.b2, d, b2))) return finish(rc);
+    if ((rc = vec(&w.ln1g, d, ln1g)) || (rc = vec(&w.ln1b, d, ln1b)) || (rc = vec(&w.ln2g, d, ln2g)) ||
+        (rc = vec(&w.ln2b, d, ln2b)) || (rc = vec(&w.ln3g, d, ln3g)) || (rc = vec(&w.ln3b, d, ln3b)))
+      return finish(rc);
+    // cross K/V projection of this layer: rows [k; v] of the stacked all-layer matrix
+    char* wc = static_cast<char*>(h->w_cross) + (size_t)l * 2 * d * d * es;
+    if ((rc = upload(h, wc, wck, (size_t)d * d))) return finish(rc);
+    if ((rc = upload(h, wc + (size_t)d * d * es, wcv, (size_t)d * d))) return finish(rc);
+    std::vector<float> bc(2 * d, 0.f);
+    std::memcpy(bc.data() + d, bcv, d * 4);
+    if ((rc = upload_f32(h, h->b_cross + (size_t)l * 2 * d, bc.data(), 2 * d))) return finish(rc);
+    if (h->bf16) {
+      bool ok = make_tmap_bf16(&w.m_wqkv, w.wqkv, 3 * d, d, 128) && make_tmap_bf16(&w.m_wo, w.wo, d, d, 128) &&
+                make_tmap_bf16(&w.m_wcq, w.wcq, d, d, 128) && make_tmap_bf16(&w.m_wco, w.wco, d, d, 128) &&
+                make_tmap_bf16(&w.m_w1, w.w1, F, d, 128) && make_tmap_bf16(&w.m_w2, w.w2, d, F, 128);
+      if (!ok) return finish(fail(h, ASR_E_CUDA, "tensor map encode failed"));
+    }
+  }
+  const float* lnfg = take(d);
+  const float* lnfb = take(d);
+  if ((rc = dalloc(h, &h->lnf_g, d * 4)) || (rc = upload_f32(h, h->lnf_g, lnfg, d))) return finish(rc);
+  if ((rc = dalloc(h, &h->lnf_b, d * 4)) || (rc = upload_f32(h, h->lnf_b, lnfb, d))) return finish(rc);
+  if (h->bf16 && !make_tmap_bf16(&h->m_tok, h->w_tok, h->V, d, 128))
+    return finish(fail(h, ASR_E_CUDA, "tensor map encode failed"));
+
+  // caches
+  const size_t self_bytes = (size_t)L * h->Bmax * h->H * h->maxpos * 64 * es;
+  const size_t cross_bytes = (size_t)L * 2 * h->Bmax * h->H * h->Tmax * 64 * es;
+  if ((rc = dalloc(h, &h->kself, self_bytes)) || (rc = dalloc(h, &h->vself, self_bytes)) ||
+      (rc = dalloc(h, &h->xkv, cross_bytes)))
+    return finish(rc);
+  if ((rc = dalloc(h, &h->enc_len, h->Bmax * 4)) || (rc = dalloc(h, &h->kv_len, h->Bmax * 4)) ||
+      (rc = dalloc(h, &h->pending, h->Bmax * 4)) || (rc = dalloc(h, &h->ready, h->Bmax * 4)))
+    return finish(rc);
+  CK(cudaMemset(h->ready, 0, h->Bmax * 4));
+  CK(cudaMemset(h->kv_len, 0, h->Bmax * 4));
+  CK(cudaMemset(h->pending, 0, h->Bmax * 4));
+  CK(cudaMemset(h->enc_len, 0, h->Bmax * 4));
+
+  // work buffers
+  h->R_max = h->Bmax * (h->kmax + 1);
+  h->R_pad = ((h->R_max + 255) / 256) * 256;
+  const size_t R = h->R_pad;
+  if ((rc = dalloc(h, &h->x, R * d * 4)) || (rc = dalloc(h, &h->q, R * d * 4)) ||
+      (rc = dalloc(h, &h->q_anchor, R * d * 4)) || (rc = dalloc(h, &h->ml, R * h->H * 2 * 4)) ||
+      (rc = dalloc(h, &h->xn, R * d * es)) || (rc = dalloc(h, &h->att, R * d * es)) ||
+      (rc = dalloc(h, &h->hbuf, R * F * es)) || (rc = dalloc(h, &h->xf, R * d * es)))
+    return finish(rc);
+  CK(cudaMemset(h->xn, 0, R * d * es));
+  CK(cudaMemset(h->att, 0, R * d * es));
+  CK(cudaMemset(h->hbuf, 0, R * F * es));
+  CK(cudaMemset(h->xf, 0, R * d * es));
+  const int chunk = attn_chunk_len(h->bf16);
+  const int n_chunks = (std::max(h->maxpos, h->Tmax) + chunk - 1) / chunk;
+  if ((rc = dalloc(h, &h->part, (size_t)h->Bmax * h->H * n_chunks * (h->kmax + 1) * 66 * 4))) return finish(rc);
+  if ((rc = dalloc(h, &h->plan.row_b, R * 4)) || (rc = dalloc(h, &h->plan.row_i, R * 4)) ||
+      (rc = dalloc(h, &h->plan.row_pos, R * 4)) || (rc = dalloc(h, &h->plan.row_tok, R * 4)) ||
+      (rc = dalloc(h, &h->plan.row_start, (h->Bmax + 1) * 4)) || (rc = dalloc(h, &h->plan.n_rows, 4)) ||
+      (rc = dalloc(h, &h->plan.n_utt_rows, h->Bmax * 4)))
+    return finish(rc);
+  CK(cudaMemset(h->plan.n_rows, 0, 4));
+  if ((rc = dalloc(h, &h->row_key, R * 8)) || (rc = dalloc(h, &h->frame_key, h->Bmax * 12)) ||
+      (rc = dalloc(h, &h->anchor_row, h->Bmax * 4)))
+    return finish(rc);
+  CK(cudaMemset(h->frame_key, 0, h->Bmax * 12));
+  if ((rc = dalloc(h, &h->draft_buf, (size_t)h->Bmax * std::max(h->kmax, 1) * 4)) ||
+      (rc = dalloc(h, &h->lens_buf, h->Bmax * 4)) || (rc = dalloc(h, &h->prompt_buf, (size_t)h->Bmax * h->maxpos * 4)) ||
+      (rc = dalloc(h, &h->out4, 4 * h->Bmax * 4)) || (rc = dalloc(h, &h->misc, 64 * 4)) ||
+      (rc = dalloc(h, &h->status, 4)))
+    return finish(rc);
+  CK(cudaMemset(h->status, 0, 4));
+  h->ws_floats = (size_t)16 << 20;  // 64 MB of split-K partials
+  h->n_tickets = 8192;
+  if ((rc = dalloc(h, &h->ws, h->ws_floats * 4)) || (rc = dalloc(h, &h->tickets, h->n_tickets * 4))) return finish(rc);
+  CK(cudaMemset(h->tickets, 0, h->n_tickets * 4));
+  CK(cudaDeviceSynchronize());
+  return finish(0);
+}
+
+int asr_spec_set_host_io(asr_spec_handle h, int host_io) {
+  if (!h) return ASR_E_INVAL;
+  h->host_io = host_io ? 1 : 0;
+  return ASR_OK;
+}
+
+int asr_spec_encode_cache(asr_spec_handle h, int32_t B, const void* enc_states, int32_t t_max,
+                          const int32_t* enc_lens) {
+  if (!h) return ASR_E_INVAL;
+  if (B < 1 || B > h->Bmax || !enc_states || !enc_lens || t_max < 1) return fail(h, ASR_E_INVAL, "bad arguments");
+  if (t_max > h->Tmax) return fail(h, ASR_E_CAPACITY, "t_max exceeds max_enc");
+  if (int rc = copy_in(h, h->enc_len, enc_lens, B)) return rc;
+  launch_mark_ready(h->enc_len, B, t_max, h->ready, h->kv_len, h->pending, h->status, h->st);
+  const int d = h->d;
+  Epi e{};
+  e.bias = h->b_cross;
+  e.d = d;
+  e.kcache = h->xkv;
+  e.kv_bf16 = h->bf16;
+  e.n_heads = h->H;
+  e.enc_len = h->enc_len;
+  e.t_max = t_max;
+  e.max_enc = h->Tmax;
+  e.b_max = h->Bmax;
+  const int M = B * t_max, N = h->L * 2 * d;
+  e.M = M;
+  e.N = N;
+  if (h->bf16) {
+    TcGemm g{};
+    if (!make_tmap_bf16(&g.mapA, enc_states, M, d, 128) || !make_tmap_bf16(&g.mapB, h->w_cross, N, d, 256))
+      return fail(h, ASR_E_INVAL, "encoder states must be 16-byte aligned");
+    g.M = M;
+    g.N = N;
+    g.K = d;
+    g.bn = 256;
+    g.splits = 1;
+    g.ws = h->ws;
+    g.tickets = h->tickets;
+    launch_gemm_tc(g, EPI_CROSSKV, e, h->status, h->st);
+  } else {
+    launch_gemm_simt(enc_states, 0, h->w_cross, 0, M, N, d, EPI_CROSSKV, e, h->st);
+  }
+  CK(cudaGetLastError());
+  h->B = B;
+  h->t_max = t_max;
+  h->state = 1;
+  if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
+}
+
+int asr_spec_prefill(asr_spec_handle h, const int32_t* prompt, int32_t P0) {
+  if (!h) return ASR_E_INVAL;
+  if (h->state < 1) return fail(h, ASR_E_STATE, "prefill before encode_cache");
+  if (!prompt || P0 < 1) return fail(h, ASR_E_INVAL, "bad arguments");
+  if (P0 > h->maxpos) return fail(h, ASR_E_CAPACITY, "prompt longer than max_pos");
+  if (int rc = copy_in(h, h->prompt_buf, prompt, (size_t)h->B * P0)) return rc;
+  const int c_max = h->kmax + 1;
+  for (int p0 = 0; p0 < P0 - 1; p0 += c_max) {
+    const int c = std::min(c_max, P0 - 1 - p0);
+    launch_plan_prefill_chunk(h->prompt_buf, P0, p0, c, h->B, h->V, h->ready, h->plan, h->status, h->st);
+    if (int rc = run_layers(h, h->B * c)) return rc;
+    launch_prefill_advance(h->B, c, h->plan.n_utt_rows, h->kv_len, h->st);
+  }
+  launch_prefill_finish(h->prompt_buf, P0, h->B, h->pending, h->ready, h->st);
+  CK(cudaGetLastError());
+  h->state = 2;
+  if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
+}
+
+int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens, int32_t k, int32_t* accepted,
+                    int32_t* bonus, int32_t* kv_len, int32_t* anchor) {
+  if (!h) return ASR_E_INVAL;
+  if (h->state < 2) return fail(h, ASR_E_STATE, "verify before prefill");
+  if (k < 0 || k > h->kmax) return fail(h, ASR_E_INVAL, "k outside [0, max_draft]");
+  if (!lens || (k > 0 && !draft) || !accepted || !bonus || !kv_len || !anchor)
+    return fail(h, ASR_E_INVAL, "null pointer");
+  const int B = h->B;
+  if (k > 0) {
+    if (int rc = copy_in(h, h->draft_buf, draft, (size_t)B * k)) return rc;
+  }
+  if (int rc = copy_in(h, h->lens_buf, lens, B)) return rc;
+  launch_plan_verify(h->draft_buf, h->lens_buf, k, B, h->V, h->maxpos, h->kv_len, h->pending, h->ready, h->plan,
+                     h->row_key, h->status, h->st);
+  const int N = B * (k + 1);
+  if (int rc = run_layers(h, N)) return rc;
+  launch_layernorm(h->x, h->lnf_g, h->lnf_b, h->xf, h->bf16, h->plan.n_rows, N, h->d, h->st);
+  Epi e{};
+  e.n_valid = h->plan.n_rows;
+  e.row_key = h->row_key;
+  e.d = h->d;
+  if (int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, N, EPI_ARGMAX, e)) return rc;
+  int* o_acc = h->out4;
+  int* o_bonus = h->out4 + h->Bmax;
+  int* o_len = h->out4 + 2 * h->Bmax;
+  int* o_anchor = h->out4 + 3 * h->Bmax;
+  launch_accept(h->draft_buf, h->lens_buf, k, B, h->plan, h->row_key, h->kv_len, h->pending, o_acc, o_bonus, o_len,
+                h->anchor_row, o_anchor, h->st);
+  const size_t cross_half = (size_t)h->Bmax * h->H * h->Tmax * 64 * h->es;
+  const char* kx = static_cast<const char*>(h->xkv) + (size_t)h->anchor * 2 * cross_half;
+  launch_anchor(h->q_anchor, h->ml, kx, h->bf16, h->Tmax, h->enc_len, h->anchor_row, B, h->H, h->d, h->frame_key,
+                reinterpret_cast<int*>(h->frame_key + h->Bmax), o_anchor, h->st);
+  CK(cudaGetLastError());
+  if (int rc = copy_out(h, accepted, o_acc, B)) return rc;
+  if (int rc = copy_out(h, bonus, o_bonus, B)) return rc;
+  if (int rc = copy_out(h, kv_len, o_len, B)) return rc;
+  if (int rc = copy_out(h, anchor, o_anchor, B)) return rc;
+  if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
+}
+
+int asr_spec_rollback(asr_spec_handle h, const int32_t* new_len, const int32_t* new_pending) {
+  if (!h) return ASR_E_INVAL;
+  if (h->state < 2) return fail(h, ASR_E_STATE, "rollback before prefill");
+  if (!new_len || !new_pending) return fail(h, ASR_E_INVAL, "null pointer");
+  if (int rc = copy_in(h, h->misc, new_len, h->B)) return rc;
+  if (int rc = copy_in(h, h->lens_buf, new_pending, h->B)) return rc;
+  launch_rollback(h->misc, h->lens_buf, h->B, h->V, h->kv_len, h->pending, h->status, h->st);
+  CK(cudaGetLastError());
+  if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
+}
+
+int asr_spec_state(asr_spec_handle h, int32_t* kv_len, int32_t* pending) {
+  if (!h || !kv_len || !pending) return ASR_E_INVAL;
+  if (int rc = copy_out(h, kv_len, h->kv_len, h->B)) return rc;
+  if (int rc = copy_out(h, pending, h->pending, h->B)) return rc;
+  if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
+}
+
+int asr_spec_debug_logits(asr_spec_handle h, float* out, int32_t max_rows) {
+  if (!h || !out) return ASR_E_INVAL;
+  int R = 0;
+  CK(cudaMemcpyAsync(&R, h->plan.n_rows, 4, cudaMemcpyDeviceToHost, h->st));
+  CK(cudaStreamSynchronize(h->st));
+  if (R > max_rows) return fail(h, ASR_E_INVAL, "output too small");
+  if (R == 0) return 0;
+  float* dst = out;
+  float* tmp = nullptr;
+  if (h->host_io) {
+    CK(cudaMalloc(&tmp, (size_t)R * h->V * 4));
+    dst = tmp;
+  }
+  Epi e{};
+  e.out_f32 = dst;
+  e.ld = h->V;
+  e.n_valid = h->plan.n_rows;
+  int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, R, EPI_F32, e);
+  if (!rc && h->host_io) {
+    CK(cudaMemcpyAsync(out, tmp, (size_t)R * h->V * 4, cudaMemcpyDeviceToHost, h->st));
+  }
+  CK(cudaStreamSynchronize(h->st));
+  if (tmp) cudaFree(tmp);
+  return rc ? rc : R;
+}
+
+int asr_spec_status(asr_spec_handle h) {
+  if (!h) return ASR_E_INVAL;
+  int s = 0;
+  CK(cudaStreamSynchronize(h->st));
+  CK(cudaMemcpy(&s, h->status, 4, cudaMemcpyDeviceToHost));
+  CK(cudaMemset(h->status, 0, 4));
+  return s;
+}
+
+const char* asr_spec_last_error(asr_spec_handle h) { return h ? h->err.c_str() : "null handle"; }
+
+void asr_spec_destroy(asr_spec_handle h) {
+  if (!h) return;
+  cudaStreamSynchronize(h->st);
+  for (void* p : h->allocs) cudaFree(p);
+  delete h;
+}
+
+int asr_spec_synth_drafts(asr_spec_handle h, const int32_t* truth, const int32_t* total_len, const int32_t* repl,
+                          int32_t k_repl, const int32_t* shift, int32_t k, int32_t* draft_out, int32_t* lens_out) {
+  if (!h || !truth || !total_len || !repl || !shift || !draft_out || !lens_out) return ASR_E_INVAL;
+  if (k < 1 || k > k_repl) return fail(h, ASR_E_INVAL, "k outside [1, k_repl]");
+  launch_synth_drafts(truth, total_len, repl, k_repl, shift, k, h->B, h->maxpos, h->kv_len, draft_out, lens_out,
+                      h->st);
+  CK(cudaGetLastError());
+  return ASR_OK;
+}
+
+int asr_spec_test_gemm(int32_t impl, const void* A, const void* B, float* C, int32_t M, int32_t N, int32_t K,
+                       void* stream) {
+  asr_spec* h = nullptr;
+  if (!A || !B || !C || M < 1 || N < 1 || K < 64 || K % 64) return ASR_E_INVAL;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  Epi e{};
+  e.M = M;
+  e.N = N;
+  e.out_f32 = C;
+  e.ld = N;
+  if (impl == 1) {
+    launch_gemm_simt(A, 1, B, 1, M, N, K, EPI_F32_MN, e, st);
+  } else {
+    TcGemm g{};
+    g.bn = tc_pick_bn(N);
+    if (!make_tmap_bf16(&g.mapA, A, M, K, 128) || !make_tmap_bf16(&g.mapB, B, N, K, g.bn)) return ASR_E_INVAL;
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    const int tiles = ((M + 127) / 128) * ((N + g.bn - 1) / g.bn);
+    g.splits = impl == 2 ? std::min(3, K / 64) : 1;
+    int* status = nullptr;
+    CK(cudaMalloc(&status, 4));
+    CK(cudaMemset(status, 0, 4));
+    if (g.splits > 1) {
+      CK(cudaMalloc(&g.ws, (size_t)g.splits * tiles * 128 * g.bn * 4));
+      CK(cudaMalloc(&g.tickets, (size_t)tiles * 4));
+      CK(cudaMemset(g.tickets, 0, (size_t)tiles * 4));
+    }
+    launch_gemm_tc(g, EPI_F32_MN, e, status, st);
+    CK(cudaGetLastError());
+    CK(cudaStreamSynchronize(st));
+    int s = 0;
+    CK(cudaMemcpy(&s, status, 4, cudaMemcpyDeviceToHost));
+    cudaFree(status);
+    if (g.ws) cudaFree(g.ws);
+    if (g.tickets) cudaFree(g.tickets);
+    if (s) return ASR_E_DEVICE;
+  }
+  CK(cudaGetLastError());
+  CK(cudaStreamSynchronize(st));
+  return ASR_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,244 @@
+// Split-KV attention over the verify rows, and the re-anchoring readout.
+//
+// Self-attention (Sec. 3 "Speculative Loop": the target checks the whole
+// draft block in one pass): row i of utterance b sits at position P_b + i and
+// attends to cached keys 0 .. P_b + i, i.e. the committed cache plus rows
+// 0..i of its own block (a block-causal mask).  Cross-attention: every row
+// attends to the utterance's enc_len[b] encoder frames.
+//
+// One CTA takes one (utterance, head, key chunk): it stages the chunk's K and V
+// in shared memory once and serves every row of that utterance from it.  Each
+// chunk leaves (max, sum, unnormalised output) per row; a merge kernel
+// combines the chunks in chunk order.
+//
+// Anchor (Sec. 5 "Verification-Attention Correction"; App. "Runtime anchor
+// construction"): the head mean of the per-head softmax attention of one row
+// at the anchor layer, recomputed from the cached keys with the (max, sum) that
+// the attention pass left, then its peak frame.
+#include "kernels.h"
+
+namespace asrspec {
+
+constexpr float ATTN_SCALE = 0.125f;  // 1 / sqrt(64)
+
+// q . k over 64 dims, visiting the 32 element pairs starting at pair (j mod 32):
+// consecutive rows of a shared-memory tile then hit different banks.  The same
+// order is used by the anchor readout so both compute identical scores.
+template <typename T>
+__device__ __forceinline__ float dot64_rot(const float* q, const T* k, int j) {
+  float acc = 0.f;
+#pragma unroll 8
+  for (int t = 0; t < 32; ++t) {
+    const int w = (t + j) & 31;
+    acc = fmaf(q[2 * w], to_f<T>(k[2 * w]), acc);
+    acc = fmaf(q[2 * w + 1], to_f<T>(k[2 * w + 1]), acc);
+  }
+  return acc;
+}
+
+constexpr int ATTN_THREADS = 256;
+constexpr int ATTN_MAX_ROWS = 32;   // rows per utterance served by one CTA (k + 1 <= 32)
+
+template <typename T, int CHUNK>
+__global__ void __launch_bounds__(ATTN_THREADS) attn_chunk_kernel(AttnArgs a) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  T* Ks = reinterpret_cast<T*>(smem);
+  T* Vs = Ks + CHUNK * 64;
+  float* Qs = reinterpret_cast<float*>(Vs + CHUNK * 64);     // [rows][64]
+  float* S = Qs + ATTN_MAX_ROWS * 64;                        // [rows][CHUNK]
+  __shared__ float s_m[ATTN_MAX_ROWS], s_l[ATTN_MAX_ROWS];
+
+  const int chunk = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int nr = a.plan.n_utt_rows[b];
+  if (nr == 0) return;
+  const int row0 = a.plan.row_start[b];
+  const int n_keys = a.causal ? a.kv_len[b] + nr : a.enc_len[b];
+  const int key0 = chunk * CHUNK;
+  if (key0 >= n_keys) return;
+  const int nk = min(CHUNK, n_keys - key0);
+  const int tid = threadIdx.x;
+
+  // stage K, V (contiguous [nk][64] for this (b, h)) and the rows' queries
+  const size_t base = (((size_t)b * a.H + h) * a.t_alloc + key0) * 64;
+  const T* gK = static_cast<const T*>(a.kc) + base;
+  const T* gV = static_cast<const T*>(a.vc) + base;
+  constexpr int VEC = 16 / sizeof(T);
+  const int nvec = nk * 64 / VEC;
+  for (int v = tid; v < nvec; v += ATTN_THREADS) {
+    reinterpret_cast<uint4*>(Ks)[v] = __ldg(reinterpret_cast<const uint4*>(gK) + v);
+    reinterpret_cast<uint4*>(Vs)[v] = __ldg(reinterpret_cast<const uint4*>(gV) + v);
+  }
+  for (int e = tid; e < nr * 64; e += ATTN_THREADS) {
+    const int i = e >> 6, c = e & 63;
+    Qs[e] = a.q[(size_t)(row0 + i) * a.d + h * 64 + c];
+  }
+  __syncthreads();
+
+  // scores
+  for (int e = tid; e < nr * nk; e += ATTN_THREADS) {
+    const int i = e / nk, j = e - i * nk;
+    const int key = key0 + j;
+    float s = dot64_rot<T>(Qs + i * 64, Ks + j * 64, j) * ATTN_SCALE;
+    if (a.causal && key > a.plan.row_pos[row0 + i]) s = -INFINITY;
+    S[i * CHUNK + j] = s;
+  }
+  __syncthreads();
+
+  // per-row max and sum over the chunk (one warp per row)
+  const int warp = tid >> 5, lane = tid & 31;
+  for (int i = warp; i < nr; i += ATTN_THREADS / 32) {
+    float m = -INFINITY;
+    for (int j = lane; j < nk; j += 32) m = fmaxf(m, S[i * CHUNK + j]);
+    m = warp_max(m);
+    float l = 0.f;
+    for (int j = lane; j < nk; j += 32) {
+      const float s = S[i * CHUNK + j];
+      const float p = (s == -INFINITY) ? 0.f : expf(s - m);
+      S[i * CHUNK + j] = p;
+      l += p;
+    }
+    l = warp_sum(l);
+    if (lane == 0) {
+      s_m[i] = m;
+      s_l[i] = l;
+    }
+  }
+  __syncthreads();
+
+  // unnormalised output of the chunk
+  float* part = a.part + (((size_t)b * a.H + h) * a.n_chunks + chunk) * a.k1 * 66;
+  for (int e = tid; e < nr * 64; e += ATTN_THREADS) {
+    const int i = e >> 6, c = e & 63;
+    float o = 0.f;
+    const float* p = S + i * CHUNK;
+    for (int j = 0; j < nk; ++j) o = fmaf(p[j], to_f<T>(Vs[j * 64 + c]), o);
+    part[i * 66 + c] = o;
+  }
+  if (tid < nr) {
+    part[tid * 66 + 64] = s_m[tid];
+    part[tid * 66 + 65] = s_l[tid];
+  }
+}
+
+// Merge the chunks of one (row, head) in chunk order.
+__global__ void attn_merge_kernel(AttnArgs a, int chunk_len) {
+  const int i = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int nr = a.plan.n_utt_rows[b];
+  if (i >= nr) return;
+  const int r = a.plan.row_start[b] + i;
+  const int n_keys = a.causal ? a.kv_len[b] + nr : a.enc_len[b];
+  const int nc = (n_keys + chunk_len - 1) / chunk_len;
+  const float* part = a.part + ((size_t)b * a.H + h) * a.n_chunks * a.k1 * 66 + (size_t)i * 66;
+  const size_t cstride = (size_t)a.k1 * 66;
+  float M = -INFINITY;
+  for (int c = 0; c < nc; ++c) M = fmaxf(M, part[c * cstride + 64]);
+  float l = 0.f, o = 0.f;
+  const int cc = threadIdx.x;   // 64 threads, one per output dim
+  for (int c = 0; c < nc; ++c) {
+    const float m_c = part[c * cstride + 64];
+    const float w = (m_c == -INFINITY) ? 0.f : expf(m_c - M);
+    l += part[c * cstride + 65] * w;
+    o += part[c * cstride + cc] * w;
+  }
+  o = o / l;
+  const size_t oi = (size_t)r * a.d + h * 64 + cc;
+  if (a.out_bf16) reinterpret_cast<__nv_bfloat16*>(a.out)[oi] = f2bf(o);
+  else reinterpret_cast<float*>(a.out)[oi] = o;
+  if (a.ml_out && cc == 0) {
+    a.ml_out[((size_t)r * a.H + h) * 2 + 0] = M;
+    a.ml_out[((size_t)r * a.H + h) * 2 + 1] = l;
+  }
+}
+
+template <typename T, int CHUNK>
+static size_t attn_smem() {
+  return (size_t)2 * CHUNK * 64 * sizeof(T) + (size_t)ATTN_MAX_ROWS * 64 * 4 + (size_t)ATTN_MAX_ROWS * CHUNK * 4;
+}
+
+template <typename T, int CHUNK>
+static void launch_attn_t(const AttnArgs& a, cudaStream_t st) {
+  static bool configured = false;
+  const size_t sm = attn_smem<T, CHUNK>();
+  if (!configured) {
+    cudaFuncSetAttribute(attn_chunk_kernel<T, CHUNK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    configured = true;
+  }
+  dim3 grid(a.n_chunks, a.H, a.B);
+  attn_chunk_kernel<T, CHUNK><<<grid, ATTN_THREADS, sm, st>>>(a);
+  dim3 mgrid(a.k1, a.H, a.B);
+  attn_merge_kernel<<<mgrid, 64, 0, st>>>(a, CHUNK);
+}
+
+void launch_attention(const AttnArgs& a, cudaStream_t st) {
+  if (a.kv_bf16) launch_attn_t<__nv_bfloat16, 256>(a, st);
+  else launch_attn_t<float, 128>(a, st);
+}
+
+int attn_chunk_len(int kv_bf16) { return kv_bf16 ? 256 : 128; }
+
+// ---------------------------------------------------------------------------
+// Anchor readout
+// ---------------------------------------------------------------------------
+constexpr int ANCHOR_FRAMES = 256;
+
+template <typename T>
+__global__ void __launch_bounds__(ANCHOR_FRAMES)
+anchor_kernel(const float* __restrict__ q_anchor, const float* __restrict__ ml, const T* __restrict__ kc, int t_alloc,
+              const int* __restrict__ enc_len, const int* __restrict__ anchor_row, int H, int d,
+              unsigned long long* frame_key, int* tickets, int* anchor_out) {
+  __shared__ float qs[64];
+  __shared__ unsigned long long red[ANCHOR_FRAMES / 32];
+  __shared__ int s_last;
+  const int b = blockIdx.y;
+  const int r = anchor_row[b];
+  if (r < 0) return;  // uniform: the utterance sat out or the step was refused
+  const int n_frames = enc_len[b];
+  const int j = blockIdx.x * ANCHOR_FRAMES + threadIdx.x;
+  float pbar = 0.f;
+  for (int h = 0; h < H; ++h) {
+    __syncthreads();
+    if (threadIdx.x < 64) qs[threadIdx.x] = q_anchor[(size_t)r * d + h * 64 + threadIdx.x];
+    __syncthreads();
+    if (j < n_frames) {
+      const T* krow = kc + (((size_t)b * H + h) * t_alloc + j) * 64;
+      const float s = dot64_rot<T>(qs, krow, j) * ATTN_SCALE;
+      const float M = ml[((size_t)r * H + h) * 2 + 0];
+      const float l = ml[((size_t)r * H + h) * 2 + 1];
+      pbar += expf(s - M) / l;
+    }
+  }
+  pbar = pbar / (float)H;
+  unsigned long long key = j < n_frames ? argmax_key(pbar, (uint32_t)j) : 0ull;
+  key = warp_max_u64(key);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = key;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long k = red[0];
+    for (int w = 1; w < ANCHOR_FRAMES / 32; ++w) k = red[w] > k ? red[w] : k;
+    atomicMax(frame_key + b, k);
+    __threadfence();
+    s_last = (atomicAdd(tickets + b, 1) == (int)gridDim.x - 1);
+    if (s_last) {
+      __threadfence();
+      const unsigned long long fk = atomicExch(frame_key + b, 0ull);
+      anchor_out[b] = (int)argmax_index(fk);
+      tickets[b] = 0;
+    }
+  }
+}
+
+void launch_anchor(const float* q_anchor, const float* ml, const void* kc, int kv_bf16, int t_alloc,
+                   const int* enc_len, const int* anchor_row, int B, int H, int d, unsigned long long* frame_key,
+                   int* tickets, int* anchor_out, cudaStream_t st) {
+  dim3 grid((t_alloc + ANCHOR_FRAMES - 1) / ANCHOR_FRAMES, B);
+  if (kv_bf16)
+    anchor_kernel<__nv_bfloat16><<<grid, ANCHOR_FRAMES, 0, st>>>(q_anchor, ml,
+                                                                 static_cast<const __nv_bfloat16*>(kc), t_alloc,
+                                                                 enc_len, anchor_row, H, d, frame_key, tickets,
+                                                                 anchor_out);
+  else
+    anchor_kernel<float><<<grid, ANCHOR_FRAMES, 0, st>>>(q_anchor, ml, static_cast<const float*>(kc), t_alloc,
+                                                         enc_len, anchor_row, H, d, frame_key, tickets, anchor_out);
+}
+
+}  // namespace asrspec

@@ -1,0 +1,280 @@
+// tcgen05 tensor-core GEMM for the decoder projections, the LM head and the
+// per-utterance cross-attention K/V build.
+//
+// C[m][n] = sum_k A[m][k] B[n][k], A and B bf16 and K-major, fp32 accumulators
+// in tensor memory.  One CTA computes one 128 x BN output tile (optionally one
+// split of its K range):
+//   warp 0 / lane 0 : TMA producer, STAGES-deep ring of (A, B) k-blocks
+//   warp 1 / lane 0 : issues tcgen05.mma (M=128, N=BN, K=16) x 4 per k-block
+//   warps 0..3      : epilogue, each reading its 32 TMEM lanes (= 32 values of m)
+// Split-K partials go to a workspace; the last CTA of a tile (atomic ticket)
+// sums them in split order, so results do not depend on CTA timing.
+#include <cstdio>
+#include <mutex>
+
+#include "kernels.h"
+
+namespace asrspec {
+
+constexpr int TC_BM = 128;
+constexpr int TC_BK = 64;
+constexpr int TC_STAGES = 4;
+
+template <int BN>
+struct TcCfg {
+  static constexpr int A_BYTES = TC_BM * TC_BK * 2;
+  static constexpr int B_BYTES = BN * TC_BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int BAR_OFF = TC_STAGES * STAGE_BYTES;
+  static constexpr int SMEM = 1024 + BAR_OFF + 256;
+  static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+  static_assert(B_BYTES % 1024 == 0, "B tile must keep 1024-byte alignment");
+};
+
+template <int BN, int MODE>
+__global__ void __launch_bounds__(128, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, int K, int splits,
+               float* __restrict__ ws, int* __restrict__ tickets, Epi epi, int* status) {
+  using C = TcCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + TC_STAGES * C::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::BAR_OFF);
+  uint64_t* empty = full + TC_STAGES;
+  uint64_t* done = empty + TC_STAGES;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  __shared__ unsigned long long red[4][BN];
+  __shared__ int s_last;
+
+  const int tile_m = blockIdx.x, tile_n = blockIdx.y, split = blockIdx.z;
+  const int m0 = tile_m * TC_BM, n0 = tile_n * BN;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_valid = epi.n_valid ? *epi.n_valid : epi.N;
+  const int nkb_total = K / TC_BK;
+  const int kb0 = (nkb_total * split) / splits;
+  const int kb1 = (nkb_total * (split + 1)) / splits;
+  const int nkb = kb1 - kb0;
+  if (n0 >= n_valid || nkb <= 0) return;  // uniform over the CTA and over all splits of a tile
+
+  if (warp == 0) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  if (threadIdx.x == 32) {
+    for (int s = 0; s < TC_STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(done, 1);
+    fence_mbar_init();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&mapA);
+    tma_prefetch_desc(&mapB);
+    int issued = 0;
+    for (int i = 0; i < nkb; ++i) {
+      const int s = i % TC_STAGES;
+      const uint32_t ph = (i / TC_STAGES) & 1;
+      if (!mbar_wait(&empty[s], ph ^ 1, status)) break;
+      mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
+      tma_load_2d(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0);
+      tma_load_2d(sB + s * C::B_BYTES, &mapB, &full[s], (kb0 + i) * TC_BK, n0);
+      issued = i + 1;
+    }
+    // Drain: every issued copy has landed before this CTA can exit.
+    for (int i = issued - TC_STAGES > 0 ? issued - TC_STAGES : 0; i < issued; ++i)
+      mbar_wait(&full[i % TC_STAGES], (i / TC_STAGES) & 1, status);
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t idesc = umma_idesc_bf16(TC_BM, BN);
+    for (int i = 0; i < nkb; ++i) {
+      const int s = i % TC_STAGES;
+      const uint32_t ph = (i / TC_STAGES) & 1;
+      if (!mbar_wait(&full[s], ph, status)) break;
+      tc_fence_after();
+      const uint32_t a_addr = smem_u32(sA + s * C::A_BYTES);
+      const uint32_t b_addr = smem_u32(sB + s * C::B_BYTES);
+#pragma unroll
+      for (int kk = 0; kk < TC_BK / 16; ++kk)
+        umma_bf16(tmem, umma_desc_sw128(a_addr + kk * 32), umma_desc_sw128(b_addr + kk * 32), idesc,
+                  (i | kk) != 0);
+      umma_commit(&empty[s]);
+    }
+    umma_commit(done);
+  }
+  __syncwarp();
+  mbar_wait(done, 0, status);
+  tc_fence_after();
+
+  const int m = m0 + warp * 32 + lane;
+  const uint32_t t_lane = tmem + ((uint32_t)(warp * 32) << 16);
+
+  if (splits == 1) {
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(t_lane + c0, v);
+      if constexpr (MODE == EPI_ARGMAX) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int n = n0 + c0 + i;
+          unsigned long long key = (m < epi.M && n < n_valid) ? argmax_key(v[i], (uint32_t)m) : 0ull;
+          key = warp_max_u64(key);
+          if (lane == 0) red[warp][c0 + i] = key;
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int n = n0 + c0 + i;
+          if (m < epi.M && n < n_valid) epi_apply<MODE>(epi, m, n, v[i]);
+        }
+      }
+    }
+    if constexpr (MODE == EPI_ARGMAX) {
+      __syncthreads();
+      if (threadIdx.x < BN) {
+        const int n = n0 + threadIdx.x;
+        unsigned long long k = red[0][threadIdx.x];
+#pragma unroll
+        for (int w = 1; w < 4; ++w) k = red[w][threadIdx.x] > k ? red[w][threadIdx.x] : k;
+        if (n < n_valid) atomicMax(epi.row_key + n, k);
+      }
+    }
+  } else {
+    const int tile = tile_n * gridDim.x + tile_m;
+    float* my = ws + ((size_t)(tile * splits + split) * TC_BM + warp * 32 + lane) * BN;
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(t_lane + c0, v);
+#pragma unroll
+      for (int i = 0; i < 16; i += 4)
+        *reinterpret_cast<float4*>(my + c0 + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_last = (atomicAdd(tickets + tile, 1) == splits - 1);
+    __syncthreads();
+    if (s_last) {
+      __threadfence();
+      const float* base = ws + ((size_t)tile * splits * TC_BM + warp * 32 + lane) * BN;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 4) {
+        float4 acc = __ldcg(reinterpret_cast<const float4*>(base + c0));
+        for (int s = 1; s < splits; ++s) {
+          float4 p = __ldcg(reinterpret_cast<const float4*>(base + (size_t)s * TC_BM * BN + c0));
+          acc.x += p.x; acc.y += p.y; acc.z += p.z; acc.w += p.w;
+        }
+        const float a4[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int n = n0 + c0 + i;
+          if (m < epi.M && n < n_valid) epi_apply<MODE == EPI_ARGMAX ? EPI_F32 : MODE>(epi, m, n, a4[i]);
+        }
+      }
+      if (threadIdx.x == 0) tickets[tile] = 0;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &p, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) || (cols * 2) % 16) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int tc_pick_bn(int n_max) {
+  if (n_max <= 16) return 16;
+  if (n_max <= 32) return 32;
+  if (n_max <= 64) return 64;
+  if (n_max <= 128) return 128;
+  return 256;
+}
+
+size_t tc_smem_bytes(int bn) {
+  switch (bn) {
+    case 16: return TcCfg<16>::SMEM;
+    case 32: return TcCfg<32>::SMEM;
+    case 64: return TcCfg<64>::SMEM;
+    case 128: return TcCfg<128>::SMEM;
+    default: return TcCfg<256>::SMEM;
+  }
+}
+
+template <int BN, int MODE>
+static void launch_tc_t(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
+  auto kern = gemm_tc_kernel<BN, MODE>;
+  static bool configured = false;
+  if (!configured) {
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
+    configured = true;
+  }
+  dim3 grid((g.M + TC_BM - 1) / TC_BM, (g.N + BN - 1) / BN, g.splits);
+  kern<<<grid, 128, TcCfg<BN>::SMEM, st>>>(g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
+}
+
+template <int MODE>
+static void launch_tc_mode(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
+  switch (g.bn) {
+    case 16: launch_tc_t<16, MODE>(g, epi, status, st); break;
+    case 32: launch_tc_t<32, MODE>(g, epi, status, st); break;
+    case 64: launch_tc_t<64, MODE>(g, epi, status, st); break;
+    case 128: launch_tc_t<128, MODE>(g, epi, status, st); break;
+    default: launch_tc_t<256, MODE>(g, epi, status, st); break;
+  }
+}
+
+void launch_gemm_tc(const TcGemm& g, int mode, const Epi& epi, int* status, cudaStream_t st) {
+  switch (mode) {
+    case EPI_F32: launch_tc_mode<EPI_F32>(g, epi, status, st); break;
+    case EPI_F32_MN: launch_tc_mode<EPI_F32_MN>(g, epi, status, st); break;
+    case EPI_QKV: launch_tc_mode<EPI_QKV>(g, epi, status, st); break;
+    case EPI_RESID: launch_tc_mode<EPI_RESID>(g, epi, status, st); break;
+    case EPI_Q: launch_tc_mode<EPI_Q>(g, epi, status, st); break;
+    case EPI_GELU: launch_tc_mode<EPI_GELU>(g, epi, status, st); break;
+    case EPI_CROSSKV: launch_tc_mode<EPI_CROSSKV>(g, epi, status, st); break;
+    case EPI_ARGMAX: launch_tc_mode<EPI_ARGMAX>(g, epi, status, st); break;
+  }
+}
+
+}  // namespace asrspec

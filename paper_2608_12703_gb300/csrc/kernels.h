@@ -1,0 +1,98 @@
+// Host-side launchers of the draft-verify kernels (internal to libasrspec).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda.h>
+
+#include "epilogue.cuh"
+
+namespace asrspec {
+
+// ---- GEMM: C[m][n] = sum_k A[m][k] B[n][k] (+ epilogue) ---------------------
+// tcgen05 path: A, B bf16 K-major, described by 2-D tensor maps (box 64 x 128
+// for A, 64 x BN for B, 128-byte swizzle).  K % 64 == 0.
+struct TcGemm {
+  CUtensorMap mapA;
+  CUtensorMap mapB;
+  int M, N, K;
+  int bn;        // N tile: 16, 32, 64, 128 or 256
+  int splits;    // split-K factor (1 = none)
+  float* ws;     // split-K partials (splits * tiles * 128 * bn floats)
+  int* tickets;  // one zeroed int per output tile
+};
+
+bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
+int tc_pick_bn(int n_max);
+void launch_gemm_tc(const TcGemm& g, int mode, const Epi& epi, int* status, cudaStream_t st);
+size_t tc_smem_bytes(int bn);
+
+// SIMT path (fp32 models, and a cross-check of the tensor-core path).
+// A: [M][K] of type a_bf16 ? bf16 : fp32; B: [N][K] likewise.
+void launch_gemm_simt(const void* A, int a_bf16, const void* B, int b_bf16, int M, int N, int K, int mode,
+                      const Epi& epi, cudaStream_t st);
+
+// ---- Row bookkeeping, embedding, LayerNorm ---------------------------------
+struct RowPlan {
+  int* row_b;       // [R_max]
+  int* row_i;       // [R_max]
+  int* row_pos;     // [R_max]
+  int* row_tok;     // [R_max]
+  int* row_start;   // [B_max + 1]
+  int* n_rows;      // [1] rows of this step (0 when the step is refused)
+  int* n_utt_rows;  // [B_max] rows of utterance b this step (lens+1, or 0)
+};
+
+// Validate the step's inputs, lay out the rows and reset the argmax keys.
+void launch_plan_verify(const int* draft, const int* lens, int k, int B, int vocab, int max_pos, const int* kv_len,
+                        const int* pending, const int* ready, RowPlan plan, unsigned long long* row_key,
+                        int* status, cudaStream_t st);
+void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,
+                               RowPlan plan, int* status, cudaStream_t st);
+void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
+                  cudaStream_t st);
+// y = LN(x) * g + b over rows < n_rows, written as bf16 or fp32.
+void launch_layernorm(const float* x, const float* g, const float* b, void* y, int y_bf16, const int* n_rows,
+                      int R_max, int d, cudaStream_t st);
+
+// ---- Attention ---------------------------------------------------------------
+struct AttnArgs {
+  const float* q;          // [R][d] fp32 queries
+  const void* kc;          // key cache base of this layer:   [B_max][H][T_alloc][64]
+  const void* vc;          // value cache base of this layer
+  int kv_bf16;
+  int t_alloc;             // rows per (b, h) in the cache (max_pos or max_enc)
+  int causal;              // 1: self-attention, keys 0..row_pos; 0: cross, keys 0..enc_len-1
+  const int* enc_len;      // [B_max] (cross)
+  const int* kv_len;       // [B_max] committed lengths (self; keys up to kv_len + i)
+  RowPlan plan;
+  int B, H, d, k1;         // utterances, heads, d_model, rows per utterance slot (k + 1)
+  int chunk;               // keys per split
+  int n_chunks;            // splits per (b, h)
+  float* part;             // [B][H][n_chunks][k1] x (64 + 2) partials
+  void* out;               // [R][d] attention output (bf16 or fp32)
+  int out_bf16;
+  float* ml_out;           // optional [R][H][2] (max, sum) of the full softmax
+};
+void launch_attention(const AttnArgs& a, cudaStream_t st);
+
+// Anchor readout: head-mean softmax of row anchor_row[b] at the anchor layer.
+void launch_anchor(const float* q_anchor, const float* ml, const void* kc, int kv_bf16, int t_alloc,
+                   const int* enc_len, const int* anchor_row, int B, int H, int d,
+                   unsigned long long* frame_key, int* tickets, int* anchor_out, cudaStream_t st);
+
+// ---- Accept / commit ------------------------------------------------------------
+void launch_accept(const int* draft, const int* lens, int k, int B, RowPlan plan, const unsigned long long* row_key,
+                   int* kv_len, int* pending, int* accepted, int* bonus, int* kv_len_out, int* anchor_row,
+                   int* anchor_out, cudaStream_t st);
+void launch_prefill_advance(int B, int c, const int* n_utt_rows, int* kv_len, cudaStream_t st);
+void launch_prefill_finish(const int* prompt, int P0, int B, int* pending, const int* ready, cudaStream_t st);
+void launch_rollback(const int* new_len, const int* new_pending, int B, int vocab, int* kv_len, int* pending,
+                     int* status, cudaStream_t st);
+void launch_synth_drafts(const int* truth, const int* total_len, const int* repl, int k_repl, const int* shift, int k,
+                         int B, int max_pos, const int* kv_len, int* draft_out, int* lens_out, cudaStream_t st);
+void launch_mark_ready(const int* enc_len, int B, int t_max, int* ready, int* kv_len, int* pending, int* status,
+                       cudaStream_t st);
+int attn_chunk_len(int kv_bf16);
+
+}  // namespace asrspec

@@ -1,0 +1,337 @@
+// Row bookkeeping of the verify step: input validation and row layout,
+// embeddings, LayerNorm, greedy longest-prefix acceptance with the KV-length
+// commit, rollback, and the synthetic draft source used by benchmarks.
+#include "kernels.h"
+
+namespace asrspec {
+
+constexpr int PLAN_THREADS = 1024;
+
+// Exclusive block scan of one int per thread (PLAN_THREADS threads).
+__device__ int block_excl_scan(int v, int* total) {
+  __shared__ int warp_sums[PLAN_THREADS / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sums[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = warp_sums[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    warp_sums[lane] = w;
+  }
+  __syncthreads();
+  const int incl = x + (warp > 0 ? warp_sums[warp - 1] : 0);
+  *total = warp_sums[PLAN_THREADS / 32 - 1];
+  return incl - v;
+}
+
+// Verify rows: utterance b contributes lens[b] + 1 rows (pending, then drafts),
+// at positions kv_len[b] + i.  Any invalid input refuses the whole step
+// (n_rows = 0, nothing is written) and sets the status word.
+__global__ void __launch_bounds__(PLAN_THREADS)
+plan_verify_kernel(const int* __restrict__ draft, const int* __restrict__ lens, int k, int B, int vocab, int max_pos,
+                   const int* __restrict__ kv_len, const int* __restrict__ pending, const int* __restrict__ ready,
+                   RowPlan plan, unsigned long long* row_key, int* status) {
+  __shared__ int s_err;
+  if (threadIdx.x == 0) s_err = 0;
+  __syncthreads();
+  const int b = threadIdx.x;
+  int n_b = 0, err = 0;
+  if (b < B) {
+    const int l = lens[b];
+    if (l < -1 || l > k) err |= ST_BAD_LENS;
+    else if (l >= 0) {
+      if (!ready[b]) err |= ST_NOT_READY;
+      if (kv_len[b] + l + 1 > max_pos) err |= ST_CAPACITY;
+      for (int i = 0; i < l; ++i) {
+        const int t = draft[(size_t)b * k + i];
+        if (t < 0 || t >= vocab) err |= ST_BAD_TOKEN;
+      }
+      n_b = l + 1;
+    }
+  }
+  if (err) atomicOr(&s_err, err);
+  __syncthreads();
+  if (s_err) {
+    n_b = 0;
+    if (threadIdx.x == 0) set_status(status, s_err);
+  }
+  int total;
+  const int start = block_excl_scan(n_b, &total);
+  if (b < B) {
+    plan.row_start[b] = start;
+    plan.n_utt_rows[b] = n_b;
+    for (int i = 0; i < n_b; ++i) {
+      const int r = start + i;
+      plan.row_b[r] = b;
+      plan.row_i[r] = i;
+      plan.row_pos[r] = kv_len[b] + i;
+      plan.row_tok[r] = i == 0 ? pending[b] : draft[(size_t)b * k + i - 1];
+      row_key[r] = 0ull;
+    }
+  }
+  if (threadIdx.x == 0) {
+    plan.row_start[B] = total;
+    *plan.n_rows = total;
+  }
+}
+
+// Prefill rows: prompt tokens p0 .. p0+c-1 of every utterance at positions p0 + i.
+__global__ void __launch_bounds__(PLAN_THREADS)
+plan_prefill_kernel(const int* __restrict__ prompt, int P0, int p0, int c, int B, int vocab,
+                    const int* __restrict__ ready, RowPlan plan, int* status) {
+  __shared__ int s_err;
+  if (threadIdx.x == 0) s_err = 0;
+  __syncthreads();
+  const int b = threadIdx.x;
+  int err = 0;
+  if (b < B) {
+    if (!ready[b]) err |= ST_NOT_READY;
+    for (int i = 0; i < P0; ++i) {
+      const int t = prompt[(size_t)b * P0 + i];
+      if (t < 0 || t >= vocab) err |= ST_BAD_TOKEN;
+    }
+  }
+  if (err) atomicOr(&s_err, err);
+  __syncthreads();
+  const int n_b = (b < B && !s_err) ? c : 0;
+  if (s_err && threadIdx.x == 0) set_status(status, s_err);
+  int total;
+  const int start = block_excl_scan(n_b, &total);
+  if (b < B) {
+    plan.row_start[b] = start;
+    plan.n_utt_rows[b] = n_b;
+    for (int i = 0; i < n_b; ++i) {
+      const int r = start + i;
+      plan.row_b[r] = b;
+      plan.row_i[r] = i;
+      plan.row_pos[r] = p0 + i;
+      plan.row_tok[r] = prompt[(size_t)b * P0 + p0 + i];
+    }
+  }
+  if (threadIdx.x == 0) {
+    plan.row_start[B] = total;
+    *plan.n_rows = total;
+  }
+}
+
+void launch_plan_verify(const int* draft, const int* lens, int k, int B, int vocab, int max_pos, const int* kv_len,
+                        const int* pending, const int* ready, RowPlan plan, unsigned long long* row_key,
+                        int* status, cudaStream_t st) {
+  plan_verify_kernel<<<1, PLAN_THREADS, 0, st>>>(draft, lens, k, B, vocab, max_pos, kv_len, pending, ready, plan,
+                                                 row_key, status);
+}
+
+void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,
+                               RowPlan plan, int* status, cudaStream_t st) {
+  plan_prefill_kernel<<<1, PLAN_THREADS, 0, st>>>(prompt, P0, p0, c, B, vocab, ready, plan, status);
+}
+
+// x[r] = tok_emb[token] + pos_emb[position]  (fp32 residual stream)
+template <typename T>
+__global__ void embed_kernel(const T* __restrict__ tok_emb, const T* __restrict__ pos_emb, RowPlan plan, int d,
+                             float* __restrict__ x) {
+  const int r = blockIdx.x;
+  if (r >= *plan.n_rows) return;
+  const int t = plan.row_tok[r], p = plan.row_pos[r];
+  for (int c = threadIdx.x; c < d; c += blockDim.x)
+    x[(size_t)r * d + c] = to_f<T>(tok_emb[(size_t)t * d + c]) + to_f<T>(pos_emb[(size_t)p * d + c]);
+}
+
+void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
+                  cudaStream_t st) {
+  if (w_bf16)
+    embed_kernel<__nv_bfloat16><<<R_max, 128, 0, st>>>(static_cast<const __nv_bfloat16*>(tok_emb),
+                                                       static_cast<const __nv_bfloat16*>(pos_emb), plan, d, x);
+  else
+    embed_kernel<float><<<R_max, 128, 0, st>>>(static_cast<const float*>(tok_emb),
+                                               static_cast<const float*>(pos_emb), plan, d, x);
+}
+
+// LayerNorm, one warp per row, statistics in fp32 (two passes over registers).
+constexpr int LN_MAX_PER_LANE = 64;   // d <= 2048
+template <typename TO>
+__global__ void __launch_bounds__(256)
+layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const float* __restrict__ bta,
+                 TO* __restrict__ y, const int* __restrict__ n_rows, int d) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + warp;
+  if (r >= *n_rows) return;
+  const float* xr = x + (size_t)r * d;
+  float v[LN_MAX_PER_LANE];
+  const int per = d / 32;
+  float s = 0.f;
+#pragma unroll 4
+  for (int i = 0; i < per; ++i) {
+    v[i] = xr[lane + 32 * i];
+    s += v[i];
+  }
+  const float mean = warp_sum(s) / (float)d;
+  float q = 0.f;
+#pragma unroll 4
+  for (int i = 0; i < per; ++i) {
+    const float t = v[i] - mean;
+    q += t * t;
+  }
+  const float var = warp_sum(q) / (float)d;
+  const float rstd = rsqrtf(var + 1e-5f);
+#pragma unroll 4
+  for (int i = 0; i < per; ++i) {
+    const int c = lane + 32 * i;
+    y[(size_t)r * d + c] = from_f<TO>((v[i] - mean) * rstd * g[c] + bta[c]);
+  }
+}
+
+void launch_layernorm(const float* x, const float* g, const float* b, void* y, int y_bf16, const int* n_rows,
+                      int R_max, int d, cudaStream_t st) {
+  const int grid = (R_max + 7) / 8;
+  if (y_bf16)
+    layernorm_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(x, g, b, static_cast<__nv_bfloat16*>(y), n_rows, d);
+  else
+    layernorm_kernel<float><<<grid, 256, 0, st>>>(x, g, b, static_cast<float*>(y), n_rows, d);
+}
+
+// Greedy longest-prefix acceptance (Sec. 3 "Speculative Loop") and commit:
+// n = longest prefix with draft[j] == argmax of row j; bonus = argmax of row n;
+// kv_len += 1 + n (App. "Correction and Cost": a round advances 1 + L tokens).
+__global__ void accept_kernel(const int* __restrict__ draft, const int* __restrict__ lens, int k, int B,
+                              RowPlan plan, const unsigned long long* __restrict__ row_key, int* kv_len, int* pending,
+                              int* accepted, int* bonus, int* kv_len_out, int* anchor_row, int* anchor_out) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const int nr = plan.n_utt_rows[b];
+  if (nr == 0) {
+    accepted[b] = 0;
+    bonus[b] = -1;
+    kv_len_out[b] = kv_len[b];
+    anchor_row[b] = -1;
+    anchor_out[b] = -1;
+    return;
+  }
+  const int r0 = plan.row_start[b];
+  const int l = nr - 1;
+  int n = 0;
+  while (n < l && draft[(size_t)b * k + n] == (int)argmax_index(row_key[r0 + n])) ++n;
+  const int g = (int)argmax_index(row_key[r0 + n]);
+  accepted[b] = n;
+  bonus[b] = g;
+  const int nl = kv_len[b] + 1 + n;
+  kv_len[b] = nl;
+  kv_len_out[b] = nl;
+  pending[b] = g;
+  anchor_row[b] = r0 + n;
+}
+
+void launch_accept(const int* draft, const int* lens, int k, int B, RowPlan plan, const unsigned long long* row_key,
+                   int* kv_len, int* pending, int* accepted, int* bonus, int* kv_len_out, int* anchor_row,
+                   int* anchor_out, cudaStream_t st) {
+  accept_kernel<<<(B + 127) / 128, 128, 0, st>>>(draft, lens, k, B, plan, row_key, kv_len, pending, accepted, bonus,
+                                                 kv_len_out, anchor_row, anchor_out);
+}
+
+// After a prefill chunk: the rows' K/V are cached, so the committed length moves on.
+__global__ void prefill_advance_kernel(int B, int c, const int* n_utt_rows, int* kv_len) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B && n_utt_rows[b] > 0) kv_len[b] += c;
+}
+__global__ void prefill_finish_kernel(const int* __restrict__ prompt, int P0, int B, int* pending,
+                                      const int* ready) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B && ready[b]) pending[b] = prompt[(size_t)b * P0 + P0 - 1];
+}
+void launch_prefill_advance(int B, int c, const int* n_utt_rows, int* kv_len, cudaStream_t st) {
+  prefill_advance_kernel<<<(B + 127) / 128, 128, 0, st>>>(B, c, n_utt_rows, kv_len);
+}
+void launch_prefill_finish(const int* prompt, int P0, int B, int* pending, const int* ready, cudaStream_t st) {
+  prefill_finish_kernel<<<(B + 127) / 128, 128, 0, st>>>(prompt, P0, B, pending, ready);
+}
+
+// Rollback: all-or-nothing over the batch.
+__global__ void __launch_bounds__(PLAN_THREADS)
+rollback_kernel(const int* __restrict__ new_len, const int* __restrict__ new_pending, int B, int vocab, int* kv_len,
+                int* pending, int* status) {
+  __shared__ int s_err;
+  if (threadIdx.x == 0) s_err = 0;
+  __syncthreads();
+  const int b = threadIdx.x;
+  int nl = -1, np = 0;
+  if (b < B) {
+    nl = new_len[b];
+    np = new_pending[b];
+    if (nl >= 0) {
+      if (nl > kv_len[b]) atomicOr(&s_err, ST_CAPACITY);
+      if (np < 0 || np >= vocab) atomicOr(&s_err, ST_BAD_TOKEN);
+    } else if (nl < -1) {
+      atomicOr(&s_err, ST_CAPACITY);
+    }
+  }
+  __syncthreads();
+  if (s_err) {
+    if (threadIdx.x == 0) set_status(status, s_err);
+    return;
+  }
+  if (b < B && nl >= 0) {
+    kv_len[b] = nl;
+    pending[b] = np;
+  }
+}
+void launch_rollback(const int* new_len, const int* new_pending, int B, int vocab, int* kv_len, int* pending,
+                     int* status, cudaStream_t st) {
+  rollback_kernel<<<1, PLAN_THREADS, 0, st>>>(new_len, new_pending, B, vocab, kv_len, pending, status);
+}
+
+// Synthetic draft source (workload utility, stands in for a trained draft model).
+__global__ void synth_drafts_kernel(const int* __restrict__ truth, const int* __restrict__ total_len,
+                                    const int* __restrict__ repl, int k_repl, const int* __restrict__ shift, int k,
+                                    int B, int max_pos, const int* __restrict__ kv_len, int* draft_out,
+                                    int* lens_out) {
+  const int b = blockIdx.x;
+  if (b >= B) return;
+  const int P = kv_len[b], N = min(total_len[b], max_pos);
+  const int l = (P + 1 >= N) ? -1 : min(k, N - P - 2);
+  if (threadIdx.x == 0) lens_out[b] = l;
+  for (int i = 1 + threadIdx.x; i <= k; i += blockDim.x) {
+    int t = 0;
+    if (i <= l) {
+      const int s = shift[(size_t)b * max_pos + P];
+      const int j = (s > 0 && i >= s) ? P + i - 1 : P + i;
+      t = truth[(size_t)b * max_pos + j];
+      const int rp = repl[((size_t)b * max_pos + P) * k_repl + i - 1];
+      if (rp >= 0) t = rp;
+    }
+    draft_out[(size_t)b * k + i - 1] = t;
+  }
+}
+void launch_synth_drafts(const int* truth, const int* total_len, const int* repl, int k_repl, const int* shift, int k,
+                         int B, int max_pos, const int* kv_len, int* draft_out, int* lens_out, cudaStream_t st) {
+  synth_drafts_kernel<<<B, 32, 0, st>>>(truth, total_len, repl, k_repl, shift, k, B, max_pos, kv_len, draft_out,
+                                        lens_out);
+}
+
+// After encode_cache: slot b is ready iff 1 <= enc_len[b] <= t_max; its decoder state is cleared.
+__global__ void mark_ready_kernel(const int* __restrict__ enc_len, int B, int t_max, int* ready, int* kv_len,
+                                  int* pending, int* status) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const int T = enc_len[b];
+  const int ok = (T >= 1 && T <= t_max);
+  if (!ok) set_status(status, ST_CAPACITY);
+  ready[b] = ok;
+  kv_len[b] = 0;
+  pending[b] = 0;
+}
+void launch_mark_ready(const int* enc_len, int B, int t_max, int* ready, int* kv_len, int* pending, int* status,
+                       cudaStream_t st) {
+  mark_ready_kernel<<<(B + 127) / 128, 128, 0, st>>>(enc_len, B, t_max, ready, kv_len, pending, status);
+}
+
+}  // namespace asrspec

@@ -11,3 +11,20 @@ if ROOT not in sys.path:
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a)")
     config.addinivalue_line("markers", "slow: full-size cases (minutes)")
+
+
+@pytest.fixture(scope="session")
+def built_lib():
+    """Build (if stale) and load libasrspec; GPU tests depend on it."""
+    from paper_2608_12703_gb300 import build as B
+    from paper_2608_12703_gb300 import asrspec as A
+    B.build()
+    return A.lib()
+
+
+@pytest.fixture(scope="session")
+def cuda():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.fail("GPU test run without a CUDA device")
+    return torch.device("cuda")

@@ -1,0 +1,110 @@
+"""Error paths and state handling of the C ABI on the GPU: host-side argument
+errors return codes; device-side data errors refuse the whole step, leave the
+state unchanged and set the status word.  Rollback followed by the same
+verification reproduces outputs and logits bit for bit; the host-I/O path
+returns what the device path returns."""
+import numpy as np
+import pytest
+
+import workload as W
+
+pytestmark = pytest.mark.gpu
+
+DIMS = W.ModelDims(n_layers=2, d_model=128, n_heads=2, d_ffn=256, vocab=500, dtype="bf16",
+                   max_pos=24, max_enc=64, anchor_layer=1)
+
+
+@pytest.fixture
+def sess(built_lib, cuda):
+    from paper_2608_12703_gb300.session import Session
+    blob = W.make_weights(DIMS, std=0.3)
+    s = Session(DIMS, blob, max_batch=3, max_draft=4)
+    yield s
+    s.close()
+
+
+def _ready(s):
+    enc = W.make_encoder_states(DIMS, [64, 10, 33], 64)
+    s.encode_cache(enc, [64, 10, 33])
+    s.prefill(W.make_prompt(DIMS, 3))
+
+
+def test_call_order_and_arguments(sess):
+    from paper_2608_12703_gb300 import asrspec as A
+    with pytest.raises(A.AsrSpecError, match="ASR_E_STATE"):
+        sess.verify(np.zeros((1, 1)), np.zeros(1))
+    _ready(sess)
+    with pytest.raises(A.AsrSpecError, match="ASR_E_INVAL"):
+        sess.verify(np.zeros((3, 5)), np.zeros(3))         # k > max_draft
+    enc = W.make_encoder_states(DIMS, [64], 64)
+    with pytest.raises(A.AsrSpecError, match="ASR_E_CAPACITY"):
+        import torch
+        big = torch.zeros((1, 65, 128), dtype=torch.bfloat16, device="cuda")
+        sess.encode_cache(big, [65])
+    assert sess.status() == 0
+
+
+@pytest.mark.parametrize("case,bit", [("token", 1), ("lens", 2), ("capacity", 4)])
+def test_device_errors_refuse_the_step(sess, case, bit):
+    _ready(sess)
+    kv0, p0 = sess.state()
+    draft = np.array([[1, 2, 3, 4]] * 3)
+    lens = np.array([4, 2, 0])
+    if case == "token":
+        draft[1, 1] = DIMS.vocab
+    elif case == "lens":
+        lens[2] = 5
+    else:
+        for _ in range(4):
+            sess.verify(np.array([[7, 7, 7, 7]] * 3), np.array([4, -1, -1]))
+        kv0, p0 = sess.state()
+        lens = np.array([4, 0, 0])
+        draft[0] = [7, 7, 7, 7]
+        assert kv0[0] + 5 > DIMS.max_pos or pytest.skip("did not reach capacity")
+    out = sess.verify(draft, lens)
+    assert sess.status() & bit
+    kv1, p1 = sess.state()
+    assert list(kv1) == list(kv0) and list(p1) == list(p0)
+    assert list(out.bonus) == [-1, -1, -1]
+    assert sess.status() == 0
+
+
+def test_rollback_then_reverify_is_bitwise_identical(sess):
+    _ready(sess)
+    sess.verify(np.array([[5, 6, 7, 8]] * 3), np.array([4, 1, 0]))
+    kv0, p0 = sess.state()
+    draft = np.array([[9, 10, 11, 12], [13, 14, 15, 16], [17, 18, 19, 20]])
+    lens = np.array([4, 3, 2])
+    a = sess.verify(draft, lens)
+    la = sess.debug_logits(15).cpu().numpy().copy()
+    sess.rollback(kv0, p0)
+    b = sess.verify(draft, lens)
+    lb = sess.debug_logits(15).cpu().numpy()
+    for f in ("accepted", "bonus", "kv_len", "anchor"):
+        assert list(getattr(a, f)) == list(getattr(b, f))
+    assert np.array_equal(la, lb)
+    # rollback beyond the committed length is refused
+    kv, pe = sess.state()
+    sess.rollback(kv + 1, pe)
+    assert sess.status() & 4
+    kv2, _ = sess.state()
+    assert list(kv2) == list(kv)
+    assert sess.status() == 0
+
+
+def test_host_io_matches_device_io(built_lib, cuda):
+    from paper_2608_12703_gb300.session import Session
+    blob = W.make_weights(DIMS, std=0.3)
+    outs = []
+    for host in (False, True):
+        s = Session(DIMS, blob, max_batch=3, max_draft=4)
+        s.set_host_io(host)
+        _ready(s)
+        res = []
+        for r in range(4):
+            o = s.verify(np.array([[r, 2, 3, 4]] * 3), np.array([4, 2, r % 2 - 1]))
+            res.append((list(o.accepted), list(o.bonus), list(o.kv_len), list(o.anchor)))
+        outs.append(res)
+        assert s.status() == 0
+        s.close()
+    assert outs[0] == outs[1]

@@ -1,0 +1,23 @@
+"""Kernel test of the GEMMs: tcgen05 (one pass and split-K) and SIMT against a
+plain PyTorch fp32 matmul of the same bf16 operands."""
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+SHAPES = [(128, 16, 64), (300, 9, 1280), (3840, 9, 1280), (1280, 40, 5120), (517, 200, 384),
+          (1024, 256, 768), (640, 448, 1280), (51866, 9, 1280), (256, 137, 3072)]
+
+
+@pytest.mark.parametrize("impl", [0, 2, 1])
+@pytest.mark.parametrize("M,N,K", SHAPES)
+def test_gemm_matches_torch(built_lib, cuda, impl, M, N, K):
+    from paper_2608_12703_gb300 import asrspec as A
+    g = torch.Generator(device="cpu").manual_seed(M * 7 + N * 3 + K)
+    a = torch.randn(M, K, generator=g).to(torch.bfloat16).to(cuda)
+    b = torch.randn(N, K, generator=g).to(torch.bfloat16).to(cuda)
+    c = torch.full((M, N), float("nan"), device=cuda)
+    A.asr_spec_test_gemm(impl, a, b, c, M, N, K, torch.cuda.current_stream().cuda_stream)
+    ref = a.float() @ b.float().T
+    err = (c - ref).abs().max().item()
+    assert err <= 1e-4 * K ** 0.5 * 4, err
