@@ -92,8 +92,9 @@ typedef struct {
 } asr_weights;
 
 /* Create a handle: validate dims, allocate device weights, caches and
- * work buffers, upload the weights.  stream: a cudaStream_t (NULL = the
- * legacy default stream) on which every later call is ordered.  Synchronous.
+ * work buffers, upload the weights.  stream: a cudaStream_t on which every
+ * later call is ordered; NULL makes the handle create its own blocking stream,
+ * which is ordered with work on the legacy default stream.  Synchronous.
  * Errors: ASR_E_INVAL (dims), ASR_E_OOM, ASR_E_CUDA. */
 int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void* stream,
                     asr_spec_handle* out);
@@ -164,6 +165,26 @@ const char* asr_spec_last_error(asr_spec_handle h);
 
 /* Free every device buffer of the handle.  NULL is a no-op. */
 void asr_spec_destroy(asr_spec_handle h);
+
+/* ---- Execution and measurement controls (not part of the paper's method) --
+ * asr_spec_set_graphs: replay each (B, k) verify body as a captured CUDA graph
+ * (default 1) or launch its kernels one by one (0).
+ * asr_spec_profile: when enabled, verify launches its kernels directly and
+ * brackets each kernel class with CUDA events on the handle's stream.
+ * asr_spec_profile_read: synchronise, then return per class the summed event
+ * time in ms (ms[ASR_PROF_N]), the kernel launches since the last read
+ * (launches[ASR_PROF_N]), and the algorithmic traffic counters
+ * (traffic[8]: verify calls, self K/V bytes, encoder K/V bytes, anchor key
+ * bytes, scored rows; weight bytes follow from the dims), then reset all. */
+#define ASR_PROF_PROJ 0    /* decoder projection GEMMs */
+#define ASR_PROF_SELF 1    /* self-attention (chunk + merge kernels) */
+#define ASR_PROF_CROSS 2   /* cross-attention (chunk + merge kernels) */
+#define ASR_PROF_LMHEAD 3  /* LM head with fused argmax */
+#define ASR_PROF_OTHER 4   /* row plan, embedding, LayerNorm, accept, anchor */
+#define ASR_PROF_N 5
+int asr_spec_set_graphs(asr_spec_handle h, int enable);
+int asr_spec_profile(asr_spec_handle h, int enable);
+int asr_spec_profile_read(asr_spec_handle h, double* ms, int64_t* launches, uint64_t* traffic);
 
 /* ---- Workload utility (not part of the paper's method) -------------------
  * Synthetic draft source used by benchmarks in place of a trained draft

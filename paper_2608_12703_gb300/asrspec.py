@@ -26,8 +26,9 @@ EXPORTED = [
     "asr_spec_create", "asr_spec_set_host_io", "asr_spec_encode_cache", "asr_spec_prefill",
     "asr_spec_verify", "asr_spec_rollback", "asr_spec_state", "asr_spec_debug_logits",
     "asr_spec_status", "asr_spec_last_error", "asr_spec_destroy", "asr_spec_synth_drafts",
-    "asr_spec_test_gemm",
+    "asr_spec_test_gemm", "asr_spec_set_graphs", "asr_spec_profile", "asr_spec_profile_read",
 ]
+PROF_CLASSES = ["proj_gemm", "self_attn", "cross_attn", "lm_head", "other"]
 
 
 class AsrModelDims(ctypes.Structure):
@@ -72,6 +73,9 @@ def lib():
     L.asr_spec_destroy.restype = None
     L.asr_spec_synth_drafts.argtypes = [vp, p32, p32, p32, i32, p32, i32, p32, p32]
     L.asr_spec_test_gemm.argtypes = [i32, vp, vp, vp, i32, i32, i32, vp]
+    L.asr_spec_set_graphs.argtypes = [vp, ctypes.c_int]
+    L.asr_spec_profile.argtypes = [vp, ctypes.c_int]
+    L.asr_spec_profile_read.argtypes = [vp, vp, vp, vp]
     for name in EXPORTED:
         if name not in ("asr_spec_last_error", "asr_spec_destroy"):
             getattr(L, name).restype = ctypes.c_int
@@ -160,3 +164,21 @@ def asr_spec_test_gemm(impl, A, B, C, M, N, K, stream=None):
     return _check(None, lib().asr_spec_test_gemm(impl, ptr(A), ptr(B), ptr(C), M, N, K,
                                                  None if stream is None else ctypes.c_void_p(stream)),
                   "asr_spec_test_gemm")
+
+
+def asr_spec_set_graphs(h, enable: bool):
+    return _check(h, lib().asr_spec_set_graphs(h, int(enable)), "asr_spec_set_graphs")
+
+
+def asr_spec_profile(h, enable: bool):
+    return _check(h, lib().asr_spec_profile(h, int(enable)), "asr_spec_profile")
+
+
+def asr_spec_profile_read(h):
+    """Returns (ms per class, launches per class, traffic counters)."""
+    ms = np.zeros(len(PROF_CLASSES), dtype=np.float64)
+    launches = np.zeros(len(PROF_CLASSES), dtype=np.int64)
+    traffic = np.zeros(8, dtype=np.uint64)
+    _check(h, lib().asr_spec_profile_read(h, ms.ctypes.data, launches.ctypes.data, traffic.ctypes.data),
+           "asr_spec_profile_read")
+    return ms, launches, traffic

@@ -30,6 +30,7 @@ struct asr_spec {
   bool bf16 = true;
   size_t es = 2;  // element size of weights / caches / GEMM inputs
   cudaStream_t st = nullptr;
+  bool own_stream = false;
   int host_io = 0;
   int state = 0;  // 0 created, 1 encoder cache built, 2 prefilled
   int B = 0, t_max = 0;
@@ -58,6 +59,23 @@ struct asr_spec {
   int* tickets = nullptr;
   int n_tickets = 0;
   std::map<std::pair<int, int>, CUtensorMap> bmaps;  // (buffer id, BN) -> map
+
+  // profiling: CUDA events around each kernel class (direct launches only)
+  bool prof = false;
+  bool capturing = false;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  std::vector<std::pair<int, size_t>> marks;      // (class, index of start event)
+  long long launches[ASR_PROF_N] = {};
+  long long cur[ASR_PROF_N] = {};                 // launches of the call being enqueued
+  unsigned long long* counters = nullptr;         // device traffic counters [8]
+  // CUDA graphs of the verify body, keyed by (B, k)
+  bool use_graphs = true;
+  struct Graph {
+    cudaGraphExec_t exec;
+    long long launches[ASR_PROF_N];
+  };
+  std::map<std::pair<int, int>, Graph> graphs;
 };
 
 namespace {
@@ -66,6 +84,42 @@ int fail(asr_spec* h, int code, const std::string& msg) {
   if (h) h->err = msg;
   return code;
 }
+
+cudaEvent_t next_event(asr_spec* h) {
+  if (h->ev_used == h->ev_pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    h->ev_pool.push_back(e);
+  }
+  return h->ev_pool[h->ev_used++];
+}
+
+// Counts the launches of one kernel class and, when profiling, brackets them
+// with CUDA events on the handle's stream.
+struct Prof {
+  asr_spec* h;
+  int cls;
+  size_t idx = 0;
+  bool on = false;
+  Prof(asr_spec* h_, int cls_, int n_launch) : h(h_), cls(cls_) {
+    h->cur[cls] += n_launch;
+    if (h->prof && !h->capturing) {
+      cudaEvent_t e1 = next_event(h);
+      cudaEvent_t e2 = next_event(h);
+      if (e1 && e2) {
+        idx = h->ev_used - 2;
+        cudaEventRecord(e1, h->st);
+        on = true;
+      }
+    }
+  }
+  ~Prof() {
+    if (on) {
+      cudaEventRecord(h->ev_pool[idx + 1], h->st);
+      h->marks.emplace_back(cls, idx);
+    }
+  }
+};
 
 #define CK(call)                                                                       \
   do {                                                                                 \
@@ -128,6 +182,7 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   Epi epi = epi_in;
   epi.M = M;
   epi.N = N;
+  Prof p(h, (mode == EPI_ARGMAX || mode == EPI_F32) ? ASR_PROF_LMHEAD : ASR_PROF_PROJ, 1);
   if (!h->bf16) {
     launch_gemm_simt(W, 0, X, 0, M, N, K, mode, epi, h->st);
     return 0;
@@ -167,7 +222,10 @@ int run_layers(asr_spec* h, int N) {
   base.n_heads = h->H;
   const size_t self_layer = (size_t)h->Bmax * h->H * h->maxpos * 64 * h->es;
   const size_t cross_half = (size_t)h->Bmax * h->H * h->Tmax * 64 * h->es;
-  launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st);
+  {
+    Prof p(h, ASR_PROF_OTHER, 1);
+    launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st);
+  }
   for (int l = 0; l < h->L; ++l) {
     LayerW& w = h->lw[l];
     char* ks = static_cast<char*>(h->kself) + l * self_layer;
@@ -175,7 +233,10 @@ int run_layers(asr_spec* h, int N) {
     char* kx = static_cast<char*>(h->xkv) + (size_t)l * 2 * cross_half;
     char* vx = kx + cross_half;
     // self-attention block
-    launch_layernorm(h->x, w.ln1g, w.ln1b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+    {
+      Prof p(h, ASR_PROF_OTHER, 1);
+      launch_layernorm(h->x, w.ln1g, w.ln1b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+    }
     Epi e = base;
     e.bias = w.bqkv;
     e.out_f32 = h->q;
@@ -202,13 +263,19 @@ int run_layers(asr_spec* h, int N) {
     a.out = h->att;
     a.out_bf16 = h->bf16;
     a.ml_out = nullptr;
-    launch_attention(a, h->st);
+    {
+      Prof p(h, ASR_PROF_SELF, 2);
+      launch_attention(a, h->st);
+    }
     e = base;
     e.bias = w.bo;
     e.x = h->x;
     if (int rc = gemm_rows(h, w.wo, &w.m_wo, d, d, h->att, BUF_ATT, N, EPI_RESID, e)) return rc;
     // cross-attention block
-    launch_layernorm(h->x, w.ln2g, w.ln2b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+    {
+      Prof p(h, ASR_PROF_OTHER, 1);
+      launch_layernorm(h->x, w.ln2g, w.ln2b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+    }
     float* qc = (l == h->anchor) ? h->q_anchor : h->q;
     e = base;
     e.bias = w.bcq;
@@ -221,13 +288,19 @@ int run_layers(asr_spec* h, int N) {
     a.causal = 0;
     a.n_chunks = (h->Tmax + a.chunk - 1) / a.chunk;
     a.ml_out = (l == h->anchor) ? h->ml : nullptr;
-    launch_attention(a, h->st);
+    {
+      Prof p(h, ASR_PROF_CROSS, 2);
+      launch_attention(a, h->st);
+    }
     e = base;
     e.bias = w.bco;
     e.x = h->x;
     if (int rc = gemm_rows(h, w.wco, &w.m_wco, d, d, h->att, BUF_ATT, N, EPI_RESID, e)) return rc;
     // MLP block
-    launch_layernorm(h->x, w.ln3g, w.ln3b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+    {
+      Prof p(h, ASR_PROF_OTHER, 1);
+      launch_layernorm(h->x, w.ln3g, w.ln3b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+    }
     e = base;
     e.bias = w.b1;
     e.act = h->hbuf;
@@ -256,6 +329,42 @@ int copy_out(asr_spec* h, int32_t* dst, const int* src, size_t n) {
   return 0;
 }
 
+// The verify body on the handle's stream: rows, decoder layers, LM head with
+// fused argmax, acceptance and commit, anchor readout.  Reads the internal
+// draft/lens buffers and writes the internal output block.
+int enqueue_verify(asr_spec* h, int k) {
+  const int B = h->B;
+  {
+    Prof p(h, ASR_PROF_OTHER, 1);
+    TrafficArgs tr{h->counters, h->enc_len, h->L, h->d, (int)h->es};
+    launch_plan_verify(h->draft_buf, h->lens_buf, k, B, h->V, h->maxpos, h->kv_len, h->pending, h->ready, h->plan,
+                       h->row_key, h->status, tr, h->st);
+  }
+  const int N = B * (k + 1);
+  if (int rc = run_layers(h, N)) return rc;
+  {
+    Prof p(h, ASR_PROF_OTHER, 1);
+    launch_layernorm(h->x, h->lnf_g, h->lnf_b, h->xf, h->bf16, h->plan.n_rows, N, h->d, h->st);
+  }
+  Epi e{};
+  e.n_valid = h->plan.n_rows;
+  e.row_key = h->row_key;
+  e.d = h->d;
+  if (int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, N, EPI_ARGMAX, e)) return rc;
+  int* o_acc = h->out4;
+  int* o_bonus = h->out4 + h->Bmax;
+  int* o_len = h->out4 + 2 * h->Bmax;
+  int* o_anchor = h->out4 + 3 * h->Bmax;
+  Prof p(h, ASR_PROF_OTHER, 2);
+  launch_accept(h->draft_buf, h->lens_buf, k, B, h->plan, h->row_key, h->kv_len, h->pending, o_acc, o_bonus, o_len,
+                h->anchor_row, o_anchor, h->st);
+  const size_t cross_half = (size_t)h->Bmax * h->H * h->Tmax * 64 * h->es;
+  const char* kx = static_cast<const char*>(h->xkv) + (size_t)h->anchor * 2 * cross_half;
+  launch_anchor(h->q_anchor, h->ml, kx, h->bf16, h->Tmax, h->enc_len, h->anchor_row, B, h->H, h->d, h->frame_key,
+                reinterpret_cast<int*>(h->frame_key + h->Bmax), o_anchor, h->st);
+  return 0;
+}
+
 }  // namespace
 
 extern "C" {
@@ -279,10 +388,20 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   h->bf16 = dims->dtype == 1;
   h->es = h->bf16 ? 2 : 4;
   h->st = static_cast<cudaStream_t>(stream);
+  if (!h->st) {
+    // A blocking stream of our own: ordered with the legacy default stream,
+    // and capturable into CUDA graphs (the legacy stream itself is not).
+    if (cudaStreamCreate(&h->st) != cudaSuccess) {
+      delete h;
+      return ASR_E_CUDA;
+    }
+    h->own_stream = true;
+  }
   const int d = h->d, F = h->F, L = h->L;
   const size_t per_layer = 8 * (size_t)d * d + 13 * (size_t)d + 2 * (size_t)F * d + F;
   const size_t expect = (size_t)h->V * d + (size_t)h->maxpos * d + L * per_layer + 2 * (size_t)d;
   if (weights->n_floats != expect) {
+    if (h->own_stream) cudaStreamDestroy(h->st);
     delete h;
     return ASR_E_INVAL;
   }
@@ -433,6 +552,10 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   h->n_tickets = 8192;
   if ((rc = dalloc(h, &h->ws, h->ws_floats * 4)) || (rc = dalloc(h, &h->tickets, h->n_tickets * 4))) return finish(rc);
   CK(cudaMemset(h->tickets, 0, h->n_tickets * 4));
+  if ((rc = dalloc(h, &h->counters, 8 * sizeof(unsigned long long)))) return finish(rc);
+  CK(cudaMemset(h->counters, 0, 8 * sizeof(unsigned long long)));
+  configure_gemm_tc();
+  configure_attention();
   CK(cudaDeviceSynchronize());
   return finish(0);
 }
@@ -519,32 +642,76 @@ int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens
     if (int rc = copy_in(h, h->draft_buf, draft, (size_t)B * k)) return rc;
   }
   if (int rc = copy_in(h, h->lens_buf, lens, B)) return rc;
-  launch_plan_verify(h->draft_buf, h->lens_buf, k, B, h->V, h->maxpos, h->kv_len, h->pending, h->ready, h->plan,
-                     h->row_key, h->status, h->st);
-  const int N = B * (k + 1);
-  if (int rc = run_layers(h, N)) return rc;
-  launch_layernorm(h->x, h->lnf_g, h->lnf_b, h->xf, h->bf16, h->plan.n_rows, N, h->d, h->st);
-  Epi e{};
-  e.n_valid = h->plan.n_rows;
-  e.row_key = h->row_key;
-  e.d = h->d;
-  if (int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, N, EPI_ARGMAX, e)) return rc;
-  int* o_acc = h->out4;
-  int* o_bonus = h->out4 + h->Bmax;
-  int* o_len = h->out4 + 2 * h->Bmax;
-  int* o_anchor = h->out4 + 3 * h->Bmax;
-  launch_accept(h->draft_buf, h->lens_buf, k, B, h->plan, h->row_key, h->kv_len, h->pending, o_acc, o_bonus, o_len,
-                h->anchor_row, o_anchor, h->st);
-  const size_t cross_half = (size_t)h->Bmax * h->H * h->Tmax * 64 * h->es;
-  const char* kx = static_cast<const char*>(h->xkv) + (size_t)h->anchor * 2 * cross_half;
-  launch_anchor(h->q_anchor, h->ml, kx, h->bf16, h->Tmax, h->enc_len, h->anchor_row, B, h->H, h->d, h->frame_key,
-                reinterpret_cast<int*>(h->frame_key + h->Bmax), o_anchor, h->st);
+  for (int c = 0; c < ASR_PROF_N; ++c) h->cur[c] = 0;
+  if (h->use_graphs && !h->prof) {
+    auto key = std::make_pair(B, (int)k);
+    auto it = h->graphs.find(key);
+    if (it == h->graphs.end()) {
+      cudaGraph_t graph;
+      CK(cudaStreamBeginCapture(h->st, cudaStreamCaptureModeThreadLocal));
+      h->capturing = true;
+      int rc = enqueue_verify(h, k);
+      h->capturing = false;
+      cudaError_t e = cudaStreamEndCapture(h->st, &graph);
+      if (rc) return rc;
+      if (e != cudaSuccess) return fail(h, ASR_E_CUDA, std::string("stream capture: ") + cudaGetErrorString(e));
+      asr_spec::Graph g{};
+      e = cudaGraphInstantiate(&g.exec, graph, 0);
+      cudaGraphDestroy(graph);
+      if (e != cudaSuccess) return fail(h, ASR_E_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(e));
+      for (int c = 0; c < ASR_PROF_N; ++c) g.launches[c] = h->cur[c];
+      it = h->graphs.emplace(key, g).first;
+    }
+    CK(cudaGraphLaunch(it->second.exec, h->st));
+    for (int c = 0; c < ASR_PROF_N; ++c) h->launches[c] += it->second.launches[c];
+  } else {
+    if (int rc = enqueue_verify(h, k)) return rc;
+    for (int c = 0; c < ASR_PROF_N; ++c) h->launches[c] += h->cur[c];
+  }
   CK(cudaGetLastError());
-  if (int rc = copy_out(h, accepted, o_acc, B)) return rc;
-  if (int rc = copy_out(h, bonus, o_bonus, B)) return rc;
-  if (int rc = copy_out(h, kv_len, o_len, B)) return rc;
-  if (int rc = copy_out(h, anchor, o_anchor, B)) return rc;
+  int* o = h->out4;
+  if (int rc = copy_out(h, accepted, o, B)) return rc;
+  if (int rc = copy_out(h, bonus, o + h->Bmax, B)) return rc;
+  if (int rc = copy_out(h, kv_len, o + 2 * h->Bmax, B)) return rc;
+  if (int rc = copy_out(h, anchor, o + 3 * h->Bmax, B)) return rc;
   if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
+}
+
+int asr_spec_set_graphs(asr_spec_handle h, int enable) {
+  if (!h) return ASR_E_INVAL;
+  h->use_graphs = enable != 0;
+  return ASR_OK;
+}
+
+int asr_spec_profile(asr_spec_handle h, int enable) {
+  if (!h) return ASR_E_INVAL;
+  h->prof = enable != 0;
+  return ASR_OK;
+}
+
+int asr_spec_profile_read(asr_spec_handle h, double* ms, int64_t* launches, uint64_t* traffic) {
+  if (!h) return ASR_E_INVAL;
+  CK(cudaStreamSynchronize(h->st));
+  if (ms) {
+    for (int c = 0; c < ASR_PROF_N; ++c) ms[c] = 0.0;
+    for (auto& m : h->marks) {
+      float t = 0.f;
+      CK(cudaEventElapsedTime(&t, h->ev_pool[m.second], h->ev_pool[m.second + 1]));
+      ms[m.first] += t;
+    }
+  }
+  if (launches)
+    for (int c = 0; c < ASR_PROF_N; ++c) launches[c] = h->launches[c];
+  if (traffic) {
+    unsigned long long tmp[8];
+    CK(cudaMemcpy(tmp, h->counters, sizeof(tmp), cudaMemcpyDeviceToHost));
+    for (int i = 0; i < 8; ++i) traffic[i] = tmp[i];
+  }
+  h->marks.clear();
+  h->ev_used = 0;
+  for (int c = 0; c < ASR_PROF_N; ++c) h->launches[c] = 0;
+  CK(cudaMemset(h->counters, 0, 8 * sizeof(unsigned long long)));
   return ASR_OK;
 }
 
@@ -608,7 +775,10 @@ const char* asr_spec_last_error(asr_spec_handle h) { return h ? h->err.c_str() :
 void asr_spec_destroy(asr_spec_handle h) {
   if (!h) return;
   cudaStreamSynchronize(h->st);
+  for (auto& g : h->graphs) cudaGraphExecDestroy(g.second.exec);
+  for (cudaEvent_t e : h->ev_pool) cudaEventDestroy(e);
   for (void* p : h->allocs) cudaFree(p);
+  if (h->own_stream) cudaStreamDestroy(h->st);
   delete h;
 }
 

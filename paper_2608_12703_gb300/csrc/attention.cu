@@ -155,14 +155,16 @@ static size_t attn_smem() {
   return (size_t)2 * CHUNK * 64 * sizeof(T) + (size_t)ATTN_MAX_ROWS * 64 * 4 + (size_t)ATTN_MAX_ROWS * CHUNK * 4;
 }
 
+void configure_attention() {
+  cudaFuncSetAttribute(attn_chunk_kernel<__nv_bfloat16, 256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)attn_smem<__nv_bfloat16, 256>());
+  cudaFuncSetAttribute(attn_chunk_kernel<float, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)attn_smem<float, 128>());
+}
+
 template <typename T, int CHUNK>
 static void launch_attn_t(const AttnArgs& a, cudaStream_t st) {
-  static bool configured = false;
   const size_t sm = attn_smem<T, CHUNK>();
-  if (!configured) {
-    cudaFuncSetAttribute(attn_chunk_kernel<T, CHUNK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-    configured = true;
-  }
   dim3 grid(a.n_chunks, a.H, a.B);
   attn_chunk_kernel<T, CHUNK><<<grid, ATTN_THREADS, sm, st>>>(a);
   dim3 mgrid(a.k1, a.H, a.B);

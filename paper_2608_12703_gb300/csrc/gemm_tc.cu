@@ -244,11 +244,6 @@ size_t tc_smem_bytes(int bn) {
 template <int BN, int MODE>
 static void launch_tc_t(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
   auto kern = gemm_tc_kernel<BN, MODE>;
-  static bool configured = false;
-  if (!configured) {
-    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
-    configured = true;
-  }
   dim3 grid((g.M + TC_BM - 1) / TC_BM, (g.N + BN - 1) / BN, g.splits);
   kern<<<grid, 128, TcCfg<BN>::SMEM, st>>>(g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
 }
@@ -262,6 +257,31 @@ static void launch_tc_mode(const TcGemm& g, const Epi& epi, int* status, cudaStr
     case 128: launch_tc_t<128, MODE>(g, epi, status, st); break;
     default: launch_tc_t<256, MODE>(g, epi, status, st); break;
   }
+}
+
+template <int MODE>
+static void configure_mode() {
+  cudaFuncSetAttribute(gemm_tc_kernel<16, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<16>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<32, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<32>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<64, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<64>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<128, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<128>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<256, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<256>::SMEM);
+}
+
+// Opt every instance into its dynamic shared memory once, before any launch or
+// stream capture.
+void configure_gemm_tc() {
+  static std::once_flag once;
+  std::call_once(once, [] {
+    configure_mode<EPI_F32>();
+    configure_mode<EPI_F32_MN>();
+    configure_mode<EPI_QKV>();
+    configure_mode<EPI_RESID>();
+    configure_mode<EPI_Q>();
+    configure_mode<EPI_GELU>();
+    configure_mode<EPI_CROSSKV>();
+    configure_mode<EPI_ARGMAX>();
+  });
 }
 
 void launch_gemm_tc(const TcGemm& g, int mode, const Epi& epi, int* status, cudaStream_t st) {

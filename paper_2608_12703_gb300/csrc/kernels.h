@@ -26,6 +26,8 @@ bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
 int tc_pick_bn(int n_max);
 void launch_gemm_tc(const TcGemm& g, int mode, const Epi& epi, int* status, cudaStream_t st);
 size_t tc_smem_bytes(int bn);
+void configure_gemm_tc();
+void configure_attention();
 
 // SIMT path (fp32 models, and a cross-check of the tensor-core path).
 // A: [M][K] of type a_bf16 ? bf16 : fp32; B: [N][K] likewise.
@@ -43,10 +45,19 @@ struct RowPlan {
   int* n_utt_rows;  // [B_max] rows of utterance b this step (lens+1, or 0)
 };
 
+// Per-step algorithmic traffic, accumulated on the device (bench support):
+// counters[0] verify calls, [1] self K/V bytes, [2] cross K/V bytes,
+// [3] anchor key bytes, [4] scored rows.
+struct TrafficArgs {
+  unsigned long long* counters;
+  const int* enc_len;
+  int n_layers, d, elem_bytes;
+};
+
 // Validate the step's inputs, lay out the rows and reset the argmax keys.
 void launch_plan_verify(const int* draft, const int* lens, int k, int B, int vocab, int max_pos, const int* kv_len,
                         const int* pending, const int* ready, RowPlan plan, unsigned long long* row_key,
-                        int* status, cudaStream_t st);
+                        int* status, const TrafficArgs& tr, cudaStream_t st);
 void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,
                                RowPlan plan, int* status, cudaStream_t st);
 void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,

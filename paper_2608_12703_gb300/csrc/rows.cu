@@ -40,9 +40,11 @@ __device__ int block_excl_scan(int v, int* total) {
 __global__ void __launch_bounds__(PLAN_THREADS)
 plan_verify_kernel(const int* __restrict__ draft, const int* __restrict__ lens, int k, int B, int vocab, int max_pos,
                    const int* __restrict__ kv_len, const int* __restrict__ pending, const int* __restrict__ ready,
-                   RowPlan plan, unsigned long long* row_key, int* status) {
+                   RowPlan plan, unsigned long long* row_key, int* status, TrafficArgs tr) {
   __shared__ int s_err;
+  __shared__ unsigned long long s_cnt[4];
   if (threadIdx.x == 0) s_err = 0;
+  if (threadIdx.x < 4) s_cnt[threadIdx.x] = 0;
   __syncthreads();
   const int b = threadIdx.x;
   int n_b = 0, err = 0;
@@ -78,10 +80,26 @@ plan_verify_kernel(const int* __restrict__ draft, const int* __restrict__ lens, 
       plan.row_tok[r] = i == 0 ? pending[b] : draft[(size_t)b * k + i - 1];
       row_key[r] = 0ull;
     }
+    if (n_b > 0 && tr.counters) {
+      // algorithmic bytes of this utterance: self K/V read over the visible
+      // keys of all layers, encoder K/V read by cross-attention, and one
+      // anchor-layer key pass
+      const unsigned long long es = (unsigned long long)tr.elem_bytes, d = tr.d, L = tr.n_layers;
+      const unsigned long long T = (unsigned long long)tr.enc_len[b];
+      atomicAdd(&s_cnt[0], 2ull * L * (unsigned long long)(kv_len[b] + n_b) * d * es);
+      atomicAdd(&s_cnt[1], 2ull * L * T * d * es);
+      atomicAdd(&s_cnt[2], T * d * es);
+      atomicAdd(&s_cnt[3], (unsigned long long)n_b);
+    }
   }
+  __syncthreads();
   if (threadIdx.x == 0) {
     plan.row_start[B] = total;
     *plan.n_rows = total;
+    if (tr.counters) {
+      atomicAdd(tr.counters + 0, 1ull);
+      for (int c = 0; c < 4; ++c) atomicAdd(tr.counters + 1 + c, s_cnt[c]);
+    }
   }
 }
 
@@ -126,9 +144,9 @@ plan_prefill_kernel(const int* __restrict__ prompt, int P0, int p0, int c, int B
 
 void launch_plan_verify(const int* draft, const int* lens, int k, int B, int vocab, int max_pos, const int* kv_len,
                         const int* pending, const int* ready, RowPlan plan, unsigned long long* row_key,
-                        int* status, cudaStream_t st) {
+                        int* status, const TrafficArgs& tr, cudaStream_t st) {
   plan_verify_kernel<<<1, PLAN_THREADS, 0, st>>>(draft, lens, k, B, vocab, max_pos, kv_len, pending, ready, plan,
-                                                 row_key, status);
+                                                 row_key, status, tr);
 }
 
 void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,

@@ -38,8 +38,9 @@ class Session:
             raise A.AsrSpecError("a CUDA device is required")
         self.dims = dims
         self.dev = torch.device(device)
-        self.stream = torch.cuda.current_stream(self.dev)
-        self.h = A.asr_spec_create(dims_dict(dims, max_batch, max_draft), blob, self.stream.cuda_stream)
+        # the handle runs on its own blocking stream, ordered with torch's
+        # default stream on which the tensors below are filled and read
+        self.h = A.asr_spec_create(dims_dict(dims, max_batch, max_draft), blob, None)
         self.max_batch, self.max_draft = max_batch, max_draft
         self.B = 0
         i32 = dict(dtype=torch.int32, device=self.dev)

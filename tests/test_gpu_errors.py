@@ -17,7 +17,7 @@ DIMS = W.ModelDims(n_layers=2, d_model=128, n_heads=2, d_ffn=256, vocab=500, dty
 @pytest.fixture
 def sess(built_lib, cuda):
     from paper_2608_12703_gb300.session import Session
-    blob = W.make_weights(DIMS, std=0.3)
+    blob = W.make_weights(DIMS, std=0.1)
     s = Session(DIMS, blob, max_batch=3, max_draft=4)
     yield s
     s.close()
@@ -94,7 +94,7 @@ def test_rollback_then_reverify_is_bitwise_identical(sess):
 
 def test_host_io_matches_device_io(built_lib, cuda):
     from paper_2608_12703_gb300.session import Session
-    blob = W.make_weights(DIMS, std=0.3)
+    blob = W.make_weights(DIMS, std=0.1)
     outs = []
     for host in (False, True):
         s = Session(DIMS, blob, max_batch=3, max_draft=4)
@@ -108,3 +108,28 @@ def test_host_io_matches_device_io(built_lib, cuda):
         assert s.status() == 0
         s.close()
     assert outs[0] == outs[1]
+
+
+def test_graph_replay_matches_direct_launch_and_profile(built_lib, cuda):
+    from paper_2608_12703_gb300 import asrspec as A
+    from paper_2608_12703_gb300.session import Session
+    blob = W.make_weights(DIMS, std=0.1)
+    outs = []
+    for graphs, prof in ((True, False), (False, False), (True, True)):
+        s = Session(DIMS, blob, max_batch=3, max_draft=4)
+        A.asr_spec_set_graphs(s.h, graphs)
+        A.asr_spec_profile(s.h, prof)
+        _ready(s)
+        A.asr_spec_profile_read(s.h)
+        res = []
+        for r in range(5):
+            o = s.verify(np.array([[r, 2, 3, 4]] * 3), np.array([4, 2, r % 2 - 1]))
+            res.append((list(o.accepted), list(o.bonus), list(o.kv_len), list(o.anchor)))
+        ms, launches, traffic = A.asr_spec_profile_read(s.h)
+        assert traffic[0] == 5 and launches.sum() > 0
+        if prof:
+            assert ms[A.PROF_CLASSES.index("proj_gemm")] > 0
+        outs.append(res)
+        assert s.status() == 0
+        s.close()
+    assert outs[0] == outs[1] == outs[2]
