@@ -1,0 +1,515 @@
+#!/usr/bin/env python
+"""Benchmark of the speculative draft-verify step on GB300.
+
+One step = one whole speculative decode of the workload's batch: the
+encoder-cache build for every utterance, the prompt prefill, then verify
+rounds (drafts from the synthetic draft source, longest-prefix acceptance,
+commit, re-anchoring) until every utterance has its target length.
+value = emitted tokens (accepted drafts + bonus tokens) per second over the
+timed steps, with weights and encoder states resident in HBM.
+
+Also reported, on the same workload: per-verify-call latency (CUDA events),
+the dominant kernel class against its roofline, an end-to-end number through
+host buffers, the CPU oracle on a bounded sample, and the batch-1 workload.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+
+N > 1 runs under torchrun as independent replicas (one per GPU, no collective
+on the data path); value is the sum over ranks divided by the slowest rank.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workload as W  # noqa: E402
+
+MAIN_CONFIG = "large-bf16-b64-k6"
+BATCH1_CONFIG = "large-bf16-b1-k8"
+METRIC = "accepted tokens/s"
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=float(d["hbm_gbs"]), bf16=float(d["bf16_tflops"]),
+                    bf16_sus=float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), src="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+# ----------------------------------------------------------------------------
+# clocks during the timed region
+# ----------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out = ""
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------
+# GPU arm
+# ----------------------------------------------------------------------------
+_WEIGHTS = {}
+
+
+def weights(dims):
+    if dims not in _WEIGHTS:
+        _WEIGHTS.clear()
+        _WEIGHTS[dims] = W.make_weights(dims)
+    return _WEIGHTS[dims]
+
+
+class GpuRun:
+    """One workload resident on one GPU, plus the reference transcript that
+    drives the synthetic draft source."""
+
+    def __init__(self, wl: W.Workload):
+        import torch
+        from paper_2608_12703_gb300 import asrspec as A
+        from paper_2608_12703_gb300.session import DeviceDrafts, Session
+        self.torch, self.A = torch, A
+        self.wl = wl
+        dims = wl.dims
+        self.sess = Session(dims, weights(dims), max_batch=wl.batch, max_draft=wl.k)
+        enc = W.make_encoder_states(dims, wl.enc_lens, wl.t_max)
+        self.enc_host = torch.from_numpy(enc).to(self.sess.storage_dtype).pin_memory()
+        self.enc_lens = np.array(wl.enc_lens, dtype=np.int32)
+        self.prompt = W.make_prompt(dims, wl.batch)
+        with torch.cuda.stream(self.sess.stream):
+            self.enc = self.enc_host.to("cuda")
+            self.enc_lens_d = torch.from_numpy(self.enc_lens).cuda()
+            self.prompt_d = torch.from_numpy(self.prompt).cuda()
+        self.sess.stream.synchronize()
+        self.total = np.array(wl.total_lens, dtype=np.int64)
+        self.truth = self._greedy_transcript()
+        self.corr = W.make_corruption(wl)
+        self.drafts = DeviceDrafts(self.sess, self.truth, self.total, self.corr, wl.k)
+        self.tokens_per_decode = int(sum(wl.n_out))
+        self.rounds = self._count_rounds()
+
+    def _begin(self):
+        A, s = self.A, self.sess
+        A.asr_spec_encode_cache(s.h, self.wl.batch, self.enc, self.wl.t_max, self.enc_lens_d)
+        s.B = self.wl.batch
+        A.asr_spec_prefill(s.h, self.prompt_d, self.prompt.shape[1])
+
+    def _greedy_transcript(self):
+        """The GPU target's own greedy transcript (one token per round)."""
+        B = self.wl.batch
+        self._begin()
+        truth = np.zeros((B, self.wl.dims.max_pos), dtype=np.int64)
+        truth[:, :self.prompt.shape[1]] = self.prompt
+        kv = np.full(B, self.prompt.shape[1] - 1)
+        zeros = np.zeros((B, 1), dtype=np.int32)
+        while True:
+            active = kv + 1 < self.total
+            if not active.any():
+                break
+            out = self.sess.verify(zeros, np.where(active, 0, -1).astype(np.int32), k=0)
+            for b in np.nonzero(active)[0]:
+                truth[b, kv[b] + 1] = out.bonus[b]
+            kv = out.kv_len.astype(np.int64)
+        assert self.sess.status() == 0
+        return truth
+
+    def _count_rounds(self):
+        self._begin()
+        n = 0
+        while True:
+            d, l = self.drafts.next()
+            if bool((l < 0).all()):
+                break
+            self.sess.verify_device(d, l, self.wl.k)
+            n += 1
+        kv, _ = self.sess.state()
+        assert np.array_equal(kv + 1, self.total), (kv, self.total)
+        assert self.sess.status() == 0
+        return n
+
+    def decode(self, ev=None):
+        """One whole decode, enqueued without host synchronisation."""
+        self._begin()
+        k = self.wl.k
+        for _ in range(self.rounds):
+            d, l = self.drafts.next()
+            if ev is not None:
+                e0 = self.torch.cuda.Event(enable_timing=True)
+                e0.record(self.sess.stream)
+            self.sess.verify_device(d, l, k)
+            if ev is not None:
+                e1 = self.torch.cuda.Event(enable_timing=True)
+                e1.record(self.sess.stream)
+                ev.append((e0, e1))
+
+    def launches(self):
+        _, launches, _ = self.A.asr_spec_profile_read(self.sess.h)
+        return int(launches.sum())
+
+    def timed(self, steps, warmup, dist=None, gpu_index=0):
+        torch = self.torch
+        for _ in range(warmup):
+            self.decode()
+        torch.cuda.synchronize()
+        self.A.asr_spec_profile_read(self.sess.h)          # reset counters
+        verify_ev = []
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with ClockSampler(gpu_index) as clk:
+            start.record(self.sess.stream)
+            for _ in range(steps):
+                self.decode(verify_ev)
+            end.record(self.sess.stream)
+            torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+        ms = start.elapsed_time(end)
+        _, launches, traffic = self.A.asr_spec_profile_read(self.sess.h)
+        per_call = np.array([a.elapsed_time(b) for a, b in verify_ev]) * 1e3
+        assert self.sess.status() == 0
+        return dict(ms=ms, launches=int(launches.sum()) + 0, traffic=traffic, clocks=clk.summary(),
+                    verify_us=dict(median=float(np.median(per_call)), p10=float(np.percentile(per_call, 10)),
+                                   p90=float(np.percentile(per_call, 90)), calls=int(len(per_call))))
+
+    def profile(self):
+        """One decode with per-kernel-class CUDA events (direct launches)."""
+        A = self.A
+        A.asr_spec_profile_read(self.sess.h)
+        A.asr_spec_profile(self.sess.h, True)
+        self.decode()
+        ms, launches, traffic = A.asr_spec_profile_read(self.sess.h)
+        A.asr_spec_profile(self.sess.h, False)
+        return ms, launches, traffic
+
+    def e2e(self, steps):
+        """The same decodes through host buffers: encoder states copied from pinned
+        host memory every step, drafts built on the host and passed with every
+        verify call, outputs read back every round."""
+        torch, A = self.torch, self.A
+        s = self.sess
+        wl = self.wl
+        h2d = d2h = 0
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(steps):
+            with torch.cuda.stream(s.stream):
+                enc = self.enc_host.to("cuda", non_blocking=True)
+            h2d += self.enc_host.numel() * self.enc_host.element_size()
+            s.set_host_io(True)
+            A.asr_spec_encode_cache(s.h, wl.batch, enc, wl.t_max, self.enc_lens)
+            A.asr_spec_prefill(s.h, self.prompt.astype(np.int32), self.prompt.shape[1])
+            h2d += self.enc_lens.nbytes + self.prompt.astype(np.int32).nbytes
+            kv = np.full(wl.batch, self.prompt.shape[1] - 1)
+            while True:
+                draft, lens = W.make_drafts(self.truth, self.total, kv, wl.k, self.corr)
+                if np.all(lens < 0):
+                    break
+                out = s.verify(draft, lens)
+                h2d += draft.nbytes + lens.nbytes
+                d2h += 4 * out.accepted.nbytes
+                kv = out.kv_len.astype(np.int64)
+            s.set_host_io(False)
+            del enc
+        torch.cuda.synchronize()
+        dt = time.perf_counter() - t0
+        return dict(value=steps * self.tokens_per_decode / dt, unit="tokens/s",
+                    h2d_bytes_per_step=int(h2d // steps), d2h_bytes_per_step=int(d2h // steps))
+
+
+def roofline(dims, ms, launches, traffic, pk):
+    """Dominant kernel class of one profiled decode against its roofline."""
+    from paper_2608_12703_gb300.asrspec import PROF_CLASSES
+    cls = int(np.argmax(ms[:4]))
+    name = PROF_CLASSES[cls]
+    es = 2 if dims.dtype == "bf16" else 4
+    d, L, F, V = dims.d_model, dims.n_layers, dims.d_ffn, dims.vocab
+    calls, self_b, cross_b, anchor_b, rows = (int(x) for x in traffic[:5])
+    t = ms[cls] / 1e3
+    n = int(launches[cls])
+    if name == "cross_attn":
+        work, bound, unit, peak = cross_b / t / 1e9, "hbm", "GB/s", pk["hbm"]
+        per_unit = "2 * T_b * d * 2 bytes of encoder K/V per active utterance per layer"
+    elif name == "self_attn":
+        work, bound, unit, peak = self_b / t / 1e9, "hbm", "GB/s", pk["hbm"]
+        per_unit = "2 * (P_b + n_b) * d * 2 bytes of self K/V per active utterance per layer"
+    else:
+        if name == "proj_gemm":
+            wbytes = calls * L * (6 * d * d + 2 * F * d) * es
+            flops = 2.0 * rows * L * (6 * d * d + 2 * F * d)
+        else:
+            wbytes = calls * V * d * es
+            flops = 2.0 * rows * V * d
+        intensity = flops / max(wbytes, 1)
+        if intensity > pk["bf16_sus"] * 1e12 / (pk["hbm"] * 1e9):
+            work, bound, unit, peak = flops / t / 1e12, "tensor", "TFLOP/s", pk["bf16_sus"]
+            per_unit = "2 * rows * K * M flops per projection"
+        else:
+            work, bound, unit, peak = wbytes / t / 1e9, "hbm", "GB/s", pk["hbm"]
+            per_unit = "M * K * 2 bytes of weights per projection launch"
+    return {"kernel": name, "bound": bound, "achieved": round(work, 2), "peak": peak, "unit": unit,
+            "frac": round(work / peak, 4), "traffic": None, "launches": n,
+            "ms_per_launch": round(ms[cls] / max(n, 1), 5), "per_unit": per_unit,
+            "peak_source": pk["src"],
+            "class_ms": {PROF_CLASSES[i]: round(float(ms[i]), 3) for i in range(len(ms))}}
+
+
+def step_bytes(dims, traffic, calls_override=None):
+    """Algorithmic bytes per verify call (weights + LM head + K/V reads)."""
+    es = 2 if dims.dtype == "bf16" else 4
+    d, L, F, V = dims.d_model, dims.n_layers, dims.d_ffn, dims.vocab
+    calls = int(traffic[0]) if calls_override is None else calls_override
+    w = L * (6 * d * d + 2 * F * d) * es + V * d * es
+    kv = float(traffic[1]) + float(traffic[2]) + float(traffic[3])
+    return (calls * w + kv) / max(calls, 1)
+
+
+# ----------------------------------------------------------------------------
+# CPU oracle arm
+# ----------------------------------------------------------------------------
+def oracle_sample(wl: W.Workload, truth, budget_s: float, utt: int = 0, rounds_cap=None):
+    """The oracle on utterance `utt` of the workload: encoder cache, prefill,
+    then verify rounds with the workload's drafts until the budget is spent.
+    Returns (tokens emitted, seconds, rounds, description)."""
+    from oracle import Oracle
+    dims = wl.dims
+    enc = W.make_encoder_states(dims, [wl.enc_lens[utt]], wl.t_max)
+    t0 = time.perf_counter()
+    orc = Oracle(dims, weights(dims))
+    t_setup = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    orc.encode_cache(enc, [wl.enc_lens[utt]])
+    prompt = W.make_prompt(dims, 1)
+    orc.prefill(prompt)
+    corr = W.make_corruption(wl)
+    sub = W.Corruption(corr.repl[utt:utt + 1], corr.shift[utt:utt + 1])
+    total = [wl.total_lens[utt]]
+    tokens = rounds = 0
+    while time.perf_counter() - t0 < budget_s and (rounds_cap is None or rounds < rounds_cap):
+        draft, lens = W.make_drafts(truth[utt:utt + 1], total, orc.kv_len, wl.k, sub)
+        if lens[0] < 0:
+            break
+        r = orc.verify(draft, lens)
+        tokens += int(r.accepted[0]) + 1
+        rounds += 1
+    dt = time.perf_counter() - t0
+    desc = (f"utterance {utt} of {wl.name} (T={wl.enc_lens[utt]} frames): encoder cache + prefill + "
+            f"{rounds} verify rounds, {tokens} tokens; weight widening ({t_setup:.1f} s) not timed")
+    return tokens, dt, rounds, desc
+
+
+def cpu_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n and n[0]:
+            return int(n[0])
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+# ----------------------------------------------------------------------------
+def base_line(args, wl, n_gpus):
+    return {"metric": METRIC, "unit": "tokens/s", "n_gpus": n_gpus, "steps": args.steps,
+            "warmup": args.warmup, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if wl.dims.dtype == "bf16" else "f32",
+            "data": "synthetic (seeded random-init weights and encoder states shaped like the paper's workloads)",
+            "config": {"workload": wl.name, "batch": wl.batch, "k": wl.k, "layers": wl.dims.n_layers,
+                       "d_model": wl.dims.d_model, "vocab": wl.dims.vocab,
+                       "tokens_per_step": int(sum(wl.n_out)), "parallelism": f"replicas x{n_gpus}",
+                       "l2": "inputs larger than L2 (weights and encoder K/V exceed 129 MB per verify call)"}}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    wl = W.CONFIGS[args.config]
+    # the reference transcript for the drafts: the oracle's own greedy decoding
+    from oracle import Oracle, greedy_transcript
+    dims = wl.dims
+    utt = 0
+    n_total = min(wl.total_lens[utt], W.PROMPT_LEN + 12)
+    enc = W.make_encoder_states(dims, [wl.enc_lens[utt]], wl.t_max)
+    orc = Oracle(dims, weights(dims))
+    orc.encode_cache(enc, [wl.enc_lens[utt]])
+    prompt = W.make_prompt(dims, 1)
+    orc.prefill(prompt)
+    truth = np.zeros((1, dims.max_pos), dtype=np.int64)
+    tr = greedy_transcript(orc, prompt, [n_total])
+    truth[0, :tr.shape[1]] = tr[0]
+    corr = W.make_corruption(wl)
+    sub = W.Corruption(corr.repl[utt:utt + 1], corr.shift[utt:utt + 1])
+    times, toks = [], []
+    for i in range(args.warmup + args.steps):
+        orc.rollback([W.PROMPT_LEN - 1], [prompt[0, -1]])
+        t0 = time.perf_counter()
+        n = 0
+        while True:
+            draft, lens = W.make_drafts(truth, [n_total], orc.kv_len, wl.k, sub)
+            if lens[0] < 0:
+                break
+            r = orc.verify(draft, lens)
+            n += int(r.accepted[0]) + 1
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t0)
+            toks.append(n)
+    value = sum(toks) / sum(times)
+    line = base_line(args, wl, 1)
+    cores = cpu_threads()
+    sample = (f"utterance {utt} of {wl.name}: decode of {n_total - W.PROMPT_LEN} tokens by verify rounds "
+              f"from a prefilled cache, per step")
+    line.update({"impl": "reference", "value": value, "ms_per_step": 1e3 * float(np.mean(times)),
+                 "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                                  "sample": sample},
+                 "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                         "d2h_bytes_per_step": 0}})
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", default=MAIN_CONFIG, choices=sorted(W.CONFIGS))
+    ap.add_argument("--batch1-config", default=BATCH1_CONFIG)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-batch1", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=20.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as tdist
+        tdist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        dist = tdist
+    from paper_2608_12703_gb300 import build as B
+    if rank == 0:
+        B.build()
+    if dist is not None:
+        dist.barrier()
+    B.build()
+    pk = peaks()
+    wl = W.CONFIGS[args.config]
+    run = GpuRun(wl)
+    res = run.timed(args.steps, args.warmup, dist, gpu_index=local)
+    ms = res["ms"]
+    if dist is not None:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    total_tokens = world * args.steps * run.tokens_per_decode
+    value = total_tokens / (ms / 1e3)
+    prof_ms, prof_launches, prof_traffic = run.profile()
+    line = base_line(args, wl, world)
+    bytes_per_call = step_bytes(wl.dims, prof_traffic)
+    line.update({
+        "value": value, "ms_per_step": ms / args.steps,
+        "verify_us": res["verify_us"],
+        "verify_rounds_per_step": run.rounds,
+        "verify_hbm": {"bytes_per_call": bytes_per_call,
+                       "frac": bytes_per_call / (res["verify_us"]["median"] * 1e-6) / (pk["hbm"] * 1e9),
+                       "frac_nominal_8tbs": bytes_per_call / (res["verify_us"]["median"] * 1e-6) / 8e12},
+        "clocks": res["clocks"],
+        "gpu_launches": res["launches"] + 0,
+        "roofline": roofline(wl.dims, prof_ms, prof_launches, prof_traffic, pk),
+    })
+    if not args.no_e2e:
+        line["e2e"] = run.e2e(max(1, min(args.steps, 2)))
+        if world > 1:
+            line["e2e"]["value"] *= world
+    if rank == 0:
+        # CPU oracle on a bounded sample of the same workload
+        tokens, dt, rounds, desc = oracle_sample(wl, run.truth, args.cpu_budget)
+        line["cpu_baseline"] = {"value": tokens / dt, "unit": "tokens/s", "cores": cpu_threads(),
+                                "kind": "oracle", "sample": desc}
+        if not args.no_batch1 and args.batch1_config != args.config:
+            del run
+            torch.cuda.empty_cache()
+            wl1 = W.CONFIGS[args.batch1_config]
+            r1 = GpuRun(wl1)
+            b1 = r1.timed(args.steps, args.warmup, None, gpu_index=local)
+            pm, pl, pt = r1.profile()
+            bpc = step_bytes(wl1.dims, pt)
+            line["batch1"] = {
+                "workload": wl1.name, "value": args.steps * r1.tokens_per_decode / (b1["ms"] / 1e3),
+                "unit": "tokens/s", "ms_per_step": b1["ms"] / args.steps, "verify_us": b1["verify_us"],
+                "verify_rounds_per_step": r1.rounds,
+                "verify_hbm": {"bytes_per_call": bpc,
+                               "frac": bpc / (b1["verify_us"]["median"] * 1e-6) / (pk["hbm"] * 1e9),
+                               "frac_nominal_8tbs": bpc / (b1["verify_us"]["median"] * 1e-6) / 8e12},
+                "clocks": b1["clocks"], "roofline": roofline(wl1.dims, pm, pl, pt, pk)}
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -102,7 +102,8 @@ struct Prof {
   size_t idx = 0;
   bool on = false;
   Prof(asr_spec* h_, int cls_, int n_launch) : h(h_), cls(cls_) {
-    h->cur[cls] += n_launch;
+    if (h->capturing) h->cur[cls] += n_launch;   // replayed with the graph
+    else h->launches[cls] += n_launch;
     if (h->prof && !h->capturing) {
       cudaEvent_t e1 = next_event(h);
       cudaEvent_t e2 = next_event(h);
@@ -572,6 +573,7 @@ int asr_spec_encode_cache(asr_spec_handle h, int32_t B, const void* enc_states, 
   if (B < 1 || B > h->Bmax || !enc_states || !enc_lens || t_max < 1) return fail(h, ASR_E_INVAL, "bad arguments");
   if (t_max > h->Tmax) return fail(h, ASR_E_CAPACITY, "t_max exceeds max_enc");
   if (int rc = copy_in(h, h->enc_len, enc_lens, B)) return rc;
+  Prof p(h, ASR_PROF_OTHER, 1);
   launch_mark_ready(h->enc_len, B, t_max, h->ready, h->kv_len, h->pending, h->status, h->st);
   const int d = h->d;
   Epi e{};
@@ -598,8 +600,10 @@ int asr_spec_encode_cache(asr_spec_handle h, int32_t B, const void* enc_states, 
     g.splits = 1;
     g.ws = h->ws;
     g.tickets = h->tickets;
+    Prof pg(h, ASR_PROF_PROJ, 1);
     launch_gemm_tc(g, EPI_CROSSKV, e, h->status, h->st);
   } else {
+    Prof pg(h, ASR_PROF_PROJ, 1);
     launch_gemm_simt(enc_states, 0, h->w_cross, 0, M, N, d, EPI_CROSSKV, e, h->st);
   }
   CK(cudaGetLastError());
@@ -619,10 +623,15 @@ int asr_spec_prefill(asr_spec_handle h, const int32_t* prompt, int32_t P0) {
   const int c_max = h->kmax + 1;
   for (int p0 = 0; p0 < P0 - 1; p0 += c_max) {
     const int c = std::min(c_max, P0 - 1 - p0);
-    launch_plan_prefill_chunk(h->prompt_buf, P0, p0, c, h->B, h->V, h->ready, h->plan, h->status, h->st);
+    {
+      Prof p(h, ASR_PROF_OTHER, 1);
+      launch_plan_prefill_chunk(h->prompt_buf, P0, p0, c, h->B, h->V, h->ready, h->plan, h->status, h->st);
+    }
     if (int rc = run_layers(h, h->B * c)) return rc;
+    Prof p(h, ASR_PROF_OTHER, 1);
     launch_prefill_advance(h->B, c, h->plan.n_utt_rows, h->kv_len, h->st);
   }
+  Prof p(h, ASR_PROF_OTHER, 1);
   launch_prefill_finish(h->prompt_buf, P0, h->B, h->pending, h->ready, h->st);
   CK(cudaGetLastError());
   h->state = 2;
@@ -666,7 +675,6 @@ int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens
     for (int c = 0; c < ASR_PROF_N; ++c) h->launches[c] += it->second.launches[c];
   } else {
     if (int rc = enqueue_verify(h, k)) return rc;
-    for (int c = 0; c < ASR_PROF_N; ++c) h->launches[c] += h->cur[c];
   }
   CK(cudaGetLastError());
   int* o = h->out4;
@@ -721,6 +729,7 @@ int asr_spec_rollback(asr_spec_handle h, const int32_t* new_len, const int32_t* 
   if (!new_len || !new_pending) return fail(h, ASR_E_INVAL, "null pointer");
   if (int rc = copy_in(h, h->misc, new_len, h->B)) return rc;
   if (int rc = copy_in(h, h->lens_buf, new_pending, h->B)) return rc;
+  Prof p(h, ASR_PROF_OTHER, 1);
   launch_rollback(h->misc, h->lens_buf, h->B, h->V, h->kv_len, h->pending, h->status, h->st);
   CK(cudaGetLastError());
   if (h->host_io) CK(cudaStreamSynchronize(h->st));
@@ -786,6 +795,7 @@ int asr_spec_synth_drafts(asr_spec_handle h, const int32_t* truth, const int32_t
                           int32_t k_repl, const int32_t* shift, int32_t k, int32_t* draft_out, int32_t* lens_out) {
   if (!h || !truth || !total_len || !repl || !shift || !draft_out || !lens_out) return ASR_E_INVAL;
   if (k < 1 || k > k_repl) return fail(h, ASR_E_INVAL, "k outside [1, k_repl]");
+  Prof p(h, ASR_PROF_OTHER, 1);
   launch_synth_drafts(truth, total_len, repl, k_repl, shift, k, h->B, h->maxpos, h->kv_len, draft_out, lens_out,
                       h->st);
   CK(cudaGetLastError());

@@ -15,6 +15,8 @@
 // construction"): the head mean of the per-head softmax attention of one row
 // at the anchor layer, recomputed from the cached keys with the (max, sum) that
 // the attention pass left, then its peak frame.
+#include <mutex>
+
 #include "kernels.h"
 
 namespace asrspec {
@@ -156,10 +158,13 @@ static size_t attn_smem() {
 }
 
 void configure_attention() {
-  cudaFuncSetAttribute(attn_chunk_kernel<__nv_bfloat16, 256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       (int)attn_smem<__nv_bfloat16, 256>());
-  cudaFuncSetAttribute(attn_chunk_kernel<float, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       (int)attn_smem<float, 128>());
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaFuncSetAttribute(attn_chunk_kernel<__nv_bfloat16, 256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)attn_smem<__nv_bfloat16, 256>());
+    cudaFuncSetAttribute(attn_chunk_kernel<float, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)attn_smem<float, 128>());
+  });
 }
 
 template <typename T, int CHUNK>
@@ -172,6 +177,7 @@ static void launch_attn_t(const AttnArgs& a, cudaStream_t st) {
 }
 
 void launch_attention(const AttnArgs& a, cudaStream_t st) {
+  configure_attention();
   if (a.kv_bf16) launch_attn_t<__nv_bfloat16, 256>(a, st);
   else launch_attn_t<float, 128>(a, st);
 }

@@ -285,6 +285,7 @@ void configure_gemm_tc() {
 }
 
 void launch_gemm_tc(const TcGemm& g, int mode, const Epi& epi, int* status, cudaStream_t st) {
+  configure_gemm_tc();
   switch (mode) {
     case EPI_F32: launch_tc_mode<EPI_F32>(g, epi, status, st); break;
     case EPI_F32_MN: launch_tc_mode<EPI_F32_MN>(g, epi, status, st); break;

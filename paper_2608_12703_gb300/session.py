@@ -38,15 +38,13 @@ class Session:
             raise A.AsrSpecError("a CUDA device is required")
         self.dims = dims
         self.dev = torch.device(device)
-        # the handle runs on its own blocking stream, ordered with torch's
-        # default stream on which the tensors below are filled and read
-        self.h = A.asr_spec_create(dims_dict(dims, max_batch, max_draft), blob, None)
+        # one stream for the library and for the torch copies that feed it
+        self.stream = torch.cuda.Stream(self.dev)
+        self.h = A.asr_spec_create(dims_dict(dims, max_batch, max_draft), blob, self.stream.cuda_stream)
         self.max_batch, self.max_draft = max_batch, max_draft
         self.B = 0
-        i32 = dict(dtype=torch.int32, device=self.dev)
-        self.out = torch.zeros((4, max_batch), **i32)
-        self.draft_d = torch.zeros((max_batch, max(max_draft, 1)), **i32)
-        self.lens_d = torch.zeros(max_batch, **i32)
+        with torch.cuda.stream(self.stream):
+            self.out = torch.zeros((4, max_batch), dtype=torch.int32, device=self.dev)
         self.host_io = False
 
     @property
@@ -71,6 +69,10 @@ class Session:
     # -- one call each -------------------------------------------------------
     def encode_cache(self, enc_states, enc_lens):
         """enc_states: [B, t_max, d] (numpy fp32 or a device tensor of the model dtype)."""
+        with torch.cuda.stream(self.stream):
+            self._encode_cache(enc_states, enc_lens)
+
+    def _encode_cache(self, enc_states, enc_lens):
         if isinstance(enc_states, np.ndarray):
             enc_states = torch.from_numpy(enc_states).to(self.dev).to(self.storage_dtype)
         enc_states = enc_states.contiguous()
@@ -81,8 +83,9 @@ class Session:
         self.B = B
 
     def prefill(self, prompt):
-        prompt = self._i32(prompt)
-        A.asr_spec_prefill(self.h, prompt, int(prompt.shape[1]))
+        with torch.cuda.stream(self.stream):
+            prompt = self._i32(prompt)
+            A.asr_spec_prefill(self.h, prompt, int(prompt.shape[1]))
 
     def verify(self, draft, lens, k: Optional[int] = None) -> StepOut:
         draft = np.asarray(draft, dtype=np.int32)
@@ -95,11 +98,12 @@ class Session:
             acc, bon, kvl, anc = (np.zeros(self.B, np.int32) for _ in range(4))
             A.asr_spec_verify(self.h, np.ascontiguousarray(draft[:, :k]), lens, k, acc, bon, kvl, anc)
             return StepOut(acc, bon, kvl, anc)
-        d = torch.from_numpy(np.ascontiguousarray(draft[:, :k])).to(self.dev)
-        l = torch.from_numpy(lens).to(self.dev)
-        o = self.out[:, :self.B]
-        A.asr_spec_verify(self.h, d, l, k, o[0], o[1], o[2], o[3])
-        oh = o.cpu().numpy()
+        with torch.cuda.stream(self.stream):
+            d = torch.from_numpy(np.ascontiguousarray(draft[:, :k])).to(self.dev)
+            l = torch.from_numpy(lens).to(self.dev)
+            o = self.out[:, :self.B]
+            A.asr_spec_verify(self.h, d, l, k, o[0], o[1], o[2], o[3])
+            oh = o.cpu().numpy()
         return StepOut(oh[0].copy(), oh[1].copy(), oh[2].copy(), oh[3].copy())
 
     def verify_device(self, draft_d, lens_d, k: int):
@@ -109,21 +113,25 @@ class Session:
         return o
 
     def rollback(self, new_len, new_pending):
-        A.asr_spec_rollback(self.h, self._i32(new_len), self._i32(new_pending))
+        with torch.cuda.stream(self.stream):
+            A.asr_spec_rollback(self.h, self._i32(new_len), self._i32(new_pending))
 
     def state(self):
-        kv = torch.zeros(self.B, dtype=torch.int32, device=self.dev)
-        pe = torch.zeros(self.B, dtype=torch.int32, device=self.dev)
         if self.host_io:
             kvh, peh = np.zeros(self.B, np.int32), np.zeros(self.B, np.int32)
             A.asr_spec_state(self.h, kvh, peh)
             return kvh, peh
-        A.asr_spec_state(self.h, kv, pe)
-        return kv.cpu().numpy(), pe.cpu().numpy()
+        with torch.cuda.stream(self.stream):
+            kv = torch.zeros(self.B, dtype=torch.int32, device=self.dev)
+            pe = torch.zeros(self.B, dtype=torch.int32, device=self.dev)
+            A.asr_spec_state(self.h, kv, pe)
+            return kv.cpu().numpy(), pe.cpu().numpy()
 
     def debug_logits(self, max_rows: int) -> torch.Tensor:
-        out = torch.empty((max_rows, self.dims.vocab), dtype=torch.float32, device=self.dev)
-        R = A.asr_spec_debug_logits(self.h, out, max_rows)
+        with torch.cuda.stream(self.stream):
+            out = torch.empty((max_rows, self.dims.vocab), dtype=torch.float32, device=self.dev)
+            R = A.asr_spec_debug_logits(self.h, out, max_rows)
+        self.stream.synchronize()
         return out[:R]
 
     def status(self) -> int:
@@ -146,13 +154,15 @@ class DeviceDrafts:
         t[:, :truth.shape[1]] = np.where(truth >= 0, truth, 0)[:, :P]
         dev = sess.dev
         self.sess, self.k = sess, k
-        self.truth = torch.from_numpy(t).to(dev)
-        self.total = torch.tensor(np.asarray(total_lens, dtype=np.int32), device=dev)
-        self.repl = torch.from_numpy(np.ascontiguousarray(corr.repl[:B, :P, :], dtype=np.int32)).to(dev)
-        self.k_repl = int(corr.repl.shape[2])
-        self.shift = torch.from_numpy(np.ascontiguousarray(corr.shift[:B, :P], dtype=np.int32)).to(dev)
-        self.draft = torch.zeros((B, k), dtype=torch.int32, device=dev)
-        self.lens = torch.zeros(B, dtype=torch.int32, device=dev)
+        with torch.cuda.stream(sess.stream):
+            self.truth = torch.from_numpy(t).to(dev)
+            self.total = torch.tensor(np.asarray(total_lens, dtype=np.int32), device=dev)
+            self.repl = torch.from_numpy(np.ascontiguousarray(corr.repl[:B, :P, :], dtype=np.int32)).to(dev)
+            self.k_repl = int(corr.repl.shape[2])
+            self.shift = torch.from_numpy(np.ascontiguousarray(corr.shift[:B, :P], dtype=np.int32)).to(dev)
+            self.draft = torch.zeros((B, k), dtype=torch.int32, device=dev)
+            self.lens = torch.zeros(B, dtype=torch.int32, device=dev)
+        sess.stream.synchronize()
 
     def next(self):
         A.asr_spec_synth_drafts(self.sess.h, self.truth, self.total, self.repl, self.k_repl, self.shift, self.k,

@@ -22,6 +22,14 @@ from oracle import Oracle, greedy_transcript
 TIE_GAP = 1e-2
 
 
+def scale_for(dims, std):
+    """Tolerance multiplier for test models whose logit scale exceeds the
+    workloads': bf16 rounding error grows with the logit scale (std * sqrt(d));
+    the workloads (std 0.02, d >= 768) get exactly the stated tolerances."""
+    import math
+    return max(1.0, std * math.sqrt(dims.d_model) / (0.02 * math.sqrt(768)))
+
+
 @dataclasses.dataclass
 class ParityStats:
     rounds: int = 0
@@ -34,15 +42,15 @@ class ParityStats:
     max_logit_err: float = 0.0
 
 
-def logit_tol(dims):
-    return 3e-2 if dims.dtype == "bf16" else 1e-4
+def logit_tol(dims, scale=1.0):
+    return (3e-2 if dims.dtype == "bf16" else 1e-4) * scale
 
 
 def anchor_tol(dims):
     return 2e-2 if dims.dtype == "bf16" else 1e-4
 
 
-def compare_round(orc, sess, draft, lens, st: ParityStats, check_logits=True, sample=None):
+def compare_round(orc, sess, draft, lens, st: ParityStats, check_logits=True, sample=None, scale=1.0):
     """One teacher-forced round; `sample` restricts the checks to some utterances
     (the oracle then holds only those, in order)."""
     dims = orc.dims
@@ -54,7 +62,7 @@ def compare_round(orc, sess, draft, lens, st: ParityStats, check_logits=True, sa
         assert lg.shape == ro.logits.shape
         err = float(np.abs(lg - ro.logits).max())
         st.max_logit_err = max(st.max_logit_err, err)
-        assert err <= logit_tol(dims), f"logits differ by {err}"
+        assert err <= logit_tol(dims, scale), f"logits differ by {err}"
     st.rounds += 1
     r0 = 0
     for j, b in enumerate(idx):
@@ -72,7 +80,7 @@ def compare_round(orc, sess, draft, lens, st: ParityStats, check_logits=True, sa
             row = min(n_o, n_g)
             choice = int(draft[b, row]) if n_g > row else int(rg.bonus[b])
             gap = float(lo[row, go[row]] - lo[row, choice])
-            assert gap < TIE_GAP, (f"utt {b}: accepted {n_g} vs {n_o}, bonus {rg.bonus[b]} vs {ro.bonus[j]}, "
+            assert gap < TIE_GAP * scale, (f"utt {b}: accepted {n_g} vs {n_o}, bonus {rg.bonus[b]} vs {ro.bonus[j]}, "
                                    f"oracle margin {gap} at row {row}")
             st.near_ties += 1
             orc.kv_len[j] = rg.kv_len[b]
@@ -95,7 +103,7 @@ def compare_round(orc, sess, draft, lens, st: ParityStats, check_logits=True, sa
 
 
 def run_decode(dims, blob, enc, enc_lens, prompt, total, k, corr, sess_factory, max_rounds=None,
-               check_logits=True, k_schedule=None):
+               check_logits=True, k_schedule=None, scale=1.0):
     """Full teacher-forced decode; returns stats.  Drafts come from the oracle's
     own greedy transcript through the workload corruption stream."""
     orc = Oracle(dims, blob)
@@ -114,7 +122,7 @@ def run_decode(dims, blob, enc, enc_lens, prompt, total, k, corr, sess_factory, 
         draft, lens = W.make_drafts(truth, total, orc.kv_len, kk, corr)
         if np.all(lens < 0):
             break
-        compare_round(orc, sess, draft, lens, st, check_logits=check_logits)
+        compare_round(orc, sess, draft, lens, st, check_logits=check_logits, scale=scale)
     assert sess.status() == 0
     sess.close()
     return st, truth

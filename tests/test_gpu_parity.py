@@ -10,7 +10,7 @@ import numpy as np
 import pytest
 
 import workload as W
-from tests.parity import ParityStats, compare_round, run_decode
+from tests.parity import ParityStats, compare_round, run_decode, scale_for
 
 pytestmark = pytest.mark.gpu
 
@@ -60,7 +60,7 @@ def test_small_bf16_ragged_batch(built_lib, cuda, std):
     enc = W.make_encoder_states(dims, enc_lens, 1500)
     prompt = W.make_prompt(dims, 5)
     st, _ = run_decode(dims, blob, enc, enc_lens, prompt, total, 8, W.make_corruption(wl),
-                       _session(dims, blob, 5, 8))
+                       _session(dims, blob, 5, 8), scale=scale_for(dims, std))
     _report(f"small std={std}", st)
     assert st.rows > 50
 
@@ -79,7 +79,7 @@ def test_edge_cases_bf16(built_lib, cuda):
     corr = W.make_corruption(wl)
     sched = lambda r: [16, 0, 3, 16, 1][r % 5]
     st, _ = run_decode(dims, blob, enc, enc_lens, prompt, total, 16, corr, _session(dims, blob, 3, 16),
-                       k_schedule=sched)
+                       k_schedule=sched, scale=scale_for(dims, 0.1))
     _report("edges", st)
 
 
