@@ -814,6 +814,32 @@ int asr_spec_test_gemm(int32_t impl, const void* A, const void* B, float* C, int
   e.ld = N;
   if (impl == 1) {
     launch_gemm_simt(A, 1, B, 1, M, N, K, EPI_F32_MN, e, st);
+  } else if (impl == 3) {
+    // fused argmax over m for every n: C[n] = index of the largest C[.][n]
+    TcGemm g{};
+    g.bn = tc_pick_bn(N);
+    if (!make_tmap_bf16(&g.mapA, A, M, K, 128) || !make_tmap_bf16(&g.mapB, B, N, K, g.bn)) return ASR_E_INVAL;
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    g.splits = 1;
+    unsigned long long* keys = nullptr;
+    int* status = nullptr;
+    CK(cudaMalloc(&keys, (size_t)N * 8));
+    CK(cudaMalloc(&status, 4));
+    CK(cudaMemsetAsync(keys, 0, (size_t)N * 8, st));
+    CK(cudaMemsetAsync(status, 0, 4, st));
+    e.row_key = keys;
+    launch_gemm_tc(g, EPI_ARGMAX, e, status, st);
+    CK(cudaGetLastError());
+    std::vector<unsigned long long> hk(N);
+    std::vector<float> idx(N);
+    CK(cudaMemcpyAsync(hk.data(), keys, (size_t)N * 8, cudaMemcpyDeviceToHost, st));
+    CK(cudaStreamSynchronize(st));
+    for (int n = 0; n < N; ++n) idx[n] = (float)(0xFFFFFFFFu - (uint32_t)(hk[n] & 0xFFFFFFFFull));
+    CK(cudaMemcpy(C, idx.data(), (size_t)N * 4, cudaMemcpyHostToDevice));
+    cudaFree(keys);
+    cudaFree(status);
   } else {
     TcGemm g{};
     g.bn = tc_pick_bn(N);

@@ -137,11 +137,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     }
     if constexpr (MODE == EPI_ARGMAX) {
       __syncthreads();
-      if (threadIdx.x < BN) {
-        const int n = n0 + threadIdx.x;
-        unsigned long long k = red[0][threadIdx.x];
+      for (int c = threadIdx.x; c < BN; c += blockDim.x) {
+        const int n = n0 + c;
+        unsigned long long k = red[0][c];
 #pragma unroll
-        for (int w = 1; w < 4; ++w) k = red[w][threadIdx.x] > k ? red[w][threadIdx.x] : k;
+        for (int w = 1; w < 4; ++w) k = red[w][c] > k ? red[w][c] : k;
         if (n < n_valid) atomicMax(epi.row_key + n, k);
       }
     }
