@@ -30,9 +30,14 @@ def _ready(s):
 
 
 def test_call_order_and_arguments(sess):
+    import torch
     from paper_2608_12703_gb300 import asrspec as A
+    d = torch.zeros((1, 1), dtype=torch.int32, device="cuda")
+    o = torch.zeros((5, 1), dtype=torch.int32, device="cuda")
     with pytest.raises(A.AsrSpecError, match="ASR_E_STATE"):
-        sess.verify(np.zeros((1, 1)), np.zeros(1))
+        A.asr_spec_verify(sess.h, d, o[4], 1, o[0], o[1], o[2], o[3])
+    with pytest.raises(A.AsrSpecError, match="ASR_E_STATE"):
+        A.asr_spec_prefill(sess.h, d, 1)
     _ready(sess)
     with pytest.raises(A.AsrSpecError, match="ASR_E_INVAL"):
         sess.verify(np.zeros((3, 5)), np.zeros(3))         # k > max_draft
