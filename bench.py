@@ -136,8 +136,13 @@ class GpuRun:
             self.prompt_d = torch.from_numpy(self.prompt).cuda()
         self.sess.stream.synchronize()
         self.total = np.array(wl.total_lens, dtype=np.int64)
-        self.truth = self._greedy_transcript()
         self.corr = W.make_corruption(wl)
+        # The reference transcript that drives the drafts: the target's greedy
+        # output under this workload's batching.  One-token rounds give a first
+        # transcript; one speculative decode driven by it gives the transcript
+        # of the speculative batching itself (a fixed point: its own greedy path).
+        truth0 = self._greedy_transcript()
+        self.truth, self.changed_tokens = self._speculative_transcript(DeviceDrafts, truth0)
         self.drafts = DeviceDrafts(self.sess, self.truth, self.total, self.corr, wl.k)
         self.tokens_per_decode = int(sum(wl.n_out))
         self.rounds = self._count_rounds()
@@ -167,12 +172,35 @@ class GpuRun:
         assert self.sess.status() == 0
         return truth
 
+    def _speculative_transcript(self, DeviceDrafts, truth0):
+        B, k = self.wl.batch, self.wl.k
+        drafts = DeviceDrafts(self.sess, truth0, self.total, self.corr, k)
+        self._begin()
+        seq = [list(self.prompt[b]) for b in range(B)]
+        while True:
+            d, l = drafts.next()
+            lh = self.sess.host(l)
+            if (lh < 0).all():
+                break
+            dh = self.sess.host(d)
+            o = self.sess.host(self.sess.verify_device(d, l, k))
+            for b in np.nonzero(lh >= 0)[0]:
+                seq[b] += [int(t) for t in dh[b, :o[0][b]]] + [int(o[1][b])]
+        truth = np.zeros_like(truth0)
+        changed = 0
+        for b in range(B):
+            assert len(seq[b]) == self.total[b], (b, len(seq[b]), self.total[b])
+            truth[b, :len(seq[b])] = seq[b]
+            changed += int((truth[b, :len(seq[b])] != truth0[b, :len(seq[b])]).sum())
+        assert self.sess.status() == 0
+        return truth, changed
+
     def _count_rounds(self):
         self._begin()
         n = 0
         while True:
             d, l = self.drafts.next()
-            if bool((l < 0).all()):
+            if (self.sess.host(l) < 0).all():
                 break
             self.sess.verify_device(d, l, self.wl.k)
             n += 1
@@ -474,6 +502,7 @@ def main():
         "value": value, "ms_per_step": ms / args.steps,
         "verify_us": res["verify_us"],
         "verify_rounds_per_step": run.rounds,
+        "transcript_tokens_changed_by_batching": run.changed_tokens,
         "verify_hbm": {"bytes_per_call": bytes_per_call,
                        "frac": bytes_per_call / (res["verify_us"]["median"] * 1e-6) / (pk["hbm"] * 1e9),
                        "frac_nominal_8tbs": bytes_per_call / (res["verify_us"]["median"] * 1e-6) / 8e12},

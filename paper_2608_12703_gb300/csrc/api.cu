@@ -58,6 +58,8 @@ struct asr_spec {
   size_t ws_floats = 0;
   int* tickets = nullptr;
   int n_tickets = 0;
+  int* attn_tickets = nullptr;                       // [B_max * H], tensor-core attention merge
+  CUtensorMap m_kself[2], m_vself[2], m_xkv[2];      // boxes of 128 and 256 rows
   std::map<std::pair<int, int>, CUtensorMap> bmaps;  // (buffer id, BN) -> map
 
   // profiling: CUDA events around each kernel class (direct launches only)
@@ -190,7 +192,10 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   }
   TcGemm g{};
   g.mapA = *mW;
-  g.bn = tc_pick_bn(N);
+  // Few rows (batch 1): one narrow N tile, split K across CTAs so that every SM
+  // streams weights.  Many rows: 64-wide N tiles, split K only while the grid
+  // is short of one wave.
+  g.bn = N <= 64 ? tc_pick_bn(N) : 64;
   const CUtensorMap* mb = bmap(h, x_id, X, h->R_pad, K, g.bn);
   if (!mb) return fail(h, ASR_E_CUDA, "tensor map encode failed");
   g.mapB = *mb;
@@ -198,7 +203,9 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   g.N = N;
   g.K = K;
   const int tiles = ((M + 127) / 128) * ((N + g.bn - 1) / g.bn);
-  g.splits = mode == EPI_ARGMAX || mode == EPI_F32 ? 1 : pick_splits(tiles, K / 64);
+  if (mode == EPI_ARGMAX || mode == EPI_F32) g.splits = 1;
+  else if (N <= 64) g.splits = pick_splits(tiles, K / 64);
+  else g.splits = tiles >= NUM_SMS_TARGET ? 1 : std::min((NUM_SMS_TARGET + tiles - 1) / tiles, std::max(1, K / 256));
   while (g.splits > 1 && (size_t)g.splits * tiles * 128 * g.bn > h->ws_floats) --g.splits;
   if (tiles > h->n_tickets && g.splits > 1) g.splits = 1;
   g.ws = h->ws;
@@ -210,7 +217,34 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
 enum BufId { BUF_XN = 1, BUF_ATT = 2, BUF_H = 3, BUF_XF = 4 };
 
 // The decoder layers over the rows laid out by the last plan kernel.
+// Keys per attention CTA: small grids (few utterances) split keys finer.
+int attn_chunk_for(asr_spec* h, int t_alloc) {
+  if (!h->bf16) return attn_chunk_len(0);
+  const int ctas256 = h->B * h->H * ((t_alloc + 255) / 256);
+  return ctas256 >= 2 * NUM_SMS_TARGET ? 256 : 128;
+}
+
+void attention(asr_spec* h, AttnArgs& a, bool self_attn, int layer) {
+  if (!h->bf16) {
+    launch_attention(a, h->st);
+    return;
+  }
+  const int ci = a.chunk == 256 ? 1 : 0;
+  if (self_attn) {
+    a.kmap = &h->m_kself[ci];
+    a.vmap = &h->m_vself[ci];
+    a.k_row0 = a.v_row0 = (long long)layer * h->Bmax * h->H * h->maxpos;
+  } else {
+    a.kmap = a.vmap = &h->m_xkv[ci];
+    a.k_row0 = (long long)layer * 2 * h->Bmax * h->H * h->Tmax;
+    a.v_row0 = a.k_row0 + (long long)h->Bmax * h->H * h->Tmax;
+  }
+  a.tickets = h->attn_tickets;
+  launch_attention_tc(a, h->status, h->st);
+}
+
 int run_layers(asr_spec* h, int N) {
+  const int rows_max = N / std::max(h->B, 1);
   const int d = h->d;
   Epi base{};
   base.n_valid = h->plan.n_rows;
@@ -258,15 +292,16 @@ int run_layers(asr_spec* h, int N) {
     a.H = h->H;
     a.d = d;
     a.k1 = h->kmax + 1;
-    a.chunk = attn_chunk_len(h->bf16);
+    a.chunk = attn_chunk_for(h, h->maxpos);
     a.n_chunks = (h->maxpos + a.chunk - 1) / a.chunk;
     a.part = h->part;
     a.out = h->att;
     a.out_bf16 = h->bf16;
     a.ml_out = nullptr;
+    a.rows_max = rows_max;
     {
-      Prof p(h, ASR_PROF_SELF, 2);
-      launch_attention(a, h->st);
+      Prof p(h, ASR_PROF_SELF, h->bf16 ? 1 : 2);
+      attention(h, a, true, l);
     }
     e = base;
     e.bias = w.bo;
@@ -287,11 +322,12 @@ int run_layers(asr_spec* h, int N) {
     a.vc = vx;
     a.t_alloc = h->Tmax;
     a.causal = 0;
+    a.chunk = attn_chunk_for(h, h->Tmax);
     a.n_chunks = (h->Tmax + a.chunk - 1) / a.chunk;
     a.ml_out = (l == h->anchor) ? h->ml : nullptr;
     {
-      Prof p(h, ASR_PROF_CROSS, 2);
-      launch_attention(a, h->st);
+      Prof p(h, ASR_PROF_CROSS, h->bf16 ? 1 : 2);
+      attention(h, a, false, l);
     }
     e = base;
     e.bias = w.bco;
@@ -530,7 +566,7 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   CK(cudaMemset(h->att, 0, R * d * es));
   CK(cudaMemset(h->hbuf, 0, R * F * es));
   CK(cudaMemset(h->xf, 0, R * d * es));
-  const int chunk = attn_chunk_len(h->bf16);
+  const int chunk = h->bf16 ? 128 : attn_chunk_len(0);   // the finest split either path uses
   const int n_chunks = (std::max(h->maxpos, h->Tmax) + chunk - 1) / chunk;
   if ((rc = dalloc(h, &h->part, (size_t)h->Bmax * h->H * n_chunks * (h->kmax + 1) * 66 * 4))) return finish(rc);
   if ((rc = dalloc(h, &h->plan.row_b, R * 4)) || (rc = dalloc(h, &h->plan.row_i, R * 4)) ||
@@ -553,6 +589,19 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   h->n_tickets = 8192;
   if ((rc = dalloc(h, &h->ws, h->ws_floats * 4)) || (rc = dalloc(h, &h->tickets, h->n_tickets * 4))) return finish(rc);
   CK(cudaMemset(h->tickets, 0, h->n_tickets * 4));
+  if ((rc = dalloc(h, &h->attn_tickets, (size_t)h->Bmax * h->H * 4))) return finish(rc);
+  CK(cudaMemset(h->attn_tickets, 0, (size_t)h->Bmax * h->H * 4));
+  if (h->bf16) {
+    const uint64_t self_rows = (uint64_t)L * h->Bmax * h->H * h->maxpos;
+    const uint64_t cross_rows = (uint64_t)L * 2 * h->Bmax * h->H * h->Tmax;
+    for (int i = 0; i < 2; ++i) {
+      const uint32_t box = i ? 256 : 128;
+      if (!make_tmap_cache(&h->m_kself[i], h->kself, self_rows, box) ||
+          !make_tmap_cache(&h->m_vself[i], h->vself, self_rows, box) ||
+          !make_tmap_cache(&h->m_xkv[i], h->xkv, cross_rows, box))
+        return finish(fail(h, ASR_E_CUDA, "tensor map encode failed"));
+    }
+  }
   if ((rc = dalloc(h, &h->counters, 8 * sizeof(unsigned long long)))) return finish(rc);
   CK(cudaMemset(h->counters, 0, 8 * sizeof(unsigned long long)));
   configure_gemm_tc();

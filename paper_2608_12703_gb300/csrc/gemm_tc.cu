@@ -163,18 +163,31 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     if (s_last) {
       __threadfence();
       const float* base = ws + ((size_t)tile * splits * TC_BM + warp * 32 + lane) * BN;
+      const int c_end = min(BN, ((n_valid - n0) + 3) & ~3);   // columns past the valid rows are not read
 #pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 4) {
-        float4 acc = __ldcg(reinterpret_cast<const float4*>(base + c0));
-        for (int s = 1; s < splits; ++s) {
-          float4 p = __ldcg(reinterpret_cast<const float4*>(base + (size_t)s * TC_BM * BN + c0));
-          acc.x += p.x; acc.y += p.y; acc.z += p.z; acc.w += p.w;
-        }
-        const float a4[4] = {acc.x, acc.y, acc.z, acc.w};
+      for (int c0 = 0; c0 < c_end; c0 += 16) {
+        // 16 columns x all splits in flight before the (split-ordered) sums
+        float4 acc[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int n = n0 + c0 + i;
-          if (m < epi.M && n < n_valid) epi_apply<MODE == EPI_ARGMAX ? EPI_F32 : MODE>(epi, m, n, a4[i]);
+        for (int q = 0; q < 4; ++q) acc[q] = __ldcg(reinterpret_cast<const float4*>(base + c0 + 4 * q));
+        for (int s = 1; s < splits; ++s) {
+          float4 p[4];
+          const float* ps = base + (size_t)s * TC_BM * BN + c0;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) p[q] = __ldcg(reinterpret_cast<const float4*>(ps + 4 * q));
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            acc[q].x += p[q].x; acc[q].y += p[q].y; acc[q].z += p[q].z; acc[q].w += p[q].w;
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float a4[4] = {acc[q].x, acc[q].y, acc[q].z, acc[q].w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int n = n0 + c0 + 4 * q + i;
+            if (m < epi.M && n < n_valid) epi_apply<MODE == EPI_ARGMAX ? EPI_F32 : MODE>(epi, m, n, a4[i]);
+          }
         }
       }
       if (threadIdx.x == 0) tickets[tile] = 0;

@@ -84,8 +84,19 @@ struct AttnArgs {
   void* out;               // [R][d] attention output (bf16 or fp32)
   int out_bf16;
   float* ml_out;           // optional [R][H][2] (max, sum) of the full softmax
+  // tensor-core path (bf16 caches): 2-D tensor maps over the whole K and V
+  // caches ([rows][64], 128-byte swizzle) and the row of (b = 0, h = 0, t = 0)
+  // of this layer in each; per-(b, h) tickets for the in-kernel chunk merge
+  const CUtensorMap* kmap = nullptr;
+  const CUtensorMap* vmap = nullptr;
+  long long k_row0 = 0, v_row0 = 0;
+  int* tickets = nullptr;
+  int rows_max = 0;        // most rows of one utterance in this call
 };
 void launch_attention(const AttnArgs& a, cudaStream_t st);
+void launch_attention_tc(const AttnArgs& a, int* status, cudaStream_t st);
+// Tensor map over a [rows][64] bf16 cache with `box_rows`-row boxes.
+bool make_tmap_cache(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows);
 
 // Anchor readout: head-mean softmax of row anchor_row[b] at the anchor layer.
 void launch_anchor(const float* q_anchor, const float* ml, const void* kc, int kv_bf16, int t_alloc,

@@ -106,6 +106,11 @@ class Session:
             oh = o.cpu().numpy()
         return StepOut(oh[0].copy(), oh[1].copy(), oh[2].copy(), oh[3].copy())
 
+    def host(self, t) -> np.ndarray:
+        """Copy a device tensor written on this session's stream to the host."""
+        self.stream.synchronize()
+        return t.cpu().numpy()
+
     def verify_device(self, draft_d, lens_d, k: int):
         """Device-resident verify: inputs and outputs stay on the GPU (no sync)."""
         o = self.out[:, :self.B]
