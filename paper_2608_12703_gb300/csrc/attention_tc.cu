@@ -254,25 +254,51 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
   __syncthreads();
   if (!s_last) return;
   __threadfence();
+  // chunk weights first (one thread per (row, chunk), all loads in flight at
+  // once), then every output element as one pass over the chunks
   const float* pb = a.part + ((size_t)b * a.H + h) * a.n_chunks * a.k1 * 66;
   const size_t cstride = (size_t)a.k1 * 66;
+  float* wgt = Ow;                               // [nr][nc] chunk weights, then [nr] sums
+  float* Lsum = Ow + MT * 16 * 32;
+  for (int e = tid; e < nr * nc; e += TCA_THREADS) {
+    const int r = e / nc, ci = e - r * nc;
+    wgt[r * 32 + ci] = __ldcg(pb + ci * cstride + r * 66 + 64);
+    Lsum[r * 32 + ci] = __ldcg(pb + ci * cstride + r * 66 + 65);
+  }
+  __syncthreads();
+  if (tid < nr) {
+    float M = -INFINITY;
+    for (int ci = 0; ci < nc; ++ci) M = fmaxf(M, wgt[tid * 32 + ci]);
+    float L = 0.f;
+    for (int ci = 0; ci < nc; ++ci) {
+      const float mc = wgt[tid * 32 + ci];
+      const float f = (mc == -INFINITY) ? 0.f : __expf(mc - M);
+      L += Lsum[tid * 32 + ci] * f;
+      wgt[tid * 32 + ci] = f;
+    }
+    for (int ci = 0; ci < nc; ++ci) wgt[tid * 32 + ci] /= L;
+    if (a.ml_out) {
+      a.ml_out[((size_t)(row0 + tid) * a.H + h) * 2 + 0] = M;
+      a.ml_out[((size_t)(row0 + tid) * a.H + h) * 2 + 1] = L;
+    }
+  }
+  __syncthreads();
   for (int e = tid; e < nr * 64; e += TCA_THREADS) {
     const int r = e >> 6, c = e & 63;
-    float M = -INFINITY;
-    for (int ci = 0; ci < nc; ++ci) M = fmaxf(M, __ldcg(pb + ci * cstride + r * 66 + 64));
-    float L = 0.f, o = 0.f;
-    for (int ci = 0; ci < nc; ++ci) {
-      const float mc = __ldcg(pb + ci * cstride + r * 66 + 64);
-      const float f = (mc == -INFINITY) ? 0.f : __expf(mc - M);
-      L += __ldcg(pb + ci * cstride + r * 66 + 65) * f;
-      o += __ldcg(pb + ci * cstride + r * 66 + c) * f;
+    float o = 0.f;
+    int ci = 0;
+    for (; ci + 4 <= nc; ci += 4) {
+      const float p0 = __ldcg(pb + (ci + 0) * cstride + r * 66 + c);
+      const float p1 = __ldcg(pb + (ci + 1) * cstride + r * 66 + c);
+      const float p2 = __ldcg(pb + (ci + 2) * cstride + r * 66 + c);
+      const float p3 = __ldcg(pb + (ci + 3) * cstride + r * 66 + c);
+      o += p0 * wgt[r * 32 + ci];
+      o += p1 * wgt[r * 32 + ci + 1];
+      o += p2 * wgt[r * 32 + ci + 2];
+      o += p3 * wgt[r * 32 + ci + 3];
     }
-    const size_t oi = (size_t)(row0 + r) * a.d + h * 64 + c;
-    reinterpret_cast<__nv_bfloat16*>(a.out)[oi] = f2bf(o / L);
-    if (a.ml_out && c == 0) {
-      a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 0] = M;
-      a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 1] = L;
-    }
+    for (; ci < nc; ++ci) o += __ldcg(pb + ci * cstride + r * 66 + c) * wgt[r * 32 + ci];
+    reinterpret_cast<__nv_bfloat16*>(a.out)[(size_t)(row0 + r) * a.d + h * 64 + c] = f2bf(o);
   }
   if (tid == 0) a.tickets[b * a.H + h] = 0;
 }

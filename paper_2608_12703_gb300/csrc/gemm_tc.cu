@@ -170,7 +170,23 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
         float4 acc[4];
 #pragma unroll
         for (int q = 0; q < 4; ++q) acc[q] = __ldcg(reinterpret_cast<const float4*>(base + c0 + 4 * q));
-        for (int s = 1; s < splits; ++s) {
+        int s = 1;
+        for (; s + 2 <= splits; s += 2) {   // two splits' loads in flight, summed in split order
+          float4 p[2][4];
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const float* ps = base + (size_t)(s + u) * TC_BM * BN + c0;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) p[u][q] = __ldcg(reinterpret_cast<const float4*>(ps + 4 * q));
+          }
+#pragma unroll
+          for (int u = 0; u < 2; ++u)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              acc[q].x += p[u][q].x; acc[q].y += p[u][q].y; acc[q].z += p[u][q].z; acc[q].w += p[u][q].w;
+            }
+        }
+        for (; s < splits; ++s) {
           float4 p[4];
           const float* ps = base + (size_t)s * TC_BM * BN + c0;
 #pragma unroll
