@@ -175,8 +175,8 @@ void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan 
                                                static_cast<const float*>(pos_emb), plan, d, x);
 }
 
-// LayerNorm, one warp per row, statistics in fp32 (two passes over registers).
-constexpr int LN_MAX_PER_LANE = 64;   // d <= 2048
+// LayerNorm, one warp per row, statistics in fp32: a sum pass and a centred
+// sum-of-squares pass over the row (L2-resident), then the affine write.
 template <typename TO>
 __global__ void __launch_bounds__(256)
 layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const float* __restrict__ bta,
@@ -184,28 +184,30 @@ layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = blockIdx.x * 8 + warp;
   if (r >= *n_rows) return;
-  const float* xr = x + (size_t)r * d;
-  float v[LN_MAX_PER_LANE];
-  const int per = d / 32;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)r * d);
+  const int n4 = d >> 2;
   float s = 0.f;
-#pragma unroll 4
-  for (int i = 0; i < per; ++i) {
-    v[i] = xr[lane + 32 * i];
-    s += v[i];
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = xr[i];
+    s += (v.x + v.y) + (v.z + v.w);
   }
   const float mean = warp_sum(s) / (float)d;
   float q = 0.f;
-#pragma unroll 4
-  for (int i = 0; i < per; ++i) {
-    const float t = v[i] - mean;
-    q += t * t;
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = xr[i];
+    const float a = v.x - mean, b = v.y - mean, c = v.z - mean, e = v.w - mean;
+    q += (a * a + b * b) + (c * c + e * e);
   }
-  const float var = warp_sum(q) / (float)d;
-  const float rstd = rsqrtf(var + 1e-5f);
-#pragma unroll 4
-  for (int i = 0; i < per; ++i) {
-    const int c = lane + 32 * i;
-    y[(size_t)r * d + c] = from_f<TO>((v[i] - mean) * rstd * g[c] + bta[c]);
+  const float rstd = rsqrtf(warp_sum(q) / (float)d + 1e-5f);
+  TO* yr = y + (size_t)r * d;
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = xr[i];
+    const float4 gg = reinterpret_cast<const float4*>(g)[i];
+    const float4 bb = reinterpret_cast<const float4*>(bta)[i];
+    yr[4 * i + 0] = from_f<TO>((v.x - mean) * rstd * gg.x + bb.x);
+    yr[4 * i + 1] = from_f<TO>((v.y - mean) * rstd * gg.y + bb.y);
+    yr[4 * i + 2] = from_f<TO>((v.z - mean) * rstd * gg.z + bb.z);
+    yr[4 * i + 3] = from_f<TO>((v.w - mean) * rstd * gg.w + bb.w);
   }
 }
 
