@@ -207,6 +207,29 @@ int asr_spec_synth_drafts(asr_spec_handle h, const int32_t* truth, const int32_t
 int asr_spec_test_gemm(int32_t impl, const void* A, const void* B, float* C, int32_t M, int32_t N,
                        int32_t K, void* stream);
 
+/* ---- Split-K GEMM without device allocation ------------------------------
+ * The paper has no counterpart to this entry: it serves callers that may not
+ * allocate device memory at all, such as a host framework that owns every
+ * device byte through its own pool, a serving loop that forbids allocation
+ * after start-up because cudaMalloc/cudaFree can synchronise the whole device,
+ * or code running while another thread captures a CUDA graph in a mode that
+ * rejects such calls.
+ * Computes C[m][n] = sum_k A[m][k] * B[n][k] with the tcgen05 GEMM, K split
+ * into `splits` ranges (1 <= splits <= K / 64) whose partial sums are added in
+ * split order; A [M][K], B [N][K] bf16 row-major, C [M][N] fp32, all device
+ * pointers owned by the caller; K % 64 == 0.  It calls no cudaMalloc, cudaFree
+ * or allocating library routine: the split-K partial sums, tile tickets and
+ * status word live in one fixed device array of about 8 MiB (2^21 partial
+ * floats, 4096 output tiles) that every GPU loading the library keeps until
+ * the process exits.  Calls needing more return ASR_E_CAPACITY.  The first
+ * call on a device looks the array's address up (make it before any stream
+ * capture on that device).  All calls share the array: each one clears the
+ * tickets and status before its kernel, and calls that overlap on the GPU
+ * race.  Synchronises `stream` before returning; ASR_E_DEVICE if a bounded
+ * pipeline wait gave up, ASR_E_INVAL for bad arguments. */
+int asr_spec_gemm_noalloc(const void* A, const void* B, float* C, int32_t M, int32_t N, int32_t K,
+                          int32_t splits, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -27,6 +27,7 @@ EXPORTED = [
     "asr_spec_verify", "asr_spec_rollback", "asr_spec_state", "asr_spec_debug_logits",
     "asr_spec_status", "asr_spec_last_error", "asr_spec_destroy", "asr_spec_synth_drafts",
     "asr_spec_test_gemm", "asr_spec_set_graphs", "asr_spec_profile", "asr_spec_profile_read",
+    "asr_spec_gemm_noalloc",
 ]
 PROF_CLASSES = ["proj_gemm", "self_attn", "cross_attn", "lm_head", "other"]
 
@@ -76,6 +77,7 @@ def lib():
     L.asr_spec_set_graphs.argtypes = [vp, ctypes.c_int]
     L.asr_spec_profile.argtypes = [vp, ctypes.c_int]
     L.asr_spec_profile_read.argtypes = [vp, vp, vp, vp]
+    L.asr_spec_gemm_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
     for name in EXPORTED:
         if name not in ("asr_spec_last_error", "asr_spec_destroy"):
             getattr(L, name).restype = ctypes.c_int
@@ -182,3 +184,10 @@ def asr_spec_profile_read(h):
     _check(h, lib().asr_spec_profile_read(h, ms.ctypes.data, launches.ctypes.data, traffic.ctypes.data),
            "asr_spec_profile_read")
     return ms, launches, traffic
+
+
+def asr_spec_gemm_noalloc(A, B, C, M, N, K, splits, stream=None):
+    """Split-K GEMM whose scratch is a fixed device array (no allocation)."""
+    return _check(None, lib().asr_spec_gemm_noalloc(ptr(A), ptr(B), ptr(C), M, N, K, splits,
+                                                    None if stream is None else ctypes.c_void_p(stream)),
+                  "asr_spec_gemm_noalloc")
