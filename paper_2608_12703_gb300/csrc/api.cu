@@ -2,6 +2,7 @@
 // encoder cache, prefill, verify, rollback.  See include/asrspec.h.
 #include <algorithm>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <string>
@@ -73,6 +74,7 @@ struct asr_spec {
   unsigned long long* counters = nullptr;         // device traffic counters [8]
   // CUDA graphs of the verify body, keyed by (B, k)
   bool use_graphs = true;
+  bool use_pdl = true;   // programmatic dependent launch between verify kernels
   struct Graph {
     cudaGraphExec_t exec;
     long long launches[ASR_PROF_N];
@@ -173,12 +175,6 @@ const CUtensorMap* bmap(asr_spec* h, int id, const void* buf, int rows, int cols
   return &(h->bmaps[key] = m);
 }
 
-int pick_splits(int tiles, int nkb) {
-  int s = (2 * NUM_SMS_TARGET + tiles / 2) / std::max(tiles, 1);
-  s = std::max(1, std::min(s, nkb / 2));
-  return s;
-}
-
 // One projection over the verify rows: out-features m (weights = A), rows n (activations = B).
 int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, const void* X, int x_id, int N,
               int mode, const Epi& epi_in) {
@@ -192,10 +188,12 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   }
   TcGemm g{};
   g.mapA = *mW;
-  // Few rows (batch 1): one narrow N tile, split K across CTAs so that every SM
-  // streams weights.  Many rows: 64-wide N tiles, split K only while the grid
-  // is short of one wave.
-  g.bn = N <= 64 ? tc_pick_bn(N) : 64;
+  // Few rows (batch 1): one narrow N tile and K split across the CTAs of a
+  // cluster so that every SM streams weights.  Many rows: 128-wide N tiles
+  // (two CTAs per SM), K split in a cluster while the grid stays within one
+  // wave and every split keeps at least four k-blocks.  Split factors are
+  // powers of two up to 16.
+  g.bn = N <= 64 ? tc_pick_bn(N) : 128;
   const CUtensorMap* mb = bmap(h, x_id, X, h->R_pad, K, g.bn);
   if (!mb) return fail(h, ASR_E_CUDA, "tensor map encode failed");
   g.mapB = *mb;
@@ -203,11 +201,14 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   g.N = N;
   g.K = K;
   const int tiles = ((M + 127) / 128) * ((N + g.bn - 1) / g.bn);
-  if (mode == EPI_ARGMAX || mode == EPI_F32) g.splits = 1;
-  else if (N <= 64) g.splits = pick_splits(tiles, K / 64);
-  else g.splits = tiles >= NUM_SMS_TARGET ? 1 : std::min((NUM_SMS_TARGET + tiles - 1) / tiles, std::max(1, K / 256));
-  while (g.splits > 1 && (size_t)g.splits * tiles * 128 * g.bn > h->ws_floats) --g.splits;
-  if (tiles > h->n_tickets && g.splits > 1) g.splits = 1;
+  const int nkb = K / 64;
+  const int target = 2 * NUM_SMS_TARGET;
+  g.splits = 1;
+  if (mode != EPI_ARGMAX && mode != EPI_F32)
+    while (g.splits < 16 && tiles * g.splits * 2 <= target && g.splits * 2 <= (N <= 64 ? nkb : nkb / 4))
+      g.splits *= 2;
+  g.cluster = g.splits > 1;
+  g.pdl = h->use_pdl;
   g.ws = h->ws;
   g.tickets = h->tickets;
   launch_gemm_tc(g, mode, epi, h->status, h->st);
@@ -217,11 +218,13 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
 enum BufId { BUF_XN = 1, BUF_ATT = 2, BUF_H = 3, BUF_XF = 4 };
 
 // The decoder layers over the rows laid out by the last plan kernel.
-// Keys per attention CTA: small grids (few utterances) split keys finer.
-int attn_chunk_for(asr_spec* h, int t_alloc) {
-  if (!h->bf16) return attn_chunk_len(0);
-  const int ctas256 = h->B * h->H * ((t_alloc + 255) / 256);
-  return ctas256 >= 2 * NUM_SMS_TARGET ? 256 : 128;
+// CTAs per (utterance, head) for the tensor-core attention: few utterances
+// (batch 1) split the keys over a cluster of up to 8 CTAs.
+int attn_splits_for(asr_spec* h, int t_alloc) {
+  const int nc_max = (t_alloc + 127) / 128;
+  int S = 1;
+  while (S < 8 && S * 2 <= nc_max && h->B * h->H * S * 2 <= 2 * NUM_SMS_TARGET) S *= 2;
+  return S;
 }
 
 void attention(asr_spec* h, AttnArgs& a, bool self_attn, int layer) {
@@ -229,7 +232,8 @@ void attention(asr_spec* h, AttnArgs& a, bool self_attn, int layer) {
     launch_attention(a, h->st);
     return;
   }
-  const int ci = a.chunk == 256 ? 1 : 0;
+  a.splits = attn_splits_for(h, a.t_alloc);
+  const int ci = 0;   // 128-row boxes
   if (self_attn) {
     a.kmap = &h->m_kself[ci];
     a.vmap = &h->m_vself[ci];
@@ -240,6 +244,7 @@ void attention(asr_spec* h, AttnArgs& a, bool self_attn, int layer) {
     a.v_row0 = a.k_row0 + (long long)h->Bmax * h->H * h->Tmax;
   }
   a.tickets = h->attn_tickets;
+  a.pdl = h->use_pdl;
   launch_attention_tc(a, h->status, h->st);
 }
 
@@ -259,7 +264,7 @@ int run_layers(asr_spec* h, int N) {
   const size_t cross_half = (size_t)h->Bmax * h->H * h->Tmax * 64 * h->es;
   {
     Prof p(h, ASR_PROF_OTHER, 1);
-    launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st);
+    launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st, h->use_pdl);
   }
   for (int l = 0; l < h->L; ++l) {
     LayerW& w = h->lw[l];
@@ -270,7 +275,7 @@ int run_layers(asr_spec* h, int N) {
     // self-attention block
     {
       Prof p(h, ASR_PROF_OTHER, 1);
-      launch_layernorm(h->x, w.ln1g, w.ln1b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+      launch_layernorm(h->x, w.ln1g, w.ln1b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st, h->use_pdl);
     }
     Epi e = base;
     e.bias = w.bqkv;
@@ -292,7 +297,7 @@ int run_layers(asr_spec* h, int N) {
     a.H = h->H;
     a.d = d;
     a.k1 = h->kmax + 1;
-    a.chunk = attn_chunk_for(h, h->maxpos);
+    a.chunk = attn_chunk_len(h->bf16);
     a.n_chunks = (h->maxpos + a.chunk - 1) / a.chunk;
     a.part = h->part;
     a.out = h->att;
@@ -310,7 +315,7 @@ int run_layers(asr_spec* h, int N) {
     // cross-attention block
     {
       Prof p(h, ASR_PROF_OTHER, 1);
-      launch_layernorm(h->x, w.ln2g, w.ln2b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+      launch_layernorm(h->x, w.ln2g, w.ln2b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st, h->use_pdl);
     }
     float* qc = (l == h->anchor) ? h->q_anchor : h->q;
     e = base;
@@ -322,7 +327,6 @@ int run_layers(asr_spec* h, int N) {
     a.vc = vx;
     a.t_alloc = h->Tmax;
     a.causal = 0;
-    a.chunk = attn_chunk_for(h, h->Tmax);
     a.n_chunks = (h->Tmax + a.chunk - 1) / a.chunk;
     a.ml_out = (l == h->anchor) ? h->ml : nullptr;
     {
@@ -336,7 +340,7 @@ int run_layers(asr_spec* h, int N) {
     // MLP block
     {
       Prof p(h, ASR_PROF_OTHER, 1);
-      launch_layernorm(h->x, w.ln3g, w.ln3b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st);
+      launch_layernorm(h->x, w.ln3g, w.ln3b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st, h->use_pdl);
     }
     e = base;
     e.bias = w.b1;
@@ -381,24 +385,39 @@ int enqueue_verify(asr_spec* h, int k) {
   if (int rc = run_layers(h, N)) return rc;
   {
     Prof p(h, ASR_PROF_OTHER, 1);
-    launch_layernorm(h->x, h->lnf_g, h->lnf_b, h->xf, h->bf16, h->plan.n_rows, N, h->d, h->st);
+    launch_layernorm(h->x, h->lnf_g, h->lnf_b, h->xf, h->bf16, h->plan.n_rows, N, h->d, h->st, h->use_pdl);
   }
   Epi e{};
   e.n_valid = h->plan.n_rows;
   e.row_key = h->row_key;
   e.d = h->d;
   if (int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, N, EPI_ARGMAX, e)) return rc;
-  int* o_acc = h->out4;
-  int* o_bonus = h->out4 + h->Bmax;
-  int* o_len = h->out4 + 2 * h->Bmax;
-  int* o_anchor = h->out4 + 3 * h->Bmax;
-  Prof p(h, ASR_PROF_OTHER, 2);
-  launch_accept(h->draft_buf, h->lens_buf, k, B, h->plan, h->row_key, h->kv_len, h->pending, o_acc, o_bonus, o_len,
-                h->anchor_row, o_anchor, h->st);
+  Prof p(h, ASR_PROF_OTHER, 1);
+  AcceptAnchorArgs A{};
+  A.draft = h->draft_buf;
+  A.k = k;
+  A.B = B;
+  A.H = h->H;
+  A.d = h->d;
+  A.t_alloc = h->Tmax;
+  A.kv_bf16 = h->bf16;
+  A.plan = h->plan;
+  A.row_key = h->row_key;
+  A.kv_len = h->kv_len;
+  A.pending = h->pending;
+  A.accepted = h->out4;
+  A.bonus = h->out4 + h->Bmax;
+  A.kv_len_out = h->out4 + 2 * h->Bmax;
+  A.anchor_out = h->out4 + 3 * h->Bmax;
+  A.q_anchor = h->q_anchor;
+  A.ml = h->ml;
   const size_t cross_half = (size_t)h->Bmax * h->H * h->Tmax * 64 * h->es;
-  const char* kx = static_cast<const char*>(h->xkv) + (size_t)h->anchor * 2 * cross_half;
-  launch_anchor(h->q_anchor, h->ml, kx, h->bf16, h->Tmax, h->enc_len, h->anchor_row, B, h->H, h->d, h->frame_key,
-                reinterpret_cast<int*>(h->frame_key + h->Bmax), o_anchor, h->st);
+  A.kc = static_cast<const char*>(h->xkv) + (size_t)h->anchor * 2 * cross_half;
+  A.enc_len = h->enc_len;
+  A.frame_key = h->frame_key;
+  A.tickets = reinterpret_cast<int*>(h->frame_key + h->Bmax);
+  A.pdl = h->use_pdl;
+  launch_accept_anchor(A, h->st);
   return 0;
 }
 
@@ -423,6 +442,7 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   h->Tmax = dims->max_enc;
   h->anchor = dims->anchor_layer >= 0 ? dims->anchor_layer : (3 * h->L) / 4;
   h->bf16 = dims->dtype == 1;
+  if (const char* e = std::getenv("ASRSPEC_PDL")) h->use_pdl = std::atoi(e) != 0;
   h->es = h->bf16 ? 2 : 4;
   h->st = static_cast<cudaStream_t>(stream);
   if (!h->st) {
@@ -891,17 +911,22 @@ int asr_spec_test_gemm(int32_t impl, const void* A, const void* B, float* C, int
     cudaFree(status);
   } else {
     TcGemm g{};
-    g.bn = tc_pick_bn(N);
+    g.bn = impl == 4 && N > 64 ? tc_pick_bn_wide(N) : tc_pick_bn(N);
     if (!make_tmap_bf16(&g.mapA, A, M, K, 128) || !make_tmap_bf16(&g.mapB, B, N, K, g.bn)) return ASR_E_INVAL;
     g.M = M;
     g.N = N;
     g.K = K;
     const int tiles = ((M + 127) / 128) * ((N + g.bn - 1) / g.bn);
     g.splits = impl == 2 ? std::min(3, K / 64) : 1;
+    if (impl == 4) {   // split K inside a cluster
+      g.splits = 1;
+      while (g.splits < 8 && g.splits * 2 <= K / 64) g.splits *= 2;
+      g.cluster = g.splits > 1;
+    }
     int* status = nullptr;
     CK(cudaMalloc(&status, 4));
     CK(cudaMemset(status, 0, 4));
-    if (g.splits > 1) {
+    if (g.splits > 1 && !g.cluster) {
       CK(cudaMalloc(&g.ws, (size_t)g.splits * tiles * 128 * g.bn * 4));
       CK(cudaMalloc(&g.tickets, (size_t)tiles * 4));
       CK(cudaMemset(g.tickets, 0, (size_t)tiles * 4));

@@ -185,68 +185,122 @@ void launch_attention(const AttnArgs& a, cudaStream_t st) {
 int attn_chunk_len(int kv_bf16) { return kv_bf16 ? 256 : 128; }
 
 // ---------------------------------------------------------------------------
-// Anchor readout
+// Acceptance, commit and anchor readout, fused
 // ---------------------------------------------------------------------------
-constexpr int ANCHOR_FRAMES = 256;
+// One CTA per (32 encoder frames, utterance).  Every CTA of an utterance
+// recomputes the accepted length n from the per-row argmax keys (a few loads);
+// the first one commits: accepted, bonus, kv_len += 1 + n, pending = bonus
+// (Sec. 3 "Speculative Loop"; a round advances 1 + L tokens, App. "Correction
+// and Cost").  Then each CTA evaluates, for its frames, the head mean of the
+// per-head softmax attention of row n at the anchor layer (Sec. 5
+// "Verification-Attention Correction"), with the (max, sum) the attention pass
+// left; a fixed-order head sum per frame, an order-free atomicMax of packed
+// (value, frame) keys, and the last CTA (ticket) writes the peak frame.
+constexpr int ANCHOR_FRAMES = 32;
 
 template <typename T>
-__global__ void __launch_bounds__(ANCHOR_FRAMES)
-anchor_kernel(const float* __restrict__ q_anchor, const float* __restrict__ ml, const T* __restrict__ kc, int t_alloc,
-              const int* __restrict__ enc_len, const int* __restrict__ anchor_row, int H, int d,
-              unsigned long long* frame_key, int* tickets, int* anchor_out) {
-  __shared__ float qs[64];
-  __shared__ unsigned long long red[ANCHOR_FRAMES / 32];
-  __shared__ int s_last;
-  const int b = blockIdx.y;
-  const int r = anchor_row[b];
-  if (r < 0) return;  // uniform: the utterance sat out or the step was refused
-  const int n_frames = enc_len[b];
-  const int j = blockIdx.x * ANCHOR_FRAMES + threadIdx.x;
-  float pbar = 0.f;
-  for (int h = 0; h < H; ++h) {
-    __syncthreads();
-    if (threadIdx.x < 64) qs[threadIdx.x] = q_anchor[(size_t)r * d + h * 64 + threadIdx.x];
-    __syncthreads();
-    if (j < n_frames) {
-      const T* krow = kc + (((size_t)b * H + h) * t_alloc + j) * 64;
-      const float s = dot64_rot<T>(qs, krow, j) * ATTN_SCALE;
-      const float M = ml[((size_t)r * H + h) * 2 + 0];
-      const float l = ml[((size_t)r * H + h) * 2 + 1];
-      pbar += expf(s - M) / l;
+__global__ void __launch_bounds__(256)
+accept_anchor_kernel(AcceptAnchorArgs A) {
+  __shared__ float qs[32][64];
+  __shared__ float ph[32][ANCHOR_FRAMES + 1];
+  __shared__ int s_n, s_last;
+  pdl_wait();
+  pdl_launch();
+  const int b = blockIdx.y, f0 = blockIdx.x * ANCHOR_FRAMES, tid = threadIdx.x;
+  const int nr = A.plan.n_utt_rows[b];
+  if (nr == 0) {
+    if (blockIdx.x == 0 && tid == 0) {
+      A.accepted[b] = 0;
+      A.bonus[b] = -1;
+      A.kv_len_out[b] = A.kv_len[b];
+      A.anchor_out[b] = -1;
+    }
+    return;
+  }
+  const int r0 = A.plan.row_start[b];
+  if (tid == 0) {
+    const int l = nr - 1;
+    int n = 0;
+    while (n < l && A.draft[(size_t)b * A.k + n] == (int)argmax_index(A.row_key[r0 + n])) ++n;
+    s_n = n;
+    if (blockIdx.x == 0) {
+      const int g = (int)argmax_index(A.row_key[r0 + n]);
+      const int nl = A.kv_len[b] + 1 + n;
+      A.accepted[b] = n;
+      A.bonus[b] = g;
+      A.kv_len[b] = nl;
+      A.kv_len_out[b] = nl;
+      A.pending[b] = g;
     }
   }
-  pbar = pbar / (float)H;
-  unsigned long long key = j < n_frames ? argmax_key(pbar, (uint32_t)j) : 0ull;
-  key = warp_max_u64(key);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = key;
   __syncthreads();
-  if (threadIdx.x == 0) {
-    unsigned long long k = red[0];
-    for (int w = 1; w < ANCHOR_FRAMES / 32; ++w) k = red[w] > k ? red[w] : k;
-    atomicMax(frame_key + b, k);
-    __threadfence();
-    s_last = (atomicAdd(tickets + b, 1) == (int)gridDim.x - 1);
-    if (s_last) {
+  const int r = r0 + s_n;
+  const int H = A.H;
+  for (int e = tid; e < H * 64; e += blockDim.x) {
+    const float v = A.q_anchor[(size_t)r * A.d + e];
+    // the tensor-core attention scored bf16(q / 8) against the bf16 keys
+    qs[e >> 6][e & 63] = A.kv_bf16 ? bf2f(f2bf(v * 0.125f)) : v;
+  }
+  __syncthreads();
+  const int n_frames = A.enc_len[b];
+  const int warp = tid >> 5, lane = tid & 31;
+  const int f = f0 + lane;
+  for (int h = warp; h < H; h += 8) {
+    float p = 0.f;
+    if (f < n_frames) {
+      const T* krow = static_cast<const T*>(A.kc) + (((size_t)b * H + h) * A.t_alloc + f) * 64;
+      float s;
+      if (A.kv_bf16) {
+        // the key row as eight 16-byte loads, all in flight before the sum
+        const uint4* k16 = reinterpret_cast<const uint4*>(krow);
+        uint4 kv[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) kv[u] = __ldg(k16 + u);
+        s = 0.f;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&kv[u]);
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            const float2 kf = __bfloat1622float2(p2[w]);
+            s = fmaf(qs[h][8 * u + 2 * w], kf.x, s);
+            s = fmaf(qs[h][8 * u + 2 * w + 1], kf.y, s);
+          }
+        }
+      } else {
+        s = dot64_rot<T>(qs[h], krow, f) * ATTN_SCALE;
+      }
+      const float M = A.ml[((size_t)r * H + h) * 2 + 0];
+      const float L = A.ml[((size_t)r * H + h) * 2 + 1];
+      p = expf(s - M) / L;
+    }
+    ph[h][lane] = p;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    float pbar = 0.f;
+    for (int h = 0; h < H; ++h) pbar += ph[h][lane];
+    pbar /= (float)H;
+    unsigned long long key = f < n_frames ? argmax_key(pbar, (uint32_t)f) : 0ull;
+    key = warp_max_u64(key);
+    if (lane == 0) {
+      atomicMax(A.frame_key + b, key);
       __threadfence();
-      const unsigned long long fk = atomicExch(frame_key + b, 0ull);
-      anchor_out[b] = (int)argmax_index(fk);
-      tickets[b] = 0;
+      s_last = (atomicAdd(A.tickets + b, 1) == (int)gridDim.x - 1);
+      if (s_last) {
+        __threadfence();
+        const unsigned long long fk = atomicExch(A.frame_key + b, 0ull);
+        A.anchor_out[b] = (int)argmax_index(fk);
+        A.tickets[b] = 0;
+      }
     }
   }
 }
 
-void launch_anchor(const float* q_anchor, const float* ml, const void* kc, int kv_bf16, int t_alloc,
-                   const int* enc_len, const int* anchor_row, int B, int H, int d, unsigned long long* frame_key,
-                   int* tickets, int* anchor_out, cudaStream_t st) {
-  dim3 grid((t_alloc + ANCHOR_FRAMES - 1) / ANCHOR_FRAMES, B);
-  if (kv_bf16)
-    anchor_kernel<__nv_bfloat16><<<grid, ANCHOR_FRAMES, 0, st>>>(q_anchor, ml,
-                                                                 static_cast<const __nv_bfloat16*>(kc), t_alloc,
-                                                                 enc_len, anchor_row, H, d, frame_key, tickets,
-                                                                 anchor_out);
-  else
-    anchor_kernel<float><<<grid, ANCHOR_FRAMES, 0, st>>>(q_anchor, ml, static_cast<const float*>(kc), t_alloc,
-                                                         enc_len, anchor_row, H, d, frame_key, tickets, anchor_out);
+void launch_accept_anchor(const AcceptAnchorArgs& A, cudaStream_t st) {
+  dim3 grid((A.t_alloc + ANCHOR_FRAMES - 1) / ANCHOR_FRAMES, A.B);
+  if (A.kv_bf16) launch_ex(accept_anchor_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, A.pdl, 1, A);
+  else launch_ex(accept_anchor_kernel<float>, grid, dim3(256), 0, st, A.pdl, 1, A);
 }
 
 }  // namespace asrspec

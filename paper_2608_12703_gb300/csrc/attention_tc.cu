@@ -4,16 +4,17 @@
 // Loop": all rows of a draft block are scored in one pass; self-attention is
 // block-causal, cross-attention covers the utterance's encoder frames), laid
 // out for GB300:
-//   * one CTA = one (utterance, head, key chunk); its K and V chunks arrive by
-//     two TMA tile loads into 128-byte-swizzled shared memory (one mbarrier);
+//   * one CTA = one (utterance, head, split); it streams every S-th 128-key
+//     chunk of the utterance's K and V through a 3-deep ring of TMA tile loads
+//     into 128-byte-swizzled shared memory (one mbarrier per slot);
 //   * the utterance's rows (up to 16 per m-tile) are the M side of
-//     mma.sync m16n8k16 (bf16 in, fp32 accumulate): S = Q K^T, then the
+//     mma.sync m16n8k16 (bf16 in, fp32 accumulate): S = Q K^T, then an online
 //     softmax on the accumulator fragments (quad shuffles), then O = P V with
 //     P re-used from the S fragments and V fragments from ldmatrix.trans;
-//   * each of the 4 warps takes a quarter of the chunk's keys; the CTA
-//     combines the warps, writes the chunk's (max, sum, output) and the last
-//     CTA of the (utterance, head) merges all chunks in chunk order, so the
-//     result does not depend on which CTA finishes last.
+//   * each of the 4 warps takes a quarter of every chunk's keys; the CTA
+//     combines its warps, and the S splits of one (utterance, head) form a
+//     thread-block cluster that merges through distributed shared memory in
+//     split order, so the result does not depend on timing.
 #include <mutex>
 
 #include "kernels.h"
@@ -28,7 +29,7 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 }
 
 __device__ __forceinline__ void mma_bf16_16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm volatile(
+  asm(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
@@ -37,7 +38,7 @@ __device__ __forceinline__ void mma_bf16_16816(float* c, const uint32_t* a, uint
 
 __device__ __forceinline__ void ldmatrix_x4_trans(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
                                                   uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+  asm("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
                : "r"(addr));
 }
@@ -47,51 +48,75 @@ __device__ __forceinline__ uint32_t sw128(int row, int chunk16) {
   return (uint32_t)(row * 128 + ((chunk16 ^ (row & 7)) << 4));
 }
 
-template <int CHUNK, int MT>
+constexpr int TCA_CH = 128;        // keys per chunk (one TMA tile of K and one of V)
+constexpr int TCA_STAGES = 3;      // chunks in flight per CTA
+constexpr int TCA_TILE = TCA_CH * 128;
+
+template <int MT>
 struct TcaCfg {
-  static constexpr int KW = CHUNK / 4;        // keys per warp
+  static constexpr int KW = TCA_CH / 4;       // keys per warp per chunk
   static constexpr int NT = KW / 8;           // n-tiles of keys per warp
-  static constexpr int TILE = CHUNK * 128;    // bytes of one K or V tile
+  static constexpr int RING = TCA_STAGES * 2 * TCA_TILE;
   static constexpr int OW = 4 * MT * 16 * 64 * 4;
-  static constexpr int SMEM = 1024 + (2 * TILE > OW ? 2 * TILE : OW);
+  static constexpr int PART = (32 * 64 + 64) * 4;   // this CTA's (max, sum, output) per row
+  static constexpr int SMEM = 1024 + (RING > OW ? RING : OW) + PART;
 };
 
-template <int CHUNK, int MT>
+// One CTA = one (utterance, head, split).  The CTA streams chunks split,
+// split + S, split + 2S, ... of the utterance's keys through a TMA ring,
+// keeping a running (max, sum, output) per row (online softmax).  With S > 1
+// the S splits of a (utterance, head) form one cluster and merge their
+// results through distributed shared memory, in split order.
+template <int MT>
 __global__ void __launch_bounds__(TCA_THREADS)
 attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, AttnArgs a,
                int* status) {
-  using C = TcaCfg<CHUNK, MT>;
+  using C = TcaCfg<MT>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* Ks = smem;
-  uint8_t* Vs = smem + C::TILE;
-  float* Ow = reinterpret_cast<float*>(smem);   // reused after the K/V tiles are consumed
+  float* Ow = reinterpret_cast<float*>(smem);                  // warp partials, after the ring is drained
+  float* Pm = reinterpret_cast<float*>(smem + (C::RING > C::OW ? C::RING : C::OW));   // [32] max
+  float* Pl = Pm + 32;                                          // [32] sum
+  float* Po = Pm + 64;                                          // [32][64] output (relative to max)
   __shared__ float mw[4][MT * 16], lw[4][MT * 16];
-  __shared__ __align__(8) uint64_t bar;
-  __shared__ int s_last;
+  __shared__ __align__(8) uint64_t bar[TCA_STAGES];
 
-  const int chunk = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int S = gridDim.x, split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int nr = a.plan.n_utt_rows[b];
-  if (nr == 0) return;
+  if (nr == 0) {                             // uniform over the cluster
+    pdl_wait();
+    return;
+  }
   const int row0 = a.plan.row_start[b];
   const int n_keys = a.causal ? a.kv_len[b] + nr : a.enc_len[b];
-  const int key0 = chunk * CHUNK;
-  if (key0 >= n_keys) return;
-  const int nc = (n_keys + CHUNK - 1) / CHUNK;
+  const int nc = (n_keys + TCA_CH - 1) / TCA_CH;
+  const int n_iter = split < nc ? (nc - split + S - 1) / S : 0;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, t = lane & 3;
+  const long long rb = ((long long)b * a.H + h) * a.t_alloc;
 
   if (tid == 0) {
-    mbar_init(&bar, 1);
+    for (int st = 0; st < TCA_STAGES; ++st) mbar_init(&bar[st], 1);
     fence_mbar_init();
   }
   __syncthreads();
-  if (tid == 0) {
-    const long long rb = ((long long)b * a.H + h) * a.t_alloc + key0;
-    mbar_arrive_expect_tx(&bar, 2 * C::TILE);
-    tma_load_2d(Ks, &kmap, &bar, 0, (int)(a.k_row0 + rb));
-    tma_load_2d(Vs, &vmap, &bar, 0, (int)(a.v_row0 + rb));
-  }
+  auto issue = [&](int i) {
+    const int st = i % TCA_STAGES;
+    const int key0 = (split + i * S) * TCA_CH;
+    uint8_t* ks = smem + st * 2 * TCA_TILE;
+    mbar_arrive_expect_tx(&bar[st], 2 * TCA_TILE);
+    tma_load_2d(ks, &kmap, &bar[st], 0, (int)(a.k_row0 + rb + key0));
+    tma_load_2d(ks + TCA_TILE, &vmap, &bar[st], 0, (int)(a.v_row0 + rb + key0));
+  };
+  // The encoder K/V cache is constant during a verify call: its first chunks
+  // load while the previous kernel finishes.  Self-attention keys include rows
+  // the previous kernel appends, so those loads wait for it.
+  if (tid == 0 && !a.causal)
+    for (int i = 0; i < n_iter && i < TCA_STAGES; ++i) issue(i);
+  pdl_wait();
+  if (tid == 0 && a.causal)
+    for (int i = 0; i < n_iter && i < TCA_STAGES; ++i) issue(i);
+  pdl_launch();
 
   // queries of this utterance and head as A fragments, pre-scaled by 1/sqrt(64)
   uint32_t qa[MT][4][4];
@@ -111,8 +136,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
       }
     }
   }
-  // visible key limit per fragment row (exclusive)
-  int lim[MT][2];
+  int lim[MT][2];   // visible keys per fragment row (exclusive bound)
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
@@ -121,101 +145,115 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
       lim[mt][e] = (a.causal && r < nr) ? min(n_keys, a.plan.row_pos[row0 + r] + 1) : n_keys;
     }
 
-  mbar_wait(&bar, 0, status);
-
-  // S = Q K^T over this warp's keys
-  float S[MT][C::NT][4];
-  const uint32_t ks_base = smem_u32(Ks), vs_base = smem_u32(Vs);
-#pragma unroll
-  for (int nt = 0; nt < C::NT; ++nt) {
-    const int krow = warp * C::KW + nt * 8 + g;
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt) S[mt][nt][0] = S[mt][nt][1] = S[mt][nt][2] = S[mt][nt][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      uint32_t b0, b1;
-      asm volatile("ld.shared.b32 %0, [%1];" : "=r"(b0) : "r"(ks_base + sw128(krow, 2 * kk) + 4 * t));
-      asm volatile("ld.shared.b32 %0, [%1];" : "=r"(b1) : "r"(ks_base + sw128(krow, 2 * kk + 1) + 4 * t));
-#pragma unroll
-      for (int mt = 0; mt < MT; ++mt) mma_bf16_16816(S[mt][nt], qa[mt][kk], b0, b1);
-    }
-  }
-
-  // masked softmax statistics per row (rows g and g + 8 of each m-tile; a quad shares a row)
-  float m_row[MT][2], l_row[MT][2];
+  float m_run[MT][2], l_run[MT][2], O[MT][8][4];
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
-      float m = -INFINITY;
-#pragma unroll
-      for (int nt = 0; nt < C::NT; ++nt)
-#pragma unroll
-        for (int j = 0; j < 2; ++j) {
-          const int key = key0 + warp * C::KW + nt * 8 + 2 * t + j;
-          float& s = S[mt][nt][2 * e + j];
-          if (key >= lim[mt][e]) s = -INFINITY;
-          m = fmaxf(m, s);
-        }
-      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
-      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
-      const float mu = (m == -INFINITY) ? 0.f : m;
-      float l = 0.f;
-#pragma unroll
-      for (int nt = 0; nt < C::NT; ++nt)
-#pragma unroll
-        for (int j = 0; j < 2; ++j) {
-          float& s = S[mt][nt][2 * e + j];
-          s = (s == -INFINITY) ? 0.f : __expf(s - mu);
-          l += s;
-        }
-      l += __shfl_xor_sync(0xffffffffu, l, 1);
-      l += __shfl_xor_sync(0xffffffffu, l, 2);
-      m_row[mt][e] = m;
-      l_row[mt][e] = l;
+      m_run[mt][e] = -INFINITY;
+      l_run[mt][e] = 0.f;
     }
-  }
-
-  // O = P V over this warp's keys
-  float O[MT][8][4];
-#pragma unroll
-  for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
     for (int nd = 0; nd < 8; ++nd) O[mt][nd][0] = O[mt][nd][1] = O[mt][nd][2] = O[mt][nd][3] = 0.f;
+  }
   const int q4 = lane >> 3, rr = lane & 7;
+
+  for (int i = 0; i < n_iter; ++i) {
+    const int st = i % TCA_STAGES;
+    mbar_wait(&bar[st], (i / TCA_STAGES) & 1, status);
+    const uint32_t ks_base = smem_u32(smem + st * 2 * TCA_TILE);
+    const uint32_t vs_base = ks_base + TCA_TILE;
+    const int kbase = (split + i * S) * TCA_CH + warp * C::KW;
+
+    float Sf[MT][C::NT][4];
 #pragma unroll
-  for (int ks = 0; ks < C::KW / 16; ++ks) {
-    uint32_t pa[MT][4];
+    for (int nt = 0; nt < C::NT; ++nt) {
+      const int krow = warp * C::KW + nt * 8 + g;
 #pragma unroll
-    for (int mt = 0; mt < MT; ++mt) {
-      pa[mt][0] = pack_bf16(S[mt][2 * ks][0], S[mt][2 * ks][1]);
-      pa[mt][1] = pack_bf16(S[mt][2 * ks][2], S[mt][2 * ks][3]);
-      pa[mt][2] = pack_bf16(S[mt][2 * ks + 1][0], S[mt][2 * ks + 1][1]);
-      pa[mt][3] = pack_bf16(S[mt][2 * ks + 1][2], S[mt][2 * ks + 1][3]);
-    }
-    const int vrow = warp * C::KW + ks * 16 + (q4 & 1) * 8 + rr;
+      for (int mt = 0; mt < MT; ++mt) Sf[mt][nt][0] = Sf[mt][nt][1] = Sf[mt][nt][2] = Sf[mt][nt][3] = 0.f;
 #pragma unroll
-    for (int nd2 = 0; nd2 < 4; ++nd2) {
-      uint32_t r0, r1, r2, r3;
-      ldmatrix_x4_trans(vs_base + sw128(vrow, nd2 * 2 + (q4 >> 1)), r0, r1, r2, r3);
+      for (int kk = 0; kk < 4; ++kk) {
+        uint32_t b0, b1;
+        asm("ld.shared.b32 %0, [%1];" : "=r"(b0) : "r"(ks_base + sw128(krow, 2 * kk) + 4 * t));
+        asm("ld.shared.b32 %0, [%1];" : "=r"(b1) : "r"(ks_base + sw128(krow, 2 * kk + 1) + 4 * t));
 #pragma unroll
-      for (int mt = 0; mt < MT; ++mt) {
-        mma_bf16_16816(O[mt][2 * nd2], pa[mt], r0, r1);
-        mma_bf16_16816(O[mt][2 * nd2 + 1], pa[mt], r2, r3);
+        for (int mt = 0; mt < MT; ++mt) mma_bf16_16816(Sf[mt][nt], qa[mt][kk], b0, b1);
       }
     }
+    // online softmax: new running max, rescale, accumulate
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        float cm = -INFINITY;
+#pragma unroll
+        for (int nt = 0; nt < C::NT; ++nt)
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            float& s = Sf[mt][nt][2 * e + j];
+            if (kbase + nt * 8 + 2 * t + j >= lim[mt][e]) s = -INFINITY;
+            cm = fmaxf(cm, s);
+          }
+        cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, 1));
+        cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, 2));
+        const float m_new = fmaxf(m_run[mt][e], cm);
+        const float mu = (m_new == -INFINITY) ? 0.f : m_new;
+        const float alpha = __expf(m_run[mt][e] - mu);
+        float l = 0.f;
+#pragma unroll
+        for (int nt = 0; nt < C::NT; ++nt)
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            float& s = Sf[mt][nt][2 * e + j];
+            s = __expf(s - mu);
+            l += s;
+          }
+        l += __shfl_xor_sync(0xffffffffu, l, 1);
+        l += __shfl_xor_sync(0xffffffffu, l, 2);
+        l_run[mt][e] = l_run[mt][e] * alpha + l;
+        m_run[mt][e] = m_new;
+#pragma unroll
+        for (int nd = 0; nd < 8; ++nd) {
+          O[mt][nd][2 * e + 0] *= alpha;
+          O[mt][nd][2 * e + 1] *= alpha;
+        }
+      }
+    }
+#pragma unroll
+    for (int ks = 0; ks < C::KW / 16; ++ks) {
+      uint32_t pa[MT][4];
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) {
+        pa[mt][0] = pack_bf16(Sf[mt][2 * ks][0], Sf[mt][2 * ks][1]);
+        pa[mt][1] = pack_bf16(Sf[mt][2 * ks][2], Sf[mt][2 * ks][3]);
+        pa[mt][2] = pack_bf16(Sf[mt][2 * ks + 1][0], Sf[mt][2 * ks + 1][1]);
+        pa[mt][3] = pack_bf16(Sf[mt][2 * ks + 1][2], Sf[mt][2 * ks + 1][3]);
+      }
+      const int vrow = warp * C::KW + ks * 16 + (q4 & 1) * 8 + rr;
+#pragma unroll
+      for (int nd2 = 0; nd2 < 4; ++nd2) {
+        uint32_t r0, r1, r2, r3;
+        ldmatrix_x4_trans(vs_base + sw128(vrow, nd2 * 2 + (q4 >> 1)), r0, r1, r2, r3);
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+          mma_bf16_16816(O[mt][2 * nd2], pa[mt], r0, r1);
+          mma_bf16_16816(O[mt][2 * nd2 + 1], pa[mt], r2, r3);
+        }
+      }
+    }
+    __syncthreads();   // every warp is done with stage st
+    if (tid == 0 && i + TCA_STAGES < n_iter) issue(i + TCA_STAGES);
   }
 
-  // combine the four warps of the CTA
-  __syncthreads();   // every warp is done with the K/V tiles; Ow reuses them
+  // combine the four warps into this CTA's (max, sum, output) per row
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
       const int r = mt * 16 + g + 8 * e;
       if (t == 0) {
-        mw[warp][r] = m_row[mt][e];
-        lw[warp][r] = l_row[mt][e];
+        mw[warp][r] = m_run[mt][e];
+        lw[warp][r] = l_run[mt][e];
       }
 #pragma unroll
       for (int nd = 0; nd < 8; ++nd) {
@@ -226,7 +264,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
     }
   }
   __syncthreads();
-  float* part = a.part + (((size_t)b * a.H + h) * a.n_chunks + chunk) * a.k1 * 66;
   for (int e = tid; e < nr * 64; e += TCA_THREADS) {
     const int r = e >> 6, c = e & 63;
     float M = -INFINITY;
@@ -236,106 +273,68 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
     float L = 0.f, o = 0.f;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
-      const float f = (mw[w][r] == -INFINITY) ? 0.f : __expf(mw[w][r] - Mu);
+      const float f = __expf(mw[w][r] - Mu);
       L += lw[w][r] * f;
       o += Ow[(size_t)(w * MT * 16 + r) * 64 + c] * f;
     }
-    part[r * 66 + c] = o;
+    Po[r * 64 + c] = o;
     if (c == 0) {
-      part[r * 66 + 64] = M;
-      part[r * 66 + 65] = L;
+      Pm[r] = M;
+      Pl[r] = L;
     }
   }
 
-  // the last CTA of this (utterance, head) merges the chunks in chunk order
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) s_last = (atomicAdd(a.tickets + b * a.H + h, 1) == nc - 1);
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  // chunk weights first (one thread per (row, chunk), all loads in flight at
-  // once), then every output element as one pass over the chunks
-  const float* pb = a.part + ((size_t)b * a.H + h) * a.n_chunks * a.k1 * 66;
-  const size_t cstride = (size_t)a.k1 * 66;
-  float* wgt = Ow;                               // [nr][nc] chunk weights, then [nr] sums
-  float* Lsum = Ow + MT * 16 * 32;
-  for (int e = tid; e < nr * nc; e += TCA_THREADS) {
-    const int r = e / nc, ci = e - r * nc;
-    wgt[r * 32 + ci] = __ldcg(pb + ci * cstride + r * 66 + 64);
-    Lsum[r * 32 + ci] = __ldcg(pb + ci * cstride + r * 66 + 65);
-  }
-  __syncthreads();
-  if (tid < nr) {
-    float M = -INFINITY;
-    for (int ci = 0; ci < nc; ++ci) M = fmaxf(M, wgt[tid * 32 + ci]);
-    float L = 0.f;
-    for (int ci = 0; ci < nc; ++ci) {
-      const float mc = wgt[tid * 32 + ci];
-      const float f = (mc == -INFINITY) ? 0.f : __expf(mc - M);
-      L += Lsum[tid * 32 + ci] * f;
-      wgt[tid * 32 + ci] = f;
-    }
-    for (int ci = 0; ci < nc; ++ci) wgt[tid * 32 + ci] /= L;
-    if (a.ml_out) {
-      a.ml_out[((size_t)(row0 + tid) * a.H + h) * 2 + 0] = M;
-      a.ml_out[((size_t)(row0 + tid) * a.H + h) * 2 + 1] = L;
-    }
-  }
-  __syncthreads();
-  for (int e = tid; e < nr * 64; e += TCA_THREADS) {
+  // merge the splits of this (utterance, head) in split order
+  if (S > 1) cluster_sync();
+  else __syncthreads();
+  for (int e = split * TCA_THREADS + tid; e < nr * 64; e += S * TCA_THREADS) {
     const int r = e >> 6, c = e & 63;
-    float o = 0.f;
-    int ci = 0;
-    for (; ci + 4 <= nc; ci += 4) {
-      const float p0 = __ldcg(pb + (ci + 0) * cstride + r * 66 + c);
-      const float p1 = __ldcg(pb + (ci + 1) * cstride + r * 66 + c);
-      const float p2 = __ldcg(pb + (ci + 2) * cstride + r * 66 + c);
-      const float p3 = __ldcg(pb + (ci + 3) * cstride + r * 66 + c);
-      o += p0 * wgt[r * 32 + ci];
-      o += p1 * wgt[r * 32 + ci + 1];
-      o += p2 * wgt[r * 32 + ci + 2];
-      o += p3 * wgt[r * 32 + ci + 3];
+    float M = -INFINITY;
+    for (int s = 0; s < S; ++s) M = fmaxf(M, S > 1 ? ld_dsmem_f32(dsmem_addr(Pm + r, s)) : Pm[r]);
+    const float Mu = (M == -INFINITY) ? 0.f : M;
+    float L = 0.f, o = 0.f;
+    for (int s = 0; s < S; ++s) {
+      const float ms = S > 1 ? ld_dsmem_f32(dsmem_addr(Pm + r, s)) : Pm[r];
+      const float ls = S > 1 ? ld_dsmem_f32(dsmem_addr(Pl + r, s)) : Pl[r];
+      const float os = S > 1 ? ld_dsmem_f32(dsmem_addr(Po + r * 64 + c, s)) : Po[r * 64 + c];
+      const float f = __expf(ms - Mu);
+      L += ls * f;
+      o += os * f;
     }
-    for (; ci < nc; ++ci) o += __ldcg(pb + ci * cstride + r * 66 + c) * wgt[r * 32 + ci];
-    reinterpret_cast<__nv_bfloat16*>(a.out)[(size_t)(row0 + r) * a.d + h * 64 + c] = f2bf(o);
+    reinterpret_cast<__nv_bfloat16*>(a.out)[(size_t)(row0 + r) * a.d + h * 64 + c] = f2bf(o / L);
+    if (a.ml_out && c == 0) {
+      a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 0] = M;
+      a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 1] = L;
+    }
   }
-  if (tid == 0) a.tickets[b * a.H + h] = 0;
+  if (S > 1) cluster_sync();   // no CTA leaves while another may still read its shared memory
 }
 
-template <int CHUNK, int MT>
+template <int MT>
 static void configure_one() {
-  cudaFuncSetAttribute(attn_tc_kernel<CHUNK, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       TcaCfg<CHUNK, MT>::SMEM);
+  cudaFuncSetAttribute(attn_tc_kernel<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcaCfg<MT>::SMEM);
 }
 
 void configure_attention_tc() {
   static std::once_flag once;
   std::call_once(once, [] {
-    configure_one<128, 1>();
-    configure_one<128, 2>();
-    configure_one<256, 1>();
-    configure_one<256, 2>();
+    configure_one<1>();
+    configure_one<2>();
   });
 }
 
-template <int CHUNK, int MT>
-static void launch_one(const AttnArgs& a, int* status, cudaStream_t st) {
-  dim3 grid((a.t_alloc + CHUNK - 1) / CHUNK, a.H, a.B);
-  attn_tc_kernel<CHUNK, MT><<<grid, TCA_THREADS, TcaCfg<CHUNK, MT>::SMEM, st>>>(*a.kmap, *a.vmap, a, status);
+template <int MT>
+static void launch_one(const AttnArgs& a, int splits, int* status, cudaStream_t st) {
+  launch_ex(attn_tc_kernel<MT>, dim3(splits, a.H, a.B), dim3(TCA_THREADS), TcaCfg<MT>::SMEM, st, a.pdl, splits,
+            *a.kmap, *a.vmap, a, status);
 }
 
-// chunk: 128 or 256 keys; rows_max > 16 takes two m-tiles
+// a.splits CTAs (1, 2, 4 or 8; one cluster) per (utterance, head);
+// rows_max > 16 takes two m-tiles.
 void launch_attention_tc(const AttnArgs& a, int* status, cudaStream_t st) {
   configure_attention_tc();
-  const bool two = a.rows_max > 16;
-  if (a.chunk == 128) {
-    if (two) launch_one<128, 2>(a, status, st);
-    else launch_one<128, 1>(a, status, st);
-  } else {
-    if (two) launch_one<256, 2>(a, status, st);
-    else launch_one<256, 1>(a, status, st);
-  }
+  if (a.rows_max > 16) launch_one<2>(a, a.splits, status, st);
+  else launch_one<1>(a, a.splits, status, st);
 }
 
 bool make_tmap_cache(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {

@@ -101,4 +101,71 @@ __device__ __forceinline__ void epi_apply(const Epi& e, int m, int n, float acc)
   }
 }
 
+// U output elements at once.  The residual update loads every x value before
+// it stores any (the elements are distinct, so no store can feed a later
+// load), which keeps U loads in flight instead of U dependent round trips.
+template <int MODE, int U>
+__device__ __forceinline__ void epi_batch(const Epi& e, const int* m, const int* n, const float* v,
+                                          const bool* ok) {
+  if constexpr (MODE == EPI_RESID) {
+    float old[U], bias[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      old[u] = ok[u] ? e.x[(size_t)n[u] * e.d + m[u]] : 0.f;
+      bias[u] = ok[u] ? e.bias[m[u]] : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (ok[u]) e.x[(size_t)n[u] * e.d + m[u]] = old[u] + (v[u] + bias[u]);
+  } else if constexpr (MODE == EPI_QKV) {
+    // row metadata and biases first, then the stores
+    float bias[U];
+    int rb[U], rp[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      bias[u] = ok[u] ? e.bias[m[u]] : 0.f;
+      rb[u] = ok[u] && m[u] >= e.d ? e.row_b[n[u]] : 0;
+      rp[u] = ok[u] && m[u] >= e.d ? e.row_pos[n[u]] : 0;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (!ok[u]) continue;
+      const float val = v[u] + bias[u];
+      if (m[u] < e.d) {
+        e.out_f32[(size_t)n[u] * e.d + m[u]] = val;
+      } else {
+        const int which = (m[u] - e.d) / e.d;
+        const int f = (m[u] - e.d) - which * e.d;
+        const size_t idx = (((size_t)rb[u] * e.n_heads + (f >> 6)) * e.max_pos + rp[u]) * 64 + (f & 63);
+        void* base = which == 0 ? e.kcache : e.vcache;
+        if (e.kv_bf16) store_as<__nv_bfloat16>(base, idx, val);
+        else store_as<float>(base, idx, val);
+      }
+    }
+  } else if constexpr (MODE == EPI_Q) {
+    float bias[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) bias[u] = ok[u] ? e.bias[m[u]] : 0.f;
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (ok[u]) e.out_f32[(size_t)n[u] * e.d + m[u]] = v[u] + bias[u];
+  } else if constexpr (MODE == EPI_GELU) {
+    float bias[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) bias[u] = ok[u] ? e.bias[m[u]] : 0.f;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (!ok[u]) continue;
+      const float g = gelu_erf(v[u] + bias[u]);
+      const size_t idx = (size_t)n[u] * e.M + m[u];
+      if (e.act_bf16) store_as<__nv_bfloat16>(e.act, idx, g);
+      else store_as<float>(e.act, idx, g);
+    }
+  } else {
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (ok[u]) epi_apply<MODE>(e, m[u], n[u], v[u]);
+  }
+}
+
 }  // namespace asrspec

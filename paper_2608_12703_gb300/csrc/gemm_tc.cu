@@ -7,8 +7,14 @@
 //   warp 0 / lane 0 : TMA producer, STAGES-deep ring of (A, B) k-blocks
 //   warp 1 / lane 0 : issues tcgen05.mma (M=128, N=BN, K=16) x 4 per k-block
 //   warps 0..3      : epilogue, each reading its 32 TMEM lanes (= 32 values of m)
-// Split-K partials go to a workspace; the last CTA of a tile (atomic ticket)
-// sums them in split order, so results do not depend on CTA timing.
+// Split K, two ways, both summing the partials in split order so that results
+// do not depend on CTA timing:
+//   * cluster split (CLU): the splits of a tile form one thread-block cluster;
+//     each CTA stages its partial tile in its own shared memory, and after a
+//     cluster barrier every CTA sums a slice of the tile's rows over all
+//     splits through distributed shared memory and runs the epilogue on it;
+//   * workspace split: partials go to a global workspace and the last CTA of
+//     the tile (atomic ticket) sums them.
 #include <cstdio>
 #include <mutex>
 
@@ -18,20 +24,24 @@ namespace asrspec {
 
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;
-constexpr int TC_STAGES = 4;
 
 template <int BN>
 struct TcCfg {
+  // 4-deep ring for narrow tiles; 3-deep for 128-wide tiles so that two CTAs
+  // share an SM (one CTA's epilogue overlaps the other's main loop)
+  static constexpr int STAGES = BN == 128 ? 3 : 4;
   static constexpr int A_BYTES = TC_BM * TC_BK * 2;
   static constexpr int B_BYTES = BN * TC_BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int BAR_OFF = TC_STAGES * STAGE_BYTES;
+  static constexpr int BAR_OFF = STAGES * STAGE_BYTES;
   static constexpr int SMEM = 1024 + BAR_OFF + 256;
-  static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+  // tcgen05.alloc takes a power of two of at least 32 columns
+  static constexpr uint32_t TMEM_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "N tile of one tcgen05.mma (M = 128)");
   static_assert(B_BYTES % 1024 == 0, "B tile must keep 1024-byte alignment");
 };
 
-template <int BN, int MODE>
+template <int BN, int MODE, bool CLU>
 __global__ void __launch_bounds__(128, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, int K, int splits,
                float* __restrict__ ws, int* __restrict__ tickets, Epi epi, int* status) {
@@ -39,15 +49,18 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
-  uint8_t* sB = smem + TC_STAGES * C::A_BYTES;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::BAR_OFF);
-  uint64_t* empty = full + TC_STAGES;
-  uint64_t* done = empty + TC_STAGES;
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* done = empty + C::STAGES;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   __shared__ unsigned long long red[4][BN];
   __shared__ int s_last;
 
-  const int tile_m = blockIdx.x, tile_n = blockIdx.y, split = blockIdx.z;
+  // cluster split: the splits of a tile are consecutive CTAs along x (one cluster)
+  const int tile_m = CLU ? (int)blockIdx.x / splits : (int)blockIdx.x;
+  const int split = CLU ? (int)blockIdx.x % splits : (int)blockIdx.z;
+  const int tile_n = blockIdx.y;
   const int m0 = tile_m * TC_BM, n0 = tile_n * BN;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_valid = epi.n_valid ? *epi.n_valid : epi.N;
@@ -55,14 +68,17 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   const int kb0 = (nkb_total * split) / splits;
   const int kb1 = (nkb_total * (split + 1)) / splits;
   const int nkb = kb1 - kb0;
-  if (n0 >= n_valid || nkb <= 0) return;  // uniform over the CTA and over all splits of a tile
+  if (n0 >= n_valid || nkb <= 0) {       // uniform over the CTA and over all splits of a tile
+    pdl_wait();
+    return;
+  }
 
   if (warp == 0) {
     tmem_alloc(tmem_slot, C::TMEM_COLS);
     tmem_relinquish();
   }
   if (threadIdx.x == 32) {
-    for (int s = 0; s < TC_STAGES; ++s) {
+    for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
@@ -77,10 +93,20 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&mapA);
     tma_prefetch_desc(&mapB);
-    int issued = 0;
-    for (int i = 0; i < nkb; ++i) {
-      const int s = i % TC_STAGES;
-      const uint32_t ph = (i / TC_STAGES) & 1;
+    // The weights (A) do not depend on the previous kernel: fill the ring with
+    // them first, then wait for the predecessor before loading activations (B).
+    const int first = nkb < C::STAGES ? nkb : C::STAGES;
+    for (int i = 0; i < first; ++i) {
+      mbar_arrive_expect_tx(&full[i], C::STAGE_BYTES);
+      tma_load_2d(sA + i * C::A_BYTES, &mapA, &full[i], (kb0 + i) * TC_BK, m0);
+    }
+    pdl_wait();
+    for (int i = 0; i < first; ++i) tma_load_2d(sB + i * C::B_BYTES, &mapB, &full[i], (kb0 + i) * TC_BK, n0);
+    pdl_launch();
+    int issued = first;
+    for (int i = first; i < nkb; ++i) {
+      const int s = i % C::STAGES;
+      const uint32_t ph = (i / C::STAGES) & 1;
       if (!mbar_wait(&empty[s], ph ^ 1, status)) break;
       mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
       tma_load_2d(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0);
@@ -88,13 +114,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       issued = i + 1;
     }
     // Drain: every issued copy has landed before this CTA can exit.
-    for (int i = issued - TC_STAGES > 0 ? issued - TC_STAGES : 0; i < issued; ++i)
-      mbar_wait(&full[i % TC_STAGES], (i / TC_STAGES) & 1, status);
+    for (int i = issued - C::STAGES > 0 ? issued - C::STAGES : 0; i < issued; ++i)
+      mbar_wait(&full[i % C::STAGES], (i / C::STAGES) & 1, status);
   } else if (warp == 1 && lane == 0) {
     constexpr uint32_t idesc = umma_idesc_bf16(TC_BM, BN);
     for (int i = 0; i < nkb; ++i) {
-      const int s = i % TC_STAGES;
-      const uint32_t ph = (i / TC_STAGES) & 1;
+      const int s = i % C::STAGES;
+      const uint32_t ph = (i / C::STAGES) & 1;
       if (!mbar_wait(&full[s], ph, status)) break;
       tc_fence_after();
       const uint32_t a_addr = smem_u32(sA + s * C::A_BYTES);
@@ -106,6 +132,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       umma_commit(&empty[s]);
     }
     umma_commit(done);
+  }
+  if (!(warp == 0 && lane == 0)) {
+    pdl_wait();
+    pdl_launch();
   }
   __syncwarp();
   mbar_wait(done, 0, status);
@@ -128,11 +158,15 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
           if (lane == 0) red[warp][c0 + i] = key;
         }
       } else {
+        int mm[16], nn[16];
+        bool ok[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const int n = n0 + c0 + i;
-          if (m < epi.M && n < n_valid) epi_apply<MODE>(epi, m, n, v[i]);
+          mm[i] = m;
+          nn[i] = n0 + c0 + i;
+          ok[i] = m < epi.M && nn[i] < n_valid;
         }
+        epi_batch<MODE, 16>(epi, mm, nn, v, ok);
       }
     }
     if constexpr (MODE == EPI_ARGMAX) {
@@ -145,6 +179,63 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
         if (n < n_valid) atomicMax(epi.row_key + n, k);
       }
     }
+  } else if constexpr (CLU) {
+    // stage this split's tile in shared memory (the pipeline buffers are free now)
+    constexpr int LD = BN + 4;
+    float* red = reinterpret_cast<float*>(smem);
+    const int ml = warp * 32 + lane;
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(t_lane + c0, v);
+#pragma unroll
+      for (int i = 0; i < 16; i += 4)
+        *reinterpret_cast<float4*>(red + ml * LD + c0 + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+    }
+    cluster_sync();
+    // this CTA sums rows [rank * 128 / splits, (rank + 1) * 128 / splits) over all splits
+    const int rows_per = TC_BM / splits;
+    const int r_first = split * rows_per;
+    const int items = rows_per * (BN / 4);
+    constexpr int IU = 4;   // items per pass: IU float4 loads from every split in flight
+    for (int base = threadIdx.x; base < items; base += IU * blockDim.x) {
+      float4 acc[IU];
+      const float* local[IU];
+      int mm[4 * IU], nn[4 * IU];
+      bool ok[4 * IU];
+#pragma unroll
+      for (int u = 0; u < IU; ++u) {
+        const int it = base + u * blockDim.x;
+        const int row = r_first + (it % rows_per), c4 = it / rows_per;
+        local[u] = red + row * LD + 4 * (c4 < BN / 4 ? c4 : 0);
+        acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          mm[4 * u + i] = m0 + row;
+          nn[4 * u + i] = n0 + 4 * c4 + i;
+          ok[4 * u + i] = it < items && m0 + row < epi.M && n0 + 4 * c4 + i < n_valid;
+        }
+      }
+      for (int s = 0; s < splits; ++s) {
+        float4 p[IU];
+#pragma unroll
+        for (int u = 0; u < IU; ++u) p[u] = ld_dsmem_f4(dsmem_addr(local[u], (uint32_t)s));
+#pragma unroll
+        for (int u = 0; u < IU; ++u) {
+          acc[u].x += p[u].x; acc[u].y += p[u].y; acc[u].z += p[u].z; acc[u].w += p[u].w;
+        }
+      }
+      float vals[4 * IU];
+#pragma unroll
+      for (int u = 0; u < IU; ++u) {
+        vals[4 * u + 0] = acc[u].x;
+        vals[4 * u + 1] = acc[u].y;
+        vals[4 * u + 2] = acc[u].z;
+        vals[4 * u + 3] = acc[u].w;
+      }
+      epi_batch<MODE == EPI_ARGMAX ? EPI_F32 : MODE, 4 * IU>(epi, mm, nn, vals, ok);
+    }
+    cluster_sync();   // no CTA leaves while another may still read its shared memory
   } else {
     const int tile = tile_n * gridDim.x + tile_m;
     float* my = ws + ((size_t)(tile * splits + split) * TC_BM + warp * 32 + lane) * BN;
@@ -196,15 +287,23 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
             acc[q].x += p[q].x; acc[q].y += p[q].y; acc[q].z += p[q].z; acc[q].w += p[q].w;
           }
         }
+        int mm[16], nn[16];
+        bool ok[16];
+        float vals[16];
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          const float a4[4] = {acc[q].x, acc[q].y, acc[q].z, acc[q].w};
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int n = n0 + c0 + 4 * q + i;
-            if (m < epi.M && n < n_valid) epi_apply<MODE == EPI_ARGMAX ? EPI_F32 : MODE>(epi, m, n, a4[i]);
-          }
+          vals[4 * q + 0] = acc[q].x;
+          vals[4 * q + 1] = acc[q].y;
+          vals[4 * q + 2] = acc[q].z;
+          vals[4 * q + 3] = acc[q].w;
         }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          mm[i] = m;
+          nn[i] = n0 + c0 + i;
+          ok[i] = m < epi.M && nn[i] < n_valid;
+        }
+        epi_batch<MODE == EPI_ARGMAX ? EPI_F32 : MODE, 16>(epi, mm, nn, vals, ok);
       }
       if (threadIdx.x == 0) tickets[tile] = 0;
     }
@@ -266,15 +365,37 @@ size_t tc_smem_bytes(int bn) {
     case 32: return TcCfg<32>::SMEM;
     case 64: return TcCfg<64>::SMEM;
     case 128: return TcCfg<128>::SMEM;
+    case 192: return TcCfg<192>::SMEM;
+    case 224: return TcCfg<224>::SMEM;
     default: return TcCfg<256>::SMEM;
   }
 }
 
+// N tile for many rows: fewest tiles first, then the least padding.
+int tc_pick_bn_wide(int n) {
+  const int cand[4] = {128, 192, 224, 256};
+  int best = 256, best_nt = 1 << 30, best_pad = 1 << 30;
+  for (int c : cand) {
+    const int nt = (n + c - 1) / c, pad = nt * c - n;
+    if (nt < best_nt || (nt == best_nt && pad < best_pad)) {
+      best = c;
+      best_nt = nt;
+      best_pad = pad;
+    }
+  }
+  return best;
+}
+
 template <int BN, int MODE>
 static void launch_tc_t(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
-  auto kern = gemm_tc_kernel<BN, MODE>;
-  dim3 grid((g.M + TC_BM - 1) / TC_BM, (g.N + BN - 1) / BN, g.splits);
-  kern<<<grid, 128, TcCfg<BN>::SMEM, st>>>(g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
+  const int mt = (g.M + TC_BM - 1) / TC_BM, nt = (g.N + BN - 1) / BN;
+  if (g.cluster && g.splits > 1) {
+    launch_ex(gemm_tc_kernel<BN, MODE, true>, dim3(mt * g.splits, nt, 1), dim3(128), TcCfg<BN>::SMEM, st, g.pdl,
+              g.splits, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
+    return;
+  }
+  launch_ex(gemm_tc_kernel<BN, MODE, false>, dim3(mt, nt, g.splits), dim3(128), TcCfg<BN>::SMEM, st, g.pdl, 1,
+            g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
 }
 
 template <int MODE>
@@ -284,17 +405,28 @@ static void launch_tc_mode(const TcGemm& g, const Epi& epi, int* status, cudaStr
     case 32: launch_tc_t<32, MODE>(g, epi, status, st); break;
     case 64: launch_tc_t<64, MODE>(g, epi, status, st); break;
     case 128: launch_tc_t<128, MODE>(g, epi, status, st); break;
+    case 192: launch_tc_t<192, MODE>(g, epi, status, st); break;
+    case 224: launch_tc_t<224, MODE>(g, epi, status, st); break;
     default: launch_tc_t<256, MODE>(g, epi, status, st); break;
   }
 }
 
+template <int BN, int MODE>
+static void configure_one() {
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+}
+
 template <int MODE>
 static void configure_mode() {
-  cudaFuncSetAttribute(gemm_tc_kernel<16, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<16>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<32, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<32>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<64, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<64>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<128, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<128>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<256, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<256>::SMEM);
+  configure_one<16, MODE>();
+  configure_one<32, MODE>();
+  configure_one<64, MODE>();
+  configure_one<128, MODE>();
+  configure_one<192, MODE>();
+  configure_one<224, MODE>();
+  configure_one<256, MODE>();
 }
 
 // Opt every instance into its dynamic shared memory once, before any launch or

@@ -16,14 +16,17 @@ struct TcGemm {
   CUtensorMap mapA;
   CUtensorMap mapB;
   int M, N, K;
-  int bn;        // N tile: 16, 32, 64, 128 or 256
+  int bn;        // N tile: 16, 32, 64, 128, 192, 224 or 256
   int splits;    // split-K factor (1 = none)
-  float* ws;     // split-K partials (splits * tiles * 128 * bn floats)
-  int* tickets;  // one zeroed int per output tile
+  float* ws;     // workspace split: partials (splits * tiles * 128 * bn floats)
+  int* tickets;  // workspace split: one zeroed int per output tile
+  bool cluster = false;  // split K inside a thread-block cluster (splits in {2,4,8,16})
+  bool pdl = false;      // programmatic dependent launch after the previous kernel
 };
 
 bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
 int tc_pick_bn(int n_max);
+int tc_pick_bn_wide(int n);
 void launch_gemm_tc(const TcGemm& g, int mode, const Epi& epi, int* status, cudaStream_t st);
 size_t tc_smem_bytes(int bn);
 void configure_gemm_tc();
@@ -61,10 +64,10 @@ void launch_plan_verify(const int* draft, const int* lens, int k, int B, int voc
 void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,
                                RowPlan plan, int* status, cudaStream_t st);
 void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
-                  cudaStream_t st);
+                  cudaStream_t st, bool pdl = false);
 // y = LN(x) * g + b over rows < n_rows, written as bf16 or fp32.
 void launch_layernorm(const float* x, const float* g, const float* b, void* y, int y_bf16, const int* n_rows,
-                      int R_max, int d, cudaStream_t st);
+                      int R_max, int d, cudaStream_t st, bool pdl = false);
 
 // ---- Attention ---------------------------------------------------------------
 struct AttnArgs {
@@ -92,21 +95,34 @@ struct AttnArgs {
   long long k_row0 = 0, v_row0 = 0;
   int* tickets = nullptr;
   int rows_max = 0;        // most rows of one utterance in this call
+  int splits = 1;          // CTAs (one cluster) per (utterance, head)
+  bool pdl = false;        // programmatic dependent launch
 };
 void launch_attention(const AttnArgs& a, cudaStream_t st);
 void launch_attention_tc(const AttnArgs& a, int* status, cudaStream_t st);
 // Tensor map over a [rows][64] bf16 cache with `box_rows`-row boxes.
 bool make_tmap_cache(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows);
 
-// Anchor readout: head-mean softmax of row anchor_row[b] at the anchor layer.
-void launch_anchor(const float* q_anchor, const float* ml, const void* kc, int kv_bf16, int t_alloc,
-                   const int* enc_len, const int* anchor_row, int B, int H, int d,
-                   unsigned long long* frame_key, int* tickets, int* anchor_out, cudaStream_t st);
+// Acceptance + commit + anchor readout (one kernel).
+struct AcceptAnchorArgs {
+  const int* draft;                 // [B][k]
+  int k, B, H, d, t_alloc, kv_bf16;
+  RowPlan plan;
+  const unsigned long long* row_key;
+  int* kv_len;
+  int* pending;
+  int *accepted, *bonus, *kv_len_out, *anchor_out;
+  const float* q_anchor;            // [R][d] cross-attention queries at the anchor layer
+  const float* ml;                  // [R][H][2] their softmax (max, sum)
+  const void* kc;                   // anchor layer's encoder keys [B_max][H][t_alloc][64]
+  const int* enc_len;
+  unsigned long long* frame_key;    // [B_max], zero between calls
+  int* tickets;                     // [B_max], zero between calls
+  bool pdl;
+};
+void launch_accept_anchor(const AcceptAnchorArgs& a, cudaStream_t st);
 
 // ---- Accept / commit ------------------------------------------------------------
-void launch_accept(const int* draft, const int* lens, int k, int B, RowPlan plan, const unsigned long long* row_key,
-                   int* kv_len, int* pending, int* accepted, int* bonus, int* kv_len_out, int* anchor_row,
-                   int* anchor_out, cudaStream_t st);
 void launch_prefill_advance(int B, int c, const int* n_utt_rows, int* kv_len, cudaStream_t st);
 void launch_prefill_finish(const int* prompt, int P0, int B, int* pending, const int* ready, cudaStream_t st);
 void launch_rollback(const int* new_len, const int* new_pending, int B, int vocab, int* kv_len, int* pending,

@@ -158,6 +158,8 @@ void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, 
 template <typename T>
 __global__ void embed_kernel(const T* __restrict__ tok_emb, const T* __restrict__ pos_emb, RowPlan plan, int d,
                              float* __restrict__ x) {
+  pdl_wait();
+  pdl_launch();
   const int r = blockIdx.x;
   if (r >= *plan.n_rows) return;
   const int t = plan.row_tok[r], p = plan.row_pos[r];
@@ -166,13 +168,13 @@ __global__ void embed_kernel(const T* __restrict__ tok_emb, const T* __restrict_
 }
 
 void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
-                  cudaStream_t st) {
+                  cudaStream_t st, bool pdl) {
   if (w_bf16)
-    embed_kernel<__nv_bfloat16><<<R_max, 128, 0, st>>>(static_cast<const __nv_bfloat16*>(tok_emb),
-                                                       static_cast<const __nv_bfloat16*>(pos_emb), plan, d, x);
+    launch_ex(embed_kernel<__nv_bfloat16>, dim3(R_max), dim3(128), 0, st, pdl, 1,
+              static_cast<const __nv_bfloat16*>(tok_emb), static_cast<const __nv_bfloat16*>(pos_emb), plan, d, x);
   else
-    embed_kernel<float><<<R_max, 128, 0, st>>>(static_cast<const float*>(tok_emb),
-                                               static_cast<const float*>(pos_emb), plan, d, x);
+    launch_ex(embed_kernel<float>, dim3(R_max), dim3(128), 0, st, pdl, 1, static_cast<const float*>(tok_emb),
+              static_cast<const float*>(pos_emb), plan, d, x);
 }
 
 // LayerNorm, one warp per row, statistics in fp32: a sum pass and a centred
@@ -181,6 +183,8 @@ template <typename TO>
 __global__ void __launch_bounds__(256)
 layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const float* __restrict__ bta,
                  TO* __restrict__ y, const int* __restrict__ n_rows, int d) {
+  pdl_wait();
+  pdl_launch();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = blockIdx.x * 8 + warp;
   if (r >= *n_rows) return;
@@ -212,50 +216,13 @@ layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const
 }
 
 void launch_layernorm(const float* x, const float* g, const float* b, void* y, int y_bf16, const int* n_rows,
-                      int R_max, int d, cudaStream_t st) {
-  const int grid = (R_max + 7) / 8;
+                      int R_max, int d, cudaStream_t st, bool pdl) {
+  const dim3 grid((R_max + 7) / 8);
   if (y_bf16)
-    layernorm_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(x, g, b, static_cast<__nv_bfloat16*>(y), n_rows, d);
+    launch_ex(layernorm_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, pdl, 1, x, g, b,
+              static_cast<__nv_bfloat16*>(y), n_rows, d);
   else
-    layernorm_kernel<float><<<grid, 256, 0, st>>>(x, g, b, static_cast<float*>(y), n_rows, d);
-}
-
-// Greedy longest-prefix acceptance (Sec. 3 "Speculative Loop") and commit:
-// n = longest prefix with draft[j] == argmax of row j; bonus = argmax of row n;
-// kv_len += 1 + n (App. "Correction and Cost": a round advances 1 + L tokens).
-__global__ void accept_kernel(const int* __restrict__ draft, const int* __restrict__ lens, int k, int B,
-                              RowPlan plan, const unsigned long long* __restrict__ row_key, int* kv_len, int* pending,
-                              int* accepted, int* bonus, int* kv_len_out, int* anchor_row, int* anchor_out) {
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b >= B) return;
-  const int nr = plan.n_utt_rows[b];
-  if (nr == 0) {
-    accepted[b] = 0;
-    bonus[b] = -1;
-    kv_len_out[b] = kv_len[b];
-    anchor_row[b] = -1;
-    anchor_out[b] = -1;
-    return;
-  }
-  const int r0 = plan.row_start[b];
-  const int l = nr - 1;
-  int n = 0;
-  while (n < l && draft[(size_t)b * k + n] == (int)argmax_index(row_key[r0 + n])) ++n;
-  const int g = (int)argmax_index(row_key[r0 + n]);
-  accepted[b] = n;
-  bonus[b] = g;
-  const int nl = kv_len[b] + 1 + n;
-  kv_len[b] = nl;
-  kv_len_out[b] = nl;
-  pending[b] = g;
-  anchor_row[b] = r0 + n;
-}
-
-void launch_accept(const int* draft, const int* lens, int k, int B, RowPlan plan, const unsigned long long* row_key,
-                   int* kv_len, int* pending, int* accepted, int* bonus, int* kv_len_out, int* anchor_row,
-                   int* anchor_out, cudaStream_t st) {
-  accept_kernel<<<(B + 127) / 128, 128, 0, st>>>(draft, lens, k, B, plan, row_key, kv_len, pending, accepted, bonus,
-                                                 kv_len_out, anchor_row, anchor_out);
+    launch_ex(layernorm_kernel<float>, grid, dim3(256), 0, st, pdl, 1, x, g, b, static_cast<float*>(y), n_rows, d);
 }
 
 // After a prefill chunk: the rows' K/V are cached, so the committed length moves on.

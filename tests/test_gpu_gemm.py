@@ -6,10 +6,11 @@ import torch
 pytestmark = pytest.mark.gpu
 
 SHAPES = [(128, 16, 64), (300, 9, 1280), (3840, 9, 1280), (1280, 40, 5120), (517, 200, 384),
-          (1024, 256, 768), (640, 448, 1280), (51866, 9, 1280), (256, 137, 3072)]
+          (1024, 256, 768), (640, 448, 1280), (51866, 9, 1280), (256, 137, 3072), (1280, 544, 3072),
+          (3840, 448, 1280)]
 
 
-@pytest.mark.parametrize("impl", [0, 2, 1])
+@pytest.mark.parametrize("impl", [0, 2, 4, 1])
 @pytest.mark.parametrize("M,N,K", SHAPES)
 def test_gemm_matches_torch(built_lib, cuda, impl, M, N, K):
     from paper_2608_12703_gb300 import asrspec as A
