@@ -75,6 +75,9 @@ struct asr_spec {
   // CUDA graphs of the verify body, keyed by (B, k)
   bool use_graphs = true;
   bool use_pdl = true;   // programmatic dependent launch between verify kernels
+  bool lm_ln_fused = false;   // the last verify's LM head normalised x itself (xf not written)
+  int wide_bn = 64;      // N tile for many rows (ASRSPEC_WIDE_BN: 64, 128, 192, 224, 256)
+  int wide_target = 2 * 152;   // CTAs a many-row GEMM may fill by splitting K (ASRSPEC_WIDE_TARGET)
   struct Graph {
     cudaGraphExec_t exec;
     long long launches[ASR_PROF_N];
@@ -188,21 +191,24 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   }
   TcGemm g{};
   g.mapA = *mW;
+  g.mapB = *mW;   // unused when the B operand is LayerNorm(x) written by the kernel
   // Few rows (batch 1): one narrow N tile and K split across the CTAs of a
-  // cluster so that every SM streams weights.  Many rows: 128-wide N tiles
-  // (two CTAs per SM), K split in a cluster while the grid stays within one
-  // wave and every split keeps at least four k-blocks.  Split factors are
-  // powers of two up to 16.
-  g.bn = N <= 64 ? tc_pick_bn(N) : 128;
-  const CUtensorMap* mb = bmap(h, x_id, X, h->R_pad, K, g.bn);
-  if (!mb) return fail(h, ASR_E_CUDA, "tensor map encode failed");
-  g.mapB = *mb;
+  // cluster so that every SM streams weights.  Many rows: 64-wide N tiles
+  // (two CTAs per SM; measured best at batch 64 against 128 and 256), K split
+  // in a cluster while the grid stays within one wave and every split keeps at
+  // least four k-blocks.  Split factors are powers of two up to 16.
+  g.bn = N <= 64 ? tc_pick_bn(N) : h->wide_bn;
+  if (!epi.ln_x) {
+    const CUtensorMap* mb = bmap(h, x_id, X, h->R_pad, K, g.bn);
+    if (!mb) return fail(h, ASR_E_CUDA, "tensor map encode failed");
+    g.mapB = *mb;
+  }
   g.M = M;
   g.N = N;
   g.K = K;
   const int tiles = ((M + 127) / 128) * ((N + g.bn - 1) / g.bn);
   const int nkb = K / 64;
-  const int target = 2 * NUM_SMS_TARGET;
+  const int target = N <= 64 ? 2 * NUM_SMS_TARGET : h->wide_target;
   g.splits = 1;
   if (mode != EPI_ARGMAX && mode != EPI_F32)
     while (g.splits < 16 && tiles * g.splits * 2 <= target && g.splits * 2 <= (N <= 64 ? nkb : nkb / 4))
@@ -217,13 +223,35 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
 
 enum BufId { BUF_XN = 1, BUF_ATT = 2, BUF_H = 3, BUF_XF = 4 };
 
+// A projection whose input is LayerNorm(x).  Few rows (bf16): the GEMM
+// normalises its own B tiles from x (no separate LayerNorm launch).  Otherwise
+// a LayerNorm kernel writes `ln_out` and the GEMM loads it by TMA.
+int gemm_rows_ln(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, const float* g, const float* b,
+                 void* ln_out, int ln_out_id, int N, int mode, const Epi& epi_in, bool* fused = nullptr) {
+  Epi e = epi_in;
+  const bool fuse = h->bf16 && N <= 64;
+  if (fused) *fused = fuse;
+  if (fuse) {
+    e.ln_x = h->x;
+    e.ln_g = g;
+    e.ln_b = b;
+    return gemm_rows(h, W, mW, M, K, nullptr, ln_out_id, N, mode, e);
+  }
+  {
+    Prof p(h, ASR_PROF_OTHER, 1);
+    launch_layernorm(h->x, g, b, ln_out, h->bf16, h->plan.n_rows, N, K, h->st, h->use_pdl);
+  }
+  return gemm_rows(h, W, mW, M, K, ln_out, ln_out_id, N, mode, e);
+}
+
 // The decoder layers over the rows laid out by the last plan kernel.
 // CTAs per (utterance, head) for the tensor-core attention: few utterances
 // (batch 1) split the keys over a cluster of up to 8 CTAs.
 int attn_splits_for(asr_spec* h, int t_alloc) {
   const int nc_max = (t_alloc + 127) / 128;
   int S = 1;
-  while (S < 8 && S * 2 <= nc_max && h->B * h->H * S * 2 <= 2 * NUM_SMS_TARGET) S *= 2;
+  // split until every SM has two CTAs (the ring of each keeps 96 KB in flight)
+  while (S < 8 && S * 2 <= nc_max && h->B * h->H * S < 2 * NUM_SMS_TARGET) S *= 2;
   return S;
 }
 
@@ -273,16 +301,13 @@ int run_layers(asr_spec* h, int N) {
     char* kx = static_cast<char*>(h->xkv) + (size_t)l * 2 * cross_half;
     char* vx = kx + cross_half;
     // self-attention block
-    {
-      Prof p(h, ASR_PROF_OTHER, 1);
-      launch_layernorm(h->x, w.ln1g, w.ln1b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st, h->use_pdl);
-    }
     Epi e = base;
     e.bias = w.bqkv;
     e.out_f32 = h->q;
     e.kcache = ks;
     e.vcache = vs;
-    if (int rc = gemm_rows(h, w.wqkv, &w.m_wqkv, 3 * d, d, h->xn, BUF_XN, N, EPI_QKV, e)) return rc;
+    if (int rc = gemm_rows_ln(h, w.wqkv, &w.m_wqkv, 3 * d, d, w.ln1g, w.ln1b, h->xn, BUF_XN, N, EPI_QKV, e))
+      return rc;
     AttnArgs a{};
     a.q = h->q;
     a.kc = ks;
@@ -313,15 +338,11 @@ int run_layers(asr_spec* h, int N) {
     e.x = h->x;
     if (int rc = gemm_rows(h, w.wo, &w.m_wo, d, d, h->att, BUF_ATT, N, EPI_RESID, e)) return rc;
     // cross-attention block
-    {
-      Prof p(h, ASR_PROF_OTHER, 1);
-      launch_layernorm(h->x, w.ln2g, w.ln2b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st, h->use_pdl);
-    }
     float* qc = (l == h->anchor) ? h->q_anchor : h->q;
     e = base;
     e.bias = w.bcq;
     e.out_f32 = qc;
-    if (int rc = gemm_rows(h, w.wcq, &w.m_wcq, d, d, h->xn, BUF_XN, N, EPI_Q, e)) return rc;
+    if (int rc = gemm_rows_ln(h, w.wcq, &w.m_wcq, d, d, w.ln2g, w.ln2b, h->xn, BUF_XN, N, EPI_Q, e)) return rc;
     a.q = qc;
     a.kc = kx;
     a.vc = vx;
@@ -338,14 +359,10 @@ int run_layers(asr_spec* h, int N) {
     e.x = h->x;
     if (int rc = gemm_rows(h, w.wco, &w.m_wco, d, d, h->att, BUF_ATT, N, EPI_RESID, e)) return rc;
     // MLP block
-    {
-      Prof p(h, ASR_PROF_OTHER, 1);
-      launch_layernorm(h->x, w.ln3g, w.ln3b, h->xn, h->bf16, h->plan.n_rows, N, d, h->st, h->use_pdl);
-    }
     e = base;
     e.bias = w.b1;
     e.act = h->hbuf;
-    if (int rc = gemm_rows(h, w.w1, &w.m_w1, h->F, d, h->xn, BUF_XN, N, EPI_GELU, e)) return rc;
+    if (int rc = gemm_rows_ln(h, w.w1, &w.m_w1, h->F, d, w.ln3g, w.ln3b, h->xn, BUF_XN, N, EPI_GELU, e)) return rc;
     e = base;
     e.bias = w.b2;
     e.x = h->x;
@@ -383,15 +400,13 @@ int enqueue_verify(asr_spec* h, int k) {
   }
   const int N = B * (k + 1);
   if (int rc = run_layers(h, N)) return rc;
-  {
-    Prof p(h, ASR_PROF_OTHER, 1);
-    launch_layernorm(h->x, h->lnf_g, h->lnf_b, h->xf, h->bf16, h->plan.n_rows, N, h->d, h->st, h->use_pdl);
-  }
   Epi e{};
   e.n_valid = h->plan.n_rows;
   e.row_key = h->row_key;
   e.d = h->d;
-  if (int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, N, EPI_ARGMAX, e)) return rc;
+  if (int rc = gemm_rows_ln(h, h->w_tok, &h->m_tok, h->V, h->d, h->lnf_g, h->lnf_b, h->xf, BUF_XF, N, EPI_ARGMAX, e,
+                            &h->lm_ln_fused))
+    return rc;
   Prof p(h, ASR_PROF_OTHER, 1);
   AcceptAnchorArgs A{};
   A.draft = h->draft_buf;
@@ -443,6 +458,11 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   h->anchor = dims->anchor_layer >= 0 ? dims->anchor_layer : (3 * h->L) / 4;
   h->bf16 = dims->dtype == 1;
   if (const char* e = std::getenv("ASRSPEC_PDL")) h->use_pdl = std::atoi(e) != 0;
+  if (const char* e = std::getenv("ASRSPEC_WIDE_BN")) {
+    const int v = std::atoi(e);
+    if (v == 64 || v == 128 || v == 192 || v == 224 || v == 256) h->wide_bn = v;
+  }
+  if (const char* e = std::getenv("ASRSPEC_WIDE_TARGET")) h->wide_target = std::max(1, std::atoi(e));
   h->es = h->bf16 ? 2 : 4;
   h->st = static_cast<cudaStream_t>(stream);
   if (!h->st) {
@@ -830,6 +850,11 @@ int asr_spec_debug_logits(asr_spec_handle h, float* out, int32_t max_rows) {
   e.out_f32 = dst;
   e.ld = h->V;
   e.n_valid = h->plan.n_rows;
+  if (h->lm_ln_fused && h->bf16) {   // same B operand as the fused argmax: LayerNorm(x) built in the GEMM
+    e.ln_x = h->x;
+    e.ln_g = h->lnf_g;
+    e.ln_b = h->lnf_b;
+  }
   int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, R, EPI_F32, e);
   if (!rc && h->host_io) {
     CK(cudaMemcpyAsync(out, tmp, (size_t)R * h->V * 4, cudaMemcpyDeviceToHost, h->st));

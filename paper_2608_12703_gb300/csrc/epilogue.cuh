@@ -48,6 +48,10 @@ struct Epi {
   int b_max = 0;
   // LM head argmax
   unsigned long long* row_key = nullptr;
+  // B operand = LayerNorm(ln_x) (few-row GEMMs): fp32 rows [N][K], gain and bias [K]
+  const float* ln_x = nullptr;
+  const float* ln_g = nullptr;
+  const float* ln_b = nullptr;
 };
 
 template <typename T>

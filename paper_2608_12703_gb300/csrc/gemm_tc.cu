@@ -41,7 +41,11 @@ struct TcCfg {
   static_assert(B_BYTES % 1024 == 0, "B tile must keep 1024-byte alignment");
 };
 
-template <int BN, int MODE, bool CLU>
+// Named barrier of the two B-writer warps (warps 2 and 3) of the LayerNorm path.
+__device__ __forceinline__ void writers_sync() { asm volatile("bar.sync 1, 64;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+template <int BN, int MODE, bool CLU, bool LNB>
 __global__ void __launch_bounds__(128, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, int K, int splits,
                float* __restrict__ ws, int* __restrict__ tickets, Epi epi, int* status) {
@@ -56,6 +60,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   __shared__ unsigned long long red[4][BN];
   __shared__ int s_last;
+  __shared__ float ln_mean[LNB ? BN : 1], ln_rstd[LNB ? BN : 1];
 
   // cluster split: the splits of a tile are consecutive CTAs along x (one cluster)
   const int tile_m = CLU ? (int)blockIdx.x / splits : (int)blockIdx.x;
@@ -79,7 +84,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   }
   if (threadIdx.x == 32) {
     for (int s = 0; s < C::STAGES; ++s) {
-      mbar_init(&full[s], 1);
+      mbar_init(&full[s], LNB ? 2 : 1);   // LayerNorm path: TMA (A) + the B writers
       mbar_init(&empty[s], 1);
     }
     mbar_init(done, 1);
@@ -95,22 +100,24 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     tma_prefetch_desc(&mapB);
     // The weights (A) do not depend on the previous kernel: fill the ring with
     // them first, then wait for the predecessor before loading activations (B).
+    constexpr uint32_t TX = LNB ? C::A_BYTES : C::STAGE_BYTES;
     const int first = nkb < C::STAGES ? nkb : C::STAGES;
     for (int i = 0; i < first; ++i) {
-      mbar_arrive_expect_tx(&full[i], C::STAGE_BYTES);
+      mbar_arrive_expect_tx(&full[i], TX);
       tma_load_2d(sA + i * C::A_BYTES, &mapA, &full[i], (kb0 + i) * TC_BK, m0);
     }
     pdl_wait();
-    for (int i = 0; i < first; ++i) tma_load_2d(sB + i * C::B_BYTES, &mapB, &full[i], (kb0 + i) * TC_BK, n0);
+    if constexpr (!LNB)
+      for (int i = 0; i < first; ++i) tma_load_2d(sB + i * C::B_BYTES, &mapB, &full[i], (kb0 + i) * TC_BK, n0);
     pdl_launch();
     int issued = first;
     for (int i = first; i < nkb; ++i) {
       const int s = i % C::STAGES;
       const uint32_t ph = (i / C::STAGES) & 1;
       if (!mbar_wait(&empty[s], ph ^ 1, status)) break;
-      mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
+      mbar_arrive_expect_tx(&full[s], TX);
       tma_load_2d(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0);
-      tma_load_2d(sB + s * C::B_BYTES, &mapB, &full[s], (kb0 + i) * TC_BK, n0);
+      if constexpr (!LNB) tma_load_2d(sB + s * C::B_BYTES, &mapB, &full[s], (kb0 + i) * TC_BK, n0);
       issued = i + 1;
     }
     // Drain: every issued copy has landed before this CTA can exit.
@@ -132,8 +139,76 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       umma_commit(&empty[s]);
     }
     umma_commit(done);
+  } else if (LNB && warp >= 2) {
+    // B = bf16(LayerNorm(x)) rows n0 .. n0 + BN - 1, written straight into the
+    // 128-byte-swizzled K-major tile the MMA reads.  Statistics first: one pass
+    // of shifted sums per row (shift = the row's first element).
+    pdl_wait();
+    pdl_launch();
+    const int t = threadIdx.x - 64;
+    for (int r = warp - 2; r < BN; r += 2) {
+      const int n = n0 + r;
+      float mean = 0.f, rstd = 0.f;
+      if (n < n_valid) {
+        const float* xr = epi.ln_x + (size_t)n * K;
+        const float sh = __ldg(xr);
+        const float4* x4 = reinterpret_cast<const float4*>(xr);
+        float s1 = 0.f, s2 = 0.f;
+#pragma unroll 4
+        for (int i = lane; i < K / 4; i += 32) {
+          const float4 v = x4[i];
+          const float a = v.x - sh, b = v.y - sh, c = v.z - sh, e = v.w - sh;
+          s1 += (a + b) + (c + e);
+          s2 += (a * a + b * b) + (c * c + e * e);
+        }
+        s1 = warp_sum(s1);
+        s2 = warp_sum(s2);
+        const float m1 = s1 / (float)K;
+        mean = sh + m1;
+        rstd = rsqrtf(fmaxf(s2 / (float)K - m1 * m1, 0.f) + 1e-5f);
+      }
+      if (lane == 0) {
+        ln_mean[r] = mean;
+        ln_rstd[r] = rstd;
+      }
+    }
+    writers_sync();
+    for (int i = 0; i < nkb; ++i) {
+      const int s = i % C::STAGES;
+      const uint32_t ph = (i / C::STAGES) & 1;
+      if (!mbar_wait(&empty[s], ph ^ 1, status)) break;
+      const int k0 = (kb0 + i) * TC_BK;
+      uint8_t* bt = sB + s * C::B_BYTES;
+      for (int id = t; id < BN * 4; id += 64) {      // BN rows x 4 runs of 16 columns
+        const int r = id >> 2, c0 = (id & 3) * 16, n = n0 + r;
+        uint32_t w[8];
+        if (n < n_valid) {
+          const float4* x4 = reinterpret_cast<const float4*>(epi.ln_x + (size_t)n * K + k0 + c0);
+          const float4* g4 = reinterpret_cast<const float4*>(epi.ln_g + k0 + c0);
+          const float4* b4 = reinterpret_cast<const float4*>(epi.ln_b + k0 + c0);
+          const float mu = ln_mean[r], rs = ln_rstd[r];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float4 v = x4[q], gg = __ldg(g4 + q), bb = __ldg(b4 + q);
+            __nv_bfloat162 lo = __floats2bfloat162_rn((v.x - mu) * rs * gg.x + bb.x, (v.y - mu) * rs * gg.y + bb.y);
+            __nv_bfloat162 hi = __floats2bfloat162_rn((v.z - mu) * rs * gg.z + bb.z, (v.w - mu) * rs * gg.w + bb.w);
+            w[2 * q] = *reinterpret_cast<uint32_t*>(&lo);
+            w[2 * q + 1] = *reinterpret_cast<uint32_t*>(&hi);
+          }
+        } else {
+#pragma unroll
+          for (int q = 0; q < 8; ++q) w[q] = 0u;
+        }
+        const int ch = c0 >> 3;   // first 16-byte chunk of this run
+        *reinterpret_cast<uint4*>(bt + r * 128 + (((ch) ^ (r & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+        *reinterpret_cast<uint4*>(bt + r * 128 + (((ch + 1) ^ (r & 7)) << 4)) = make_uint4(w[4], w[5], w[6], w[7]);
+      }
+      fence_async_smem();   // make the generic-proxy writes visible to the tensor core
+      writers_sync();
+      if (t == 0) mbar_arrive(&full[s]);
+    }
   }
-  if (!(warp == 0 && lane == 0)) {
+  if (!(warp == 0 && lane == 0) && !(LNB && warp >= 2)) {
     pdl_wait();
     pdl_launch();
   }
@@ -386,16 +461,34 @@ int tc_pick_bn_wide(int n) {
   return best;
 }
 
+// LayerNorm-fused B operand exists for the few-row tiles (BN <= 64) of the
+// modes whose input is a LayerNorm output.
 template <int BN, int MODE>
-static void launch_tc_t(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
+constexpr bool ln_capable() {
+  return BN <= 64 && (MODE == EPI_QKV || MODE == EPI_Q || MODE == EPI_GELU || MODE == EPI_ARGMAX || MODE == EPI_F32);
+}
+
+template <int BN, int MODE, bool LNB>
+static void launch_tc_ln(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
   const int mt = (g.M + TC_BM - 1) / TC_BM, nt = (g.N + BN - 1) / BN;
   if (g.cluster && g.splits > 1) {
-    launch_ex(gemm_tc_kernel<BN, MODE, true>, dim3(mt * g.splits, nt, 1), dim3(128), TcCfg<BN>::SMEM, st, g.pdl,
-              g.splits, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
+    launch_ex(gemm_tc_kernel<BN, MODE, true, LNB>, dim3(mt * g.splits, nt, 1), dim3(128), TcCfg<BN>::SMEM, st,
+              g.pdl, g.splits, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
     return;
   }
-  launch_ex(gemm_tc_kernel<BN, MODE, false>, dim3(mt, nt, g.splits), dim3(128), TcCfg<BN>::SMEM, st, g.pdl, 1,
+  launch_ex(gemm_tc_kernel<BN, MODE, false, LNB>, dim3(mt, nt, g.splits), dim3(128), TcCfg<BN>::SMEM, st, g.pdl, 1,
             g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
+}
+
+template <int BN, int MODE>
+static void launch_tc_t(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
+  if constexpr (ln_capable<BN, MODE>()) {
+    if (epi.ln_x) {
+      launch_tc_ln<BN, MODE, true>(g, epi, status, st);
+      return;
+    }
+  }
+  launch_tc_ln<BN, MODE, false>(g, epi, status, st);
 }
 
 template <int MODE>
@@ -411,11 +504,19 @@ static void launch_tc_mode(const TcGemm& g, const Epi& epi, int* status, cudaStr
   }
 }
 
+template <int BN, int MODE, bool LNB>
+static void configure_ln() {
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, LNB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       TcCfg<BN>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, LNB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       TcCfg<BN>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, LNB>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+}
+
 template <int BN, int MODE>
 static void configure_one() {
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  configure_ln<BN, MODE, false>();
+  if constexpr (ln_capable<BN, MODE>()) configure_ln<BN, MODE, true>();
 }
 
 template <int MODE>

@@ -177,11 +177,11 @@ void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan 
               static_cast<const float*>(pos_emb), plan, d, x);
 }
 
-// LayerNorm, one warp per row, statistics in fp32: a sum pass and a centred
-// sum-of-squares pass over the row (L2-resident), then the affine write.
+// LayerNorm for any d % 4 == 0: a sum pass, a centred sum-of-squares pass over the
+// row (L2-resident), then the affine write.
 template <typename TO>
 __global__ void __launch_bounds__(256)
-layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const float* __restrict__ bta,
+layernorm_any_kernel(const float* __restrict__ x, const float* __restrict__ g, const float* __restrict__ bta,
                  TO* __restrict__ y, const int* __restrict__ n_rows, int d) {
   pdl_wait();
   pdl_launch();
@@ -215,14 +215,80 @@ layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const
   }
 }
 
+// LayerNorm, one warp per row, statistics in fp32.  The row is read once into
+// registers (N4 float4 per lane), then mean, centred variance and the affine
+// write come from the registers.
+template <typename TO, int N4>
+__global__ void __launch_bounds__(256)
+layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const float* __restrict__ bta,
+                 TO* __restrict__ y, const int* __restrict__ n_rows, int d) {
+  pdl_wait();
+  pdl_launch();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + warp;
+  if (r >= *n_rows) return;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)r * d);
+  float4 v[N4];
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < N4; ++i) {
+    v[i] = xr[lane + 32 * i];
+    s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
+  }
+  const float mean = warp_sum(s) / (float)d;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < N4; ++i) {
+    const float a = v[i].x - mean, b = v[i].y - mean, c = v[i].z - mean, e = v[i].w - mean;
+    q += (a * a + b * b) + (c * c + e * e);
+  }
+  const float rstd = rsqrtf(warp_sum(q) / (float)d + 1e-5f);
+  TO* yr = y + (size_t)r * d;
+#pragma unroll
+  for (int i = 0; i < N4; ++i) {
+    const int c4 = lane + 32 * i;
+    const float4 gg = reinterpret_cast<const float4*>(g)[c4];
+    const float4 bb = reinterpret_cast<const float4*>(bta)[c4];
+    yr[4 * c4 + 0] = from_f<TO>((v[i].x - mean) * rstd * gg.x + bb.x);
+    yr[4 * c4 + 1] = from_f<TO>((v[i].y - mean) * rstd * gg.y + bb.y);
+    yr[4 * c4 + 2] = from_f<TO>((v[i].z - mean) * rstd * gg.z + bb.z);
+    yr[4 * c4 + 3] = from_f<TO>((v[i].w - mean) * rstd * gg.w + bb.w);
+  }
+}
+
+template <typename TO>
+static void launch_ln_t(const float* x, const float* g, const float* b, TO* y, const int* n_rows, int R_max, int d,
+                        cudaStream_t st, bool pdl) {
+  const dim3 grid((R_max + 7) / 8), block(256);
+  switch (d / 128) {   // d is a multiple of 64; d % 128 == 64 rounds up with a guarded tail
+    case 1: launch_ex(layernorm_kernel<TO, 1>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 2: launch_ex(layernorm_kernel<TO, 2>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 3: launch_ex(layernorm_kernel<TO, 3>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 4: launch_ex(layernorm_kernel<TO, 4>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 5: launch_ex(layernorm_kernel<TO, 5>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 6: launch_ex(layernorm_kernel<TO, 6>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 8: launch_ex(layernorm_kernel<TO, 8>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 10: launch_ex(layernorm_kernel<TO, 10>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 12: launch_ex(layernorm_kernel<TO, 12>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 16: launch_ex(layernorm_kernel<TO, 16>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    default: launch_ex(layernorm_any_kernel<TO>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+  }
+}
+
 void launch_layernorm(const float* x, const float* g, const float* b, void* y, int y_bf16, const int* n_rows,
                       int R_max, int d, cudaStream_t st, bool pdl) {
-  const dim3 grid((R_max + 7) / 8);
-  if (y_bf16)
-    launch_ex(layernorm_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, pdl, 1, x, g, b,
-              static_cast<__nv_bfloat16*>(y), n_rows, d);
-  else
-    launch_ex(layernorm_kernel<float>, grid, dim3(256), 0, st, pdl, 1, x, g, b, static_cast<float*>(y), n_rows, d);
+  if (d % 128) {   // widths that are not a whole number of float4 per lane
+    const dim3 grid((R_max + 7) / 8);
+    if (y_bf16)
+      launch_ex(layernorm_any_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, pdl, 1, x, g, b,
+                static_cast<__nv_bfloat16*>(y), n_rows, d);
+    else
+      launch_ex(layernorm_any_kernel<float>, grid, dim3(256), 0, st, pdl, 1, x, g, b, static_cast<float*>(y),
+                n_rows, d);
+    return;
+  }
+  if (y_bf16) launch_ln_t(x, g, b, static_cast<__nv_bfloat16*>(y), n_rows, R_max, d, st, pdl);
+  else launch_ln_t(x, g, b, static_cast<float*>(y), n_rows, R_max, d, st, pdl);
 }
 
 // After a prefill chunk: the rows' K/V are cached, so the committed length moves on.

@@ -30,6 +30,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=2)
     ap.add_argument("--rounds", type=int, default=3)
     ap.add_argument("--no-graphs", action="store_true")
+    ap.add_argument("--classes", action="store_true",
+                    help="also time each kernel class with CUDA events (direct launches)")
     args = ap.parse_args()
 
     import torch
@@ -64,6 +66,15 @@ def main():
     st = sess.status()
     print(f"{wl.name}: verify rounds {len(us)}, us per round: " + " ".join(f"{u:.1f}" for u in us)
           + f"; status {st}")
+    if args.classes:
+        A.asr_spec_profile_read(sess.h)
+        A.asr_spec_profile(sess.h, True)
+        for i in range(args.rounds):
+            sess.verify_device(drafts[i], lens, wl.k)
+        ms, launches, _ = A.asr_spec_profile_read(sess.h)
+        A.asr_spec_profile(sess.h, False)
+        print("  per round (us, event-bracketed direct launches): " + ", ".join(
+            f"{n} {1e3 * m / args.rounds:.0f}" for n, m in zip(A.PROF_CLASSES, ms)))
     sess.close()
     if st:
         sys.exit(1)
