@@ -52,6 +52,10 @@ struct Epi {
   const float* ln_x = nullptr;
   const float* ln_g = nullptr;
   const float* ln_b = nullptr;
+  // optional phase timestamps (ns, %globaltimer) per CTA: [CTA][8]
+  // (entry, set-up done, first stage full, MMAs done, end; cluster split:
+  // partials staged, first cluster barrier passed, reduction done)
+  unsigned long long* trace = nullptr;
 };
 
 template <typename T>

@@ -9,10 +9,16 @@
 //   warps 0..3      : epilogue, each reading its 32 TMEM lanes (= 32 values of m)
 // Split K, two ways, both summing the partials in split order so that results
 // do not depend on CTA timing:
-//   * cluster split (CLU): the splits of a tile form one thread-block cluster;
-//     each CTA stages its partial tile in its own shared memory, and after a
-//     cluster barrier every CTA sums a slice of the tile's rows over all
-//     splits through distributed shared memory and runs the epilogue on it;
+//   * cluster split (CLU): the splits of a tile form one thread-block cluster
+//     and CTA r of the cluster owns rows [r * 128 / splits, (r + 1) * 128 /
+//     splits) of the tile.  Narrow tiles (BN <= 64) push: every CTA writes
+//     each row of its partial straight into the owner's receive buffer with
+//     st.async, which counts the bytes on the owner's mbarrier, so an owner
+//     waits for exactly its own data and no cluster-wide barrier sits on the
+//     critical path.  Wide tiles pull: each CTA stages its partial, and after
+//     a cluster barrier the owners read the slices through distributed shared
+//     memory.  Either way the owner sums its rows over the splits and runs
+//     the epilogue on them;
 //   * workspace split: partials go to a global workspace and the last CTA of
 //     the tile (atomic ticket) sums them.
 #include <cstdio>
@@ -25,16 +31,22 @@ namespace asrspec {
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;
 
-template <int BN>
+template <int BN, bool PUSH = false>
 struct TcCfg {
-  // 4-deep ring for narrow tiles; 3-deep for 128-wide tiles so that two CTAs
-  // share an SM (one CTA's epilogue overlaps the other's main loop)
-  static constexpr int STAGES = BN == 128 ? 3 : 4;
+  // 4-deep ring for narrow tiles; 3-deep for 128-wide tiles, and for 64-wide
+  // tiles with a receive buffer, so that two CTAs share an SM (one CTA's
+  // epilogue overlaps the other's main loop)
+  static constexpr int STAGES = (BN == 128 || (PUSH && BN == 64)) ? 3 : 4;
   static constexpr int A_BYTES = TC_BM * TC_BK * 2;
   static constexpr int B_BYTES = BN * TC_BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int BAR_OFF = STAGES * STAGE_BYTES;
-  static constexpr int SMEM = 1024 + BAR_OFF + 256;
+  // push split: receive buffer [split][row of the owner's slice][RECV_LD]
+  // (= 128 rows), padded by 16 bytes per row against bank conflicts
+  static constexpr int RECV_LD = BN + 4;
+  static constexpr int RECV_OFF = BAR_OFF + 256;
+  static constexpr int RECV_BYTES = PUSH ? TC_BM * RECV_LD * 4 : 0;
+  static constexpr int SMEM = 1024 + BAR_OFF + 256 + RECV_BYTES;
   // tcgen05.alloc takes a power of two of at least 32 columns
   static constexpr uint32_t TMEM_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
   static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "N tile of one tcgen05.mma (M = 128)");
@@ -45,11 +57,16 @@ struct TcCfg {
 __device__ __forceinline__ void writers_sync() { asm volatile("bar.sync 1, 64;" ::: "memory"); }
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
-template <int BN, int MODE, bool CLU, bool LNB>
+// MC: the N tiles of one M tile form a cluster (grid y = cluster y); each
+// k-block's A tile is loaded once, by CTA (k-block mod cluster size), and
+// multicast to every CTA of the cluster; an MMA commit frees the slot in all
+// of them, so a slot is refilled only after every CTA has consumed it.
+template <int BN, int MODE, bool CLU, bool LNB, bool MC>
 __global__ void __launch_bounds__(128, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, int K, int splits,
                float* __restrict__ ws, int* __restrict__ tickets, Epi epi, int* status) {
-  using C = TcCfg<BN>;
+  constexpr bool PUSH = CLU && BN <= 64;
+  using C = TcCfg<BN, PUSH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -57,7 +74,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::BAR_OFF);
   uint64_t* empty = full + C::STAGES;
   uint64_t* done = empty + C::STAGES;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* recv_bar = done + 1;   // push split: the peers' partial rows have landed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 2);
+  float* recv = reinterpret_cast<float*>(smem + C::RECV_OFF);
   __shared__ unsigned long long red[4][BN];
   __shared__ int s_last;
   __shared__ float ln_mean[LNB ? BN : 1], ln_rstd[LNB ? BN : 1];
@@ -68,15 +87,22 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   const int tile_n = blockIdx.y;
   const int m0 = tile_m * TC_BM, n0 = tile_n * BN;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  unsigned long long* tr = epi.trace ? epi.trace + 8ull * (blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z))
+                                     : nullptr;
+  if (tr && threadIdx.x == 0) tr[0] = global_ns();
   const int n_valid = epi.n_valid ? *epi.n_valid : epi.N;
   const int nkb_total = K / TC_BK;
   const int kb0 = (nkb_total * split) / splits;
   const int kb1 = (nkb_total * (split + 1)) / splits;
   const int nkb = kb1 - kb0;
-  if (n0 >= n_valid || nkb <= 0) {       // uniform over the CTA and over all splits of a tile
+  if (!MC && (n0 >= n_valid || nkb <= 0)) {   // uniform over the CTA and over all splits of a tile
     pdl_wait();
     return;
   }
+  // multicast clusters keep every CTA: the others wait on its share of A and its commits
+  const uint32_t mc_rank = MC ? cluster_ctarank() : 0;
+  const uint32_t mc_size = MC ? gridDim.y : 1;
+  const uint16_t mc_mask = (uint16_t)((1u << mc_size) - 1u);
 
   if (warp == 0) {
     tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -85,15 +111,25 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   if (threadIdx.x == 32) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], LNB ? 2 : 1);   // LayerNorm path: TMA (A) + the B writers
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], MC ? mc_size : 1);
     }
     mbar_init(done, 1);
+    if constexpr (PUSH) {
+      // the other splits each send this CTA's slice of their partial tile
+      mbar_init(recv_bar, 1);
+      mbar_arrive_expect_tx(recv_bar, (uint32_t)((splits - 1) * (TC_BM / splits) * BN * 4));
+    }
     fence_mbar_init();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if constexpr (MC) cluster_sync();   // every CTA's barriers exist before any multicast lands
+  // push split: announce this CTA's receive barrier; the matching wait comes
+  // just before the first remote store, long after every peer has arrived
+  if constexpr (PUSH) cluster_arrive_relaxed();
   const uint32_t tmem = *tmem_slot;
+  if (tr && threadIdx.x == 0) tr[1] = global_ns();
 
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&mapA);
@@ -104,7 +140,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     const int first = nkb < C::STAGES ? nkb : C::STAGES;
     for (int i = 0; i < first; ++i) {
       mbar_arrive_expect_tx(&full[i], TX);
-      tma_load_2d(sA + i * C::A_BYTES, &mapA, &full[i], (kb0 + i) * TC_BK, m0);
+      if constexpr (MC) {
+        if ((uint32_t)((kb0 + i) % (int)mc_size) == mc_rank)
+          tma_load_2d_mc(sA + i * C::A_BYTES, &mapA, &full[i], (kb0 + i) * TC_BK, m0, mc_mask);
+      } else {
+        tma_load_2d(sA + i * C::A_BYTES, &mapA, &full[i], (kb0 + i) * TC_BK, m0);
+      }
     }
     pdl_wait();
     if constexpr (!LNB)
@@ -116,7 +157,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       const uint32_t ph = (i / C::STAGES) & 1;
       if (!mbar_wait(&empty[s], ph ^ 1, status)) break;
       mbar_arrive_expect_tx(&full[s], TX);
-      tma_load_2d(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0);
+      if constexpr (MC) {
+        if ((uint32_t)((kb0 + i) % (int)mc_size) == mc_rank)
+          tma_load_2d_mc(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0, mc_mask);
+      } else {
+        tma_load_2d(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0);
+      }
       if constexpr (!LNB) tma_load_2d(sB + s * C::B_BYTES, &mapB, &full[s], (kb0 + i) * TC_BK, n0);
       issued = i + 1;
     }
@@ -129,6 +175,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       const int s = i % C::STAGES;
       const uint32_t ph = (i / C::STAGES) & 1;
       if (!mbar_wait(&full[s], ph, status)) break;
+      if (tr && i == 0) tr[2] = global_ns();
       tc_fence_after();
       const uint32_t a_addr = smem_u32(sA + s * C::A_BYTES);
       const uint32_t b_addr = smem_u32(sB + s * C::B_BYTES);
@@ -136,7 +183,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       for (int kk = 0; kk < TC_BK / 16; ++kk)
         umma_bf16(tmem, umma_desc_sw128(a_addr + kk * 32), umma_desc_sw128(b_addr + kk * 32), idesc,
                   (i | kk) != 0);
-      umma_commit(&empty[s]);
+      if constexpr (MC) umma_commit_mc(&empty[s], mc_mask);
+      else umma_commit(&empty[s]);
     }
     umma_commit(done);
   } else if (LNB && warp >= 2) {
@@ -146,30 +194,40 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     pdl_wait();
     pdl_launch();
     const int t = threadIdx.x - 64;
-    for (int r = warp - 2; r < BN; r += 2) {
-      const int n = n0 + r;
-      float mean = 0.f, rstd = 0.f;
-      if (n < n_valid) {
-        const float* xr = epi.ln_x + (size_t)n * K;
-        const float sh = __ldg(xr);
-        const float4* x4 = reinterpret_cast<const float4*>(xr);
-        float s1 = 0.f, s2 = 0.f;
-#pragma unroll 4
-        for (int i = lane; i < K / 4; i += 32) {
-          const float4 v = x4[i];
-          const float a = v.x - sh, b = v.y - sh, c = v.z - sh, e = v.w - sh;
-          s1 += (a + b) + (c + e);
-          s2 += (a * a + b * b) + (c * c + e * e);
-        }
-        s1 = warp_sum(s1);
-        s2 = warp_sum(s2);
-        const float m1 = s1 / (float)K;
-        mean = sh + m1;
-        rstd = rsqrtf(fmaxf(s2 / (float)K - m1 * m1, 0.f) + 1e-5f);
+    // four rows at a time per warp, all their loads in flight together
+    for (int rb = warp - 2; rb < BN; rb += 8) {
+      constexpr int RI = 4;
+      const float4* x4[RI];
+      float sh[RI], s1[RI], s2[RI];
+      bool ok[RI];
+#pragma unroll
+      for (int j = 0; j < RI; ++j) {
+        const int r = rb + 2 * j, n = n0 + r;
+        ok[j] = r < BN && n < n_valid;
+        const float* xr = epi.ln_x + (size_t)(ok[j] ? n : 0) * K;
+        x4[j] = reinterpret_cast<const float4*>(xr);
+        sh[j] = ok[j] ? __ldg(xr) : 0.f;
+        s1[j] = s2[j] = 0.f;
       }
-      if (lane == 0) {
-        ln_mean[r] = mean;
-        ln_rstd[r] = rstd;
+      for (int i = lane; i < K / 4; i += 32) {
+#pragma unroll
+        for (int j = 0; j < RI; ++j) {
+          if (!ok[j]) continue;
+          const float4 v = x4[j][i];
+          const float a = v.x - sh[j], b = v.y - sh[j], c = v.z - sh[j], e = v.w - sh[j];
+          s1[j] += (a + b) + (c + e);
+          s2[j] += (a * a + b * b) + (c * c + e * e);
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < RI; ++j) {
+        const int r = rb + 2 * j;
+        const float a1 = warp_sum(s1[j]), a2 = warp_sum(s2[j]);
+        const float m1 = a1 / (float)K;
+        if (lane == 0 && r < BN) {
+          ln_mean[r] = ok[j] ? sh[j] + m1 : 0.f;
+          ln_rstd[r] = ok[j] ? rsqrtf(fmaxf(a2 / (float)K - m1 * m1, 0.f) + 1e-5f) : 0.f;
+        }
       }
     }
     writers_sync();
@@ -214,6 +272,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   }
   __syncwarp();
   mbar_wait(done, 0, status);
+  if (tr && threadIdx.x == 0) tr[3] = global_ns();
+  __syncwarp();   // the warp leaves the wait together: the TMEM loads below are warp-aligned
   tc_fence_after();
 
   const int m = m0 + warp * 32 + lane;
@@ -254,6 +314,65 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
         if (n < n_valid) atomicMax(epi.row_key + n, k);
       }
     }
+  } else if constexpr (PUSH) {
+    cluster_wait();   // every peer's receive barrier is initialised
+    const int rows_per = TC_BM / splits;
+    const int ml = warp * 32 + lane;
+    const uint32_t owner = (uint32_t)(ml / rows_per);
+    // this split's copy of row ml sits at the same offset in the owner's buffer
+    float* slot = recv + (split * rows_per + ml % rows_per) * C::RECV_LD;
+    const bool mine = owner == (uint32_t)split;
+    const uint32_t dst = dsmem_addr(slot, owner);
+    const uint32_t bar = dsmem_addr(recv_bar, owner);
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(t_lane + c0, v);   // whole warp (tcgen05.ld is warp-aligned); only the stores branch
+#pragma unroll
+      for (int i = 0; i < 16; i += 4) {
+        const float4 q = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+        if (mine) *reinterpret_cast<float4*>(slot + c0 + i) = q;
+        else st_async_f4(dst + (uint32_t)(c0 + i) * 4u, q, bar);
+      }
+    }
+    if (tr && threadIdx.x == 0) tr[5] = global_ns();
+    __syncthreads();                    // own slice written by this CTA's threads
+    mbar_wait(recv_bar, 0, status);     // the peers' slices
+    if (tr && threadIdx.x == 0) tr[6] = global_ns();
+    // sum rows [split * rows_per, (split + 1) * rows_per) over the splits, in split order
+    const int r_first = split * rows_per;
+    const int items = rows_per * (BN / 4);
+    constexpr int IU = 4;
+    for (int base = threadIdx.x; base < items; base += IU * blockDim.x) {
+      int mm[4 * IU], nn[4 * IU];
+      bool ok[4 * IU];
+      float vals[4 * IU];
+#pragma unroll
+      for (int u = 0; u < IU; ++u) {
+        const int it = base + u * blockDim.x;
+        const int r = it % rows_per, c4 = it / rows_per;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (it < items) {
+          const float* src = recv + r * C::RECV_LD + 4 * c4;
+          for (int s2 = 0; s2 < splits; ++s2) {
+            const float4 p = *reinterpret_cast<const float4*>(src + s2 * rows_per * C::RECV_LD);
+            acc.x += p.x; acc.y += p.y; acc.z += p.z; acc.w += p.w;
+          }
+        }
+        vals[4 * u + 0] = acc.x;
+        vals[4 * u + 1] = acc.y;
+        vals[4 * u + 2] = acc.z;
+        vals[4 * u + 3] = acc.w;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          mm[4 * u + i] = m0 + r_first + r;
+          nn[4 * u + i] = n0 + 4 * c4 + i;
+          ok[4 * u + i] = it < items && m0 + r_first + r < epi.M && n0 + 4 * c4 + i < n_valid;
+        }
+      }
+      epi_batch<MODE == EPI_ARGMAX ? EPI_F32 : MODE, 4 * IU>(epi, mm, nn, vals, ok);
+    }
+    if (tr && threadIdx.x == 0) tr[7] = global_ns();
   } else if constexpr (CLU) {
     // stage this split's tile in shared memory (the pipeline buffers are free now)
     constexpr int LD = BN + 4;
@@ -267,7 +386,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       for (int i = 0; i < 16; i += 4)
         *reinterpret_cast<float4*>(red + ml * LD + c0 + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
     }
+    if (tr && threadIdx.x == 0) tr[5] = global_ns();
     cluster_sync();
+    if (tr && threadIdx.x == 0) tr[6] = global_ns();
     // this CTA sums rows [rank * 128 / splits, (rank + 1) * 128 / splits) over all splits
     const int rows_per = TC_BM / splits;
     const int r_first = split * rows_per;
@@ -310,6 +431,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       }
       epi_batch<MODE == EPI_ARGMAX ? EPI_F32 : MODE, 4 * IU>(epi, mm, nn, vals, ok);
     }
+    if (tr && threadIdx.x == 0) tr[7] = global_ns();
     cluster_sync();   // no CTA leaves while another may still read its shared memory
   } else {
     const int tile = tile_n * gridDim.x + tile_m;
@@ -384,6 +506,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     }
   }
 
+  if (tr && threadIdx.x == 0) tr[4] = global_ns();
+  // a multicast cluster stays until every CTA's commits (which arrive in all
+  // CTAs) have landed
+  if constexpr (MC) cluster_sync();
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
@@ -468,16 +594,29 @@ constexpr bool ln_capable() {
   return BN <= 64 && (MODE == EPI_QKV || MODE == EPI_Q || MODE == EPI_GELU || MODE == EPI_ARGMAX || MODE == EPI_F32);
 }
 
+template <int BN>
+constexpr bool mc_capable() {
+  return BN == 64 || BN == 128;
+}
+
 template <int BN, int MODE, bool LNB>
 static void launch_tc_ln(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
   const int mt = (g.M + TC_BM - 1) / TC_BM, nt = (g.N + BN - 1) / BN;
   if (g.cluster && g.splits > 1) {
-    launch_ex(gemm_tc_kernel<BN, MODE, true, LNB>, dim3(mt * g.splits, nt, 1), dim3(128), TcCfg<BN>::SMEM, st,
-              g.pdl, g.splits, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
+    launch_ex(gemm_tc_kernel<BN, MODE, true, LNB, false>, dim3(mt * g.splits, nt, 1), dim3(128),
+              TcCfg<BN, (BN <= 64)>::SMEM, st, g.pdl, g.splits, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi,
+              status);
     return;
   }
-  launch_ex(gemm_tc_kernel<BN, MODE, false, LNB>, dim3(mt, nt, g.splits), dim3(128), TcCfg<BN>::SMEM, st, g.pdl, 1,
-            g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
+  if constexpr (!LNB && mc_capable<BN>()) {
+    if (g.mc && g.splits == 1 && nt >= 2 && nt <= 8) {
+      launch_ex2(gemm_tc_kernel<BN, MODE, false, false, true>, dim3(mt, nt, 1), dim3(128), TcCfg<BN>::SMEM, st,
+                 g.pdl, 1, nt, g.mapA, g.mapB, g.K, 1, g.ws, g.tickets, epi, status);
+      return;
+    }
+  }
+  launch_ex(gemm_tc_kernel<BN, MODE, false, LNB, false>, dim3(mt, nt, g.splits), dim3(128), TcCfg<BN>::SMEM, st,
+            g.pdl, 1, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
 }
 
 template <int BN, int MODE>
@@ -506,11 +645,14 @@ static void launch_tc_mode(const TcGemm& g, const Epi& epi, int* status, cudaStr
 
 template <int BN, int MODE, bool LNB>
 static void configure_ln() {
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, LNB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, LNB, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        TcCfg<BN>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, LNB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       TcCfg<BN>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, LNB>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, LNB, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       TcCfg<BN, (BN <= 64)>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, LNB, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if constexpr (!LNB && mc_capable<BN>())
+    cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         TcCfg<BN>::SMEM);
 }
 
 template <int BN, int MODE>
