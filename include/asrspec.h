@@ -186,6 +186,33 @@ int asr_spec_set_graphs(asr_spec_handle h, int enable);
 int asr_spec_profile(asr_spec_handle h, int enable);
 int asr_spec_profile_read(asr_spec_handle h, double* ms, int64_t* launches, uint64_t* traffic);
 
+/* ---- Launch timeline (diagnostics; no counterpart in the paper) ----------
+ * asr_spec_timeline: when enabled, verify launches its kernels directly (no
+ * graph) and each launch of the verify chain records, from the GPU's global
+ * timer (ns), when its first CTA started, when its first CTA was past its
+ * wait on the previous kernel (programmatic dependent launch; the kernel's
+ * own prefetch of constant operands comes before that point), when its last
+ * CTA reached the kernel's midpoint (GEMM: its tensor-core MMAs done;
+ * attention: its key loop done; others: not recorded), and when its last CTA
+ * ended.  Enabling or disabling clears the record.  Each launch
+ * costs three atomics per CTA; up to ASR_TL_CAP launches are recorded.
+ * asr_spec_timeline_read: synchronise, then write up to `cap` launches in
+ * launch order: ns[4 * i + 0..3] = (start, past the wait, midpoint, end), 0
+ * where nothing was recorded, kind[i] as below; *count = the
+ * launches recorded since the last read; then clear.  Host pointers. */
+#define ASR_TL_CAP 8192
+#define ASR_TL_OTHER 0
+#define ASR_TL_PLAN 1          /* row plan of a verify step */
+#define ASR_TL_EMBED 2         /* token + position embedding */
+#define ASR_TL_LAYERNORM 3     /* stand-alone LayerNorm */
+#define ASR_TL_ATTN_SELF 4     /* self-attention */
+#define ASR_TL_ATTN_CROSS 5    /* cross-attention */
+#define ASR_TL_ACCEPT 6        /* acceptance, commit and anchor readout */
+#define ASR_TL_GEMM 16         /* + epilogue: 0 plain, 1 QKV + cache append, 2 residual, 3 query, 4 GELU, 6 argmax */
+#define ASR_TL_LN_FUSED 32     /* added to a GEMM kind whose B operand is LayerNorm(x), normalised in the GEMM */
+int asr_spec_timeline(asr_spec_handle h, int32_t enable);
+int asr_spec_timeline_read(asr_spec_handle h, uint64_t* ns, int32_t* kind, int32_t cap, int32_t* count);
+
 /* ---- Workload utility (not part of the paper's method) -------------------
  * Synthetic draft source used by benchmarks in place of a trained draft
  * model: draft i (1-based) of a round at committed length P is

@@ -27,9 +27,21 @@ EXPORTED = [
     "asr_spec_verify", "asr_spec_rollback", "asr_spec_state", "asr_spec_debug_logits",
     "asr_spec_status", "asr_spec_last_error", "asr_spec_destroy", "asr_spec_synth_drafts",
     "asr_spec_test_gemm", "asr_spec_set_graphs", "asr_spec_profile", "asr_spec_profile_read",
-    "asr_spec_gemm_noalloc",
+    "asr_spec_gemm_noalloc", "asr_spec_timeline", "asr_spec_timeline_read",
 ]
 PROF_CLASSES = ["proj_gemm", "self_attn", "cross_attn", "lm_head", "other"]
+TL_CAP = 8192
+TL_GEMM, TL_LN_FUSED = 16, 32
+TL_KINDS = {0: "other", 1: "plan", 2: "embed", 3: "layernorm", 4: "attn_self", 5: "attn_cross", 6: "accept_anchor"}
+TL_GEMM_EPILOGUES = {0: "plain", 1: "qkv", 2: "residual", 3: "query", 4: "gelu", 5: "cross_kv", 6: "argmax"}
+
+
+def tl_kind_name(kind: int) -> str:
+    """Readable name of a timeline launch kind (ASR_TL_* codes)."""
+    if kind >= TL_GEMM:
+        name = "gemm_" + TL_GEMM_EPILOGUES.get((kind - TL_GEMM) % TL_GEMM, str(kind))
+        return name + ("+ln" if kind & TL_LN_FUSED else "")
+    return TL_KINDS.get(kind, str(kind))
 
 
 class AsrModelDims(ctypes.Structure):
@@ -78,6 +90,8 @@ def lib():
     L.asr_spec_profile.argtypes = [vp, ctypes.c_int]
     L.asr_spec_profile_read.argtypes = [vp, vp, vp, vp]
     L.asr_spec_gemm_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
+    L.asr_spec_timeline.argtypes = [vp, i32]
+    L.asr_spec_timeline_read.argtypes = [vp, vp, vp, i32, vp]
     for name in EXPORTED:
         if name not in ("asr_spec_last_error", "asr_spec_destroy"):
             getattr(L, name).restype = ctypes.c_int
@@ -184,6 +198,21 @@ def asr_spec_profile_read(h):
     _check(h, lib().asr_spec_profile_read(h, ms.ctypes.data, launches.ctypes.data, traffic.ctypes.data),
            "asr_spec_profile_read")
     return ms, launches, traffic
+
+
+def asr_spec_timeline(h, enable: bool):
+    return _check(h, lib().asr_spec_timeline(h, 1 if enable else 0), "asr_spec_timeline")
+
+
+def asr_spec_timeline_read(h):
+    """Returns (ns [n][4] = start, past the wait, midpoint, end; kinds [n]) of the recorded launches."""
+    ns = np.zeros((TL_CAP, 4), dtype=np.uint64)
+    kinds = np.zeros(TL_CAP, dtype=np.int32)
+    count = ctypes.c_int32(0)
+    _check(h, lib().asr_spec_timeline_read(h, ns.ctypes.data, kinds.ctypes.data, TL_CAP, ctypes.byref(count)),
+           "asr_spec_timeline_read")
+    n = min(count.value, TL_CAP)
+    return ns[:n].copy(), kinds[:n].copy()
 
 
 def asr_spec_gemm_noalloc(A, B, C, M, N, K, splits, stream=None):

@@ -75,10 +75,20 @@ struct asr_spec {
   // CUDA graphs of the verify body, keyed by (B, k)
   bool use_graphs = true;
   bool use_pdl = true;   // programmatic dependent launch between verify kernels
-  bool lm_ln_fused = false;
-  bool use_mc = false;        // multicast weight tiles across the row tiles (ASRSPEC_MC=1; slower as measured)   // the last verify's LM head normalised x itself (xf not written)
+  bool lm_ln_fused = false;   // the last verify's LM head normalised x itself (xf not written)
+  bool use_mc = false;        // multicast weight tiles across the row tiles (ASRSPEC_MC=1; slower as measured)
+  // GEMMs over at most this many rows normalise their own B operand
+  // (ASRSPEC_LN_FUSE_MAX, <= 64); off by default: a separate LayerNorm launch
+  // measured faster at batch 1 (1.99 vs 2.48 ms per large-decoder round)
+  int ln_fuse_max = 0;
   int wide_bn = 64;      // N tile for many rows (ASRSPEC_WIDE_BN: 64, 128, 192, 224, 256)
   int wide_target = 2 * 152;   // CTAs a many-row GEMM may fill by splitting K (ASRSPEC_WIDE_TARGET)
+  // launch timeline (diagnostics): [ASR_TL_CAP][4] device slots, the kind of
+  // each recorded launch, and the slot of the launch being enqueued
+  bool tl_on = false;
+  unsigned long long* tl_buf = nullptr;
+  std::vector<int> tl_kind;
+  unsigned long long* tl_cur = nullptr;
   struct Graph {
     cudaGraphExec_t exec;
     long long launches[ASR_PROF_N];
@@ -128,6 +138,19 @@ struct Prof {
       h->marks.emplace_back(cls, idx);
     }
   }
+};
+
+// Gives the next launch a timeline slot (h->tl_cur) when the timeline is on.
+struct Tl {
+  asr_spec* h;
+  Tl(asr_spec* h_, int kind) : h(h_) {
+    h->tl_cur = nullptr;
+    if (h->tl_on && !h->capturing && h->tl_buf && (int)h->tl_kind.size() < ASR_TL_CAP) {
+      h->tl_cur = h->tl_buf + 4 * h->tl_kind.size();
+      h->tl_kind.push_back(kind);
+    }
+  }
+  ~Tl() { h->tl_cur = nullptr; }
 };
 
 #define CK(call)                                                                       \
@@ -219,6 +242,8 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   g.pdl = h->use_pdl;
   g.ws = h->ws;
   g.tickets = h->tickets;
+  Tl t(h, ASR_TL_GEMM + mode + (epi.ln_x ? ASR_TL_LN_FUSED : 0));
+  epi.tl = h->tl_cur;
   launch_gemm_tc(g, mode, epi, h->status, h->st);
   return 0;
 }
@@ -231,7 +256,7 @@ enum BufId { BUF_XN = 1, BUF_ATT = 2, BUF_H = 3, BUF_XF = 4 };
 int gemm_rows_ln(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, const float* g, const float* b,
                  void* ln_out, int ln_out_id, int N, int mode, const Epi& epi_in, bool* fused = nullptr) {
   Epi e = epi_in;
-  const bool fuse = h->bf16 && N <= 64;
+  const bool fuse = h->bf16 && N <= std::min(h->ln_fuse_max, 64);
   if (fused) *fused = fuse;
   if (fuse) {
     e.ln_x = h->x;
@@ -241,7 +266,8 @@ int gemm_rows_ln(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K
   }
   {
     Prof p(h, ASR_PROF_OTHER, 1);
-    launch_layernorm(h->x, g, b, ln_out, h->bf16, h->plan.n_rows, N, K, h->st, h->use_pdl);
+    Tl t(h, ASR_TL_LAYERNORM);
+    launch_layernorm(h->x, g, b, ln_out, h->bf16, h->plan.n_rows, N, K, h->st, h->use_pdl, h->tl_cur);
   }
   return gemm_rows(h, W, mW, M, K, ln_out, ln_out_id, N, mode, e);
 }
@@ -275,7 +301,10 @@ void attention(asr_spec* h, AttnArgs& a, bool self_attn, int layer) {
   }
   a.tickets = h->attn_tickets;
   a.pdl = h->use_pdl;
+  Tl t(h, self_attn ? ASR_TL_ATTN_SELF : ASR_TL_ATTN_CROSS);
+  a.tl = h->tl_cur;
   launch_attention_tc(a, h->status, h->st);
+  a.tl = nullptr;
 }
 
 int run_layers(asr_spec* h, int N) {
@@ -294,7 +323,8 @@ int run_layers(asr_spec* h, int N) {
   const size_t cross_half = (size_t)h->Bmax * h->H * h->Tmax * 64 * h->es;
   {
     Prof p(h, ASR_PROF_OTHER, 1);
-    launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st, h->use_pdl);
+    Tl t(h, ASR_TL_EMBED);
+    launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st, h->use_pdl, h->tl_cur);
   }
   for (int l = 0; l < h->L; ++l) {
     LayerW& w = h->lw[l];
@@ -396,9 +426,10 @@ int enqueue_verify(asr_spec* h, int k) {
   const int B = h->B;
   {
     Prof p(h, ASR_PROF_OTHER, 1);
+    Tl t(h, ASR_TL_PLAN);
     TrafficArgs tr{h->counters, h->enc_len, h->L, h->d, (int)h->es};
     launch_plan_verify(h->draft_buf, h->lens_buf, k, B, h->V, h->maxpos, h->kv_len, h->pending, h->ready, h->plan,
-                       h->row_key, h->status, tr, h->st);
+                       h->row_key, h->status, tr, h->st, h->tl_cur);
   }
   const int N = B * (k + 1);
   if (int rc = run_layers(h, N)) return rc;
@@ -433,7 +464,10 @@ int enqueue_verify(asr_spec* h, int k) {
   A.enc_len = h->enc_len;
   A.frame_key = h->frame_key;
   A.tickets = reinterpret_cast<int*>(h->frame_key + h->Bmax);
+  A.status = h->status;
   A.pdl = h->use_pdl;
+  Tl t(h, ASR_TL_ACCEPT);
+  A.tl = h->tl_cur;
   launch_accept_anchor(A, h->st);
   return 0;
 }
@@ -461,6 +495,7 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   h->bf16 = dims->dtype == 1;
   if (const char* e = std::getenv("ASRSPEC_PDL")) h->use_pdl = std::atoi(e) != 0;
   if (const char* e = std::getenv("ASRSPEC_MC")) h->use_mc = std::atoi(e) != 0;
+  if (const char* e = std::getenv("ASRSPEC_LN_FUSE_MAX")) h->ln_fuse_max = std::atoi(e);
   if (const char* e = std::getenv("ASRSPEC_WIDE_BN")) {
     const int v = std::atoi(e);
     if (v == 64 || v == 128 || v == 192 || v == 224 || v == 256) h->wide_bn = v;
@@ -744,7 +779,7 @@ int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens
   }
   if (int rc = copy_in(h, h->lens_buf, lens, B)) return rc;
   for (int c = 0; c < ASR_PROF_N; ++c) h->cur[c] = 0;
-  if (h->use_graphs && !h->prof) {
+  if (h->use_graphs && !h->prof && !h->tl_on) {
     auto key = std::make_pair(B, (int)k);
     auto it = h->graphs.find(key);
     if (it == h->graphs.end()) {
@@ -812,6 +847,41 @@ int asr_spec_profile_read(asr_spec_handle h, double* ms, int64_t* launches, uint
   h->ev_used = 0;
   for (int c = 0; c < ASR_PROF_N; ++c) h->launches[c] = 0;
   CK(cudaMemset(h->counters, 0, 8 * sizeof(unsigned long long)));
+  return ASR_OK;
+}
+
+int asr_spec_timeline(asr_spec_handle h, int32_t enable) {
+  if (!h) return ASR_E_INVAL;
+  const size_t bytes = (size_t)ASR_TL_CAP * 4 * sizeof(unsigned long long);
+  if (enable && !h->tl_buf) {
+    if (int rc = dalloc(h, &h->tl_buf, bytes)) return rc;
+  }
+  if (h->tl_buf) CK(cudaMemsetAsync(h->tl_buf, 0, bytes, h->st));
+  h->tl_kind.clear();
+  h->tl_on = enable != 0;
+  return ASR_OK;
+}
+
+int asr_spec_timeline_read(asr_spec_handle h, uint64_t* ns, int32_t* kind, int32_t cap, int32_t* count) {
+  if (!h || cap < 0 || !count || (cap > 0 && (!ns || !kind))) return ASR_E_INVAL;
+  CK(cudaStreamSynchronize(h->st));
+  const int n = (int)h->tl_kind.size();
+  *count = n;
+  const int m = std::min(n, (int)cap);
+  if (m > 0) {
+    std::vector<unsigned long long> raw((size_t)m * 4);
+    CK(cudaMemcpy(raw.data(), h->tl_buf, raw.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
+    for (int i = 0; i < m; ++i) {
+      const unsigned long long* s = &raw[(size_t)i * 4];
+      ns[4 * i + 0] = s[0] ? ~s[0] : 0;   // entries were recorded complemented (max of ~t = min of t)
+      ns[4 * i + 1] = s[1] ? ~s[1] : 0;
+      ns[4 * i + 2] = s[3];
+      ns[4 * i + 3] = s[2];
+      kind[i] = h->tl_kind[i];
+    }
+  }
+  if (h->tl_buf) CK(cudaMemsetAsync(h->tl_buf, 0, (size_t)ASR_TL_CAP * 4 * sizeof(unsigned long long), h->st));
+  h->tl_kind.clear();
   return ASR_OK;
 }
 

@@ -187,106 +187,155 @@ int attn_chunk_len(int kv_bf16) { return kv_bf16 ? 256 : 128; }
 // ---------------------------------------------------------------------------
 // Acceptance, commit and anchor readout, fused
 // ---------------------------------------------------------------------------
-// One CTA per (32 encoder frames, utterance).  Every CTA of an utterance
-// recomputes the accepted length n from the per-row argmax keys (a few loads);
-// the first one commits: accepted, bonus, kv_len += 1 + n, pending = bonus
-// (Sec. 3 "Speculative Loop"; a round advances 1 + L tokens, App. "Correction
-// and Cost").  Then each CTA evaluates, for its frames, the head mean of the
-// per-head softmax attention of row n at the anchor layer (Sec. 5
+// One CTA per (FB encoder frames, utterance).  The anchor layer's encoder keys
+// do not change during a verify call, so each CTA starts copying its frames'
+// keys (all heads) into shared memory before it waits for the LM head.  Then
+// one warp recomputes the accepted length n from the per-row argmax keys (one
+// ballot); the first CTA commits: accepted, bonus, kv_len += 1 + n, pending =
+// bonus (Sec. 3 "Speculative Loop"; a round advances 1 + L tokens, App.
+// "Correction and Cost").  Each CTA then evaluates, for its frames, the head
+// mean of the per-head softmax attention of row n at the anchor layer (Sec. 5
 // "Verification-Attention Correction"), with the (max, sum) the attention pass
-// left; a fixed-order head sum per frame, an order-free atomicMax of packed
-// (value, frame) keys, and the last CTA (ticket) writes the peak frame.
-constexpr int ANCHOR_FRAMES = 32;
+// left: a fixed-order head sum per frame, an order-free atomicMax of packed
+// (value, frame) keys, and the last CTA of the utterance (ticket) writes the
+// peak frame.  Only CTAs that hold frames (and the first) take part.
+constexpr int ANCHOR_HMAX = 32;   // heads (d_model <= 2048)
+
+template <typename T>
+struct AnchorCfg {
+  static constexpr int FB = sizeof(T) == 2 ? 32 : 16;   // frames per CTA
+  static constexpr int ROW_BYTES = 64 * (int)sizeof(T);
+  static constexpr int SMEM = ANCHOR_HMAX * FB * ROW_BYTES;   // keys [H][FB][64]; <= 128 KB
+};
 
 template <typename T>
 __global__ void __launch_bounds__(256)
 accept_anchor_kernel(AcceptAnchorArgs A) {
-  __shared__ float qs[32][64];
-  __shared__ float ph[32][ANCHOR_FRAMES + 1];
+  using C = AnchorCfg<T>;
+  constexpr int FB = C::FB;
+  extern __shared__ __align__(128) uint8_t anchor_keys[];
+  __shared__ float qs[ANCHOR_HMAX][64];
+  __shared__ float ph[ANCHOR_HMAX][FB + 1];
+  __shared__ float sM[ANCHOR_HMAX], sL[ANCHOR_HMAX];
+  __shared__ __align__(8) uint64_t bar;
   __shared__ int s_n, s_last;
+  tl_mark(A.tl, TL_ENTRY);
+  const int b = blockIdx.y, f0 = blockIdx.x * FB, tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
+  const int H = A.H;
+  const int n_frames = A.enc_len[b];                  // constant during a verify call
+  if (blockIdx.x > 0 && f0 >= n_frames) {             // no frames here
+    pdl_wait();
+    return;
+  }
+  const int rows = min(FB, n_frames - f0) > 0 ? min(FB, n_frames - f0) : 0;
+  if (tid == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    if (rows > 0) {
+      mbar_arrive_expect_tx(&bar, (uint32_t)(H * rows * C::ROW_BYTES));
+      const char* kc = static_cast<const char*>(A.kc);
+      for (int h = 0; h < H; ++h)
+        bulk_load(anchor_keys + h * FB * C::ROW_BYTES,
+                  kc + (((size_t)b * H + h) * A.t_alloc + f0) * C::ROW_BYTES, (uint32_t)(rows * C::ROW_BYTES), &bar);
+    }
+  }
   pdl_wait();
+  tl_mark(A.tl, TL_WORK);
   pdl_launch();
-  const int b = blockIdx.y, f0 = blockIdx.x * ANCHOR_FRAMES, tid = threadIdx.x;
   const int nr = A.plan.n_utt_rows[b];
-  if (nr == 0) {
+  if (nr == 0) {                                      // uniform over the utterance's CTAs
     if (blockIdx.x == 0 && tid == 0) {
       A.accepted[b] = 0;
       A.bonus[b] = -1;
       A.kv_len_out[b] = A.kv_len[b];
       A.anchor_out[b] = -1;
     }
+    __syncthreads();
+    if (rows > 0) mbar_wait(&bar, 0, A.status);       // no CTA leaves with copies in flight
     return;
   }
   const int r0 = A.plan.row_start[b];
-  if (tid == 0) {
+  if (warp == 0) {
+    // draft i is accepted while it equals the target's argmax at row i (i < nr - 1)
     const int l = nr - 1;
-    int n = 0;
-    while (n < l && A.draft[(size_t)b * A.k + n] == (int)argmax_index(A.row_key[r0 + n])) ++n;
-    s_n = n;
-    if (blockIdx.x == 0) {
-      const int g = (int)argmax_index(A.row_key[r0 + n]);
-      const int nl = A.kv_len[b] + 1 + n;
-      A.accepted[b] = n;
-      A.bonus[b] = g;
-      A.kv_len[b] = nl;
-      A.kv_len_out[b] = nl;
-      A.pending[b] = g;
+    const unsigned long long key = lane < nr ? A.row_key[r0 + lane] : 0ull;
+    const int tok = (int)argmax_index(key);
+    const bool match = lane < l && A.draft[(size_t)b * A.k + lane] == tok;
+    const unsigned mism = ~__ballot_sync(0xffffffffu, match);
+    const int n = min(__ffs(mism) - 1, l);
+    const int g = __shfl_sync(0xffffffffu, tok, n);
+    if (lane == 0) {
+      s_n = n;
+      if (blockIdx.x == 0) {
+        const int nl = A.kv_len[b] + 1 + n;
+        A.accepted[b] = n;
+        A.bonus[b] = g;
+        A.kv_len[b] = nl;
+        A.kv_len_out[b] = nl;
+        A.pending[b] = g;
+      }
     }
   }
   __syncthreads();
   const int r = r0 + s_n;
-  const int H = A.H;
   for (int e = tid; e < H * 64; e += blockDim.x) {
     const float v = A.q_anchor[(size_t)r * A.d + e];
     // the tensor-core attention scored bf16(q / 8) against the bf16 keys
     qs[e >> 6][e & 63] = A.kv_bf16 ? bf2f(f2bf(v * 0.125f)) : v;
   }
+  if (tid < H) {
+    sM[tid] = A.ml[((size_t)r * H + tid) * 2 + 0];
+    sL[tid] = A.ml[((size_t)r * H + tid) * 2 + 1];
+  }
   __syncthreads();
-  const int n_frames = A.enc_len[b];
-  const int warp = tid >> 5, lane = tid & 31;
-  const int f = f0 + lane;
-  for (int h = warp; h < H; h += 8) {
-    float p = 0.f;
-    if (f < n_frames) {
-      const T* krow = static_cast<const T*>(A.kc) + (((size_t)b * H + h) * A.t_alloc + f) * 64;
-      float s;
-      if (A.kv_bf16) {
-        // the key row as eight 16-byte loads, all in flight before the sum
-        const uint4* k16 = reinterpret_cast<const uint4*>(krow);
-        uint4 kv[8];
+  if (rows > 0) mbar_wait(&bar, 0, A.status);
+  // scores: 8 lanes per (head, frame), each over 8 of the 64 dimensions, so
+  // that a warp reads four consecutive key rows of shared memory at once
+  const int g = lane >> 3, c = lane & 7;
+  const float scale = A.kv_bf16 ? 1.f : ATTN_SCALE;
+  for (int base = warp * 4; base < H * FB; base += 32) {   // uniform over the warp
+    const int p = base + g;
+    const int h = p / FB, fr = p - h * FB;
+    const bool ok = p < H * FB && fr < rows;
+    float s = 0.f;
+    if (ok) {
+      const uint8_t* kr = anchor_keys + (h * FB + fr) * C::ROW_BYTES;
+      const float* qh = qs[h] + 8 * c;
+      if constexpr (sizeof(T) == 2) {
+        const uint4 kv = *reinterpret_cast<const uint4*>(kr + 16 * c);
+        const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
 #pragma unroll
-        for (int u = 0; u < 8; ++u) kv[u] = __ldg(k16 + u);
-        s = 0.f;
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&kv[u]);
-#pragma unroll
-          for (int w = 0; w < 4; ++w) {
-            const float2 kf = __bfloat1622float2(p2[w]);
-            s = fmaf(qs[h][8 * u + 2 * w], kf.x, s);
-            s = fmaf(qs[h][8 * u + 2 * w + 1], kf.y, s);
-          }
+        for (int w = 0; w < 4; ++w) {
+          const float2 kf = __bfloat1622float2(k2[w]);
+          s = fmaf(qh[2 * w], kf.x, s);
+          s = fmaf(qh[2 * w + 1], kf.y, s);
         }
       } else {
-        s = dot64_rot<T>(qs[h], krow, f) * ATTN_SCALE;
+        const float4 k0 = *reinterpret_cast<const float4*>(kr + 32 * c);
+        const float4 k1 = *reinterpret_cast<const float4*>(kr + 32 * c + 16);
+        s = fmaf(qh[0], k0.x, s); s = fmaf(qh[1], k0.y, s); s = fmaf(qh[2], k0.z, s); s = fmaf(qh[3], k0.w, s);
+        s = fmaf(qh[4], k1.x, s); s = fmaf(qh[5], k1.y, s); s = fmaf(qh[6], k1.z, s); s = fmaf(qh[7], k1.w, s);
       }
-      const float M = A.ml[((size_t)r * H + h) * 2 + 0];
-      const float L = A.ml[((size_t)r * H + h) * 2 + 1];
-      p = expf(s - M) / L;
     }
-    ph[h][lane] = p;
+    s += __shfl_xor_sync(0xffffffffu, s, 1);
+    s += __shfl_xor_sync(0xffffffffu, s, 2);
+    s += __shfl_xor_sync(0xffffffffu, s, 4);
+    if (c == 0 && p < H * FB) ph[h][fr] = ok ? expf(s * scale - sM[h]) / sL[h] : 0.f;
   }
   __syncthreads();
   if (warp == 0) {
     float pbar = 0.f;
-    for (int h = 0; h < H; ++h) pbar += ph[h][lane];
+    const int fr = lane < FB ? lane : 0;
+    for (int h = 0; h < H; ++h) pbar += ph[h][fr];
     pbar /= (float)H;
-    unsigned long long key = f < n_frames ? argmax_key(pbar, (uint32_t)f) : 0ull;
+    unsigned long long key = lane < rows ? argmax_key(pbar, (uint32_t)(f0 + lane)) : 0ull;
     key = warp_max_u64(key);
     if (lane == 0) {
+      const int n_cta = n_frames > FB ? (n_frames + FB - 1) / FB : 1;   // CTAs of this utterance that take part
       atomicMax(A.frame_key + b, key);
       __threadfence();
-      s_last = (atomicAdd(A.tickets + b, 1) == (int)gridDim.x - 1);
+      s_last = (atomicAdd(A.tickets + b, 1) == n_cta - 1);
       if (s_last) {
         __threadfence();
         const unsigned long long fk = atomicExch(A.frame_key + b, 0ull);
@@ -295,12 +344,27 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
       }
     }
   }
+  tl_mark(A.tl, TL_EXIT);
 }
 
 void launch_accept_anchor(const AcceptAnchorArgs& A, cudaStream_t st) {
-  dim3 grid((A.t_alloc + ANCHOR_FRAMES - 1) / ANCHOR_FRAMES, A.B);
-  if (A.kv_bf16) launch_ex(accept_anchor_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, A.pdl, 1, A);
-  else launch_ex(accept_anchor_kernel<float>, grid, dim3(256), 0, st, A.pdl, 1, A);
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaFuncSetAttribute(accept_anchor_kernel<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         AnchorCfg<__nv_bfloat16>::SMEM);
+    cudaFuncSetAttribute(accept_anchor_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         AnchorCfg<float>::SMEM);
+  });
+  if (A.kv_bf16) {
+    using C = AnchorCfg<__nv_bfloat16>;
+    dim3 grid((A.t_alloc + C::FB - 1) / C::FB, A.B);
+    launch_ex(accept_anchor_kernel<__nv_bfloat16>, grid, dim3(256), (size_t)A.H * C::FB * C::ROW_BYTES, st, A.pdl, 1,
+              A);
+  } else {
+    using C = AnchorCfg<float>;
+    dim3 grid((A.t_alloc + C::FB - 1) / C::FB, A.B);
+    launch_ex(accept_anchor_kernel<float>, grid, dim3(256), (size_t)A.H * C::FB * C::ROW_BYTES, st, A.pdl, 1, A);
+  }
 }
 
 }  // namespace asrspec

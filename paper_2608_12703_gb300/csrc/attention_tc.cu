@@ -82,6 +82,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
   __shared__ __align__(8) uint64_t bar[TCA_STAGES];
 
   const int S = gridDim.x, split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  tl_mark(a.tl, TL_ENTRY);
   const int nr = a.plan.n_utt_rows[b];
   if (nr == 0) {                             // uniform over the cluster
     pdl_wait();
@@ -114,6 +115,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
   if (tid == 0 && !a.causal)
     for (int i = 0; i < n_iter && i < TCA_STAGES; ++i) issue(i);
   pdl_wait();
+  tl_mark(a.tl, TL_WORK);
   if (tid == 0 && a.causal)
     for (int i = 0; i < n_iter && i < TCA_STAGES; ++i) issue(i);
   pdl_launch();
@@ -285,6 +287,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
   }
 
   // merge the splits of this (utterance, head) in split order
+  tl_mark(a.tl, TL_MID);
+  __syncwarp();
   if (S > 1) cluster_sync();
   else __syncthreads();
   for (int e = split * TCA_THREADS + tid; e < nr * 64; e += S * TCA_THREADS) {
@@ -308,6 +312,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
     }
   }
   if (S > 1) cluster_sync();   // no CTA leaves while another may still read its shared memory
+  tl_mark(a.tl, TL_EXIT);
 }
 
 template <int MT>

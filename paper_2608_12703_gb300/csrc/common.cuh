@@ -239,6 +239,20 @@ __device__ __forceinline__ unsigned long long global_ns() {
   return t;
 }
 
+// Launch timeline (diagnostics; a null slot records nothing).  One slot of
+// four words per launch, zeroed before the launch: [0] = max over CTAs of
+// ~(entry ns), [1] = max of ~(ns when the CTA is past its wait on the
+// previous kernel), [2] = max of exit ns, [3] = max of a kernel-specific
+// midpoint (GEMM: MMAs done; attention: key loop done); thread 0 of each CTA
+// records.
+enum TlMark : int { TL_ENTRY = 0, TL_WORK = 1, TL_EXIT = 2, TL_MID = 3 };
+__device__ __forceinline__ void tl_mark(unsigned long long* slot, int which) {
+  if (slot != nullptr && threadIdx.x == 0) {
+    const unsigned long long t = global_ns();
+    atomicMax(slot + which, which >= TL_EXIT ? t : ~t);
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Programmatic dependent launch.  Every kernel of the verify chain calls
 // pdl_wait() before it touches anything its predecessor writes, and only then

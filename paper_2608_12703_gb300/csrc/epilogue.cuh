@@ -52,6 +52,8 @@ struct Epi {
   const float* ln_x = nullptr;
   const float* ln_g = nullptr;
   const float* ln_b = nullptr;
+  // launch timeline slot (see tl_mark), or null
+  unsigned long long* tl = nullptr;
   // optional phase timestamps (ns, %globaltimer) per CTA: [CTA][8]
   // (entry, set-up done, first stage full, MMAs done, end; cluster split:
   // partials staged, first cluster barrier passed, reduction done)
@@ -109,70 +111,166 @@ __device__ __forceinline__ void epi_apply(const Epi& e, int m, int n, float acc)
   }
 }
 
-// U output elements at once.  The residual update loads every x value before
-// it stores any (the elements are distinct, so no store can feed a later
-// load), which keeps U loads in flight instead of U dependent round trips.
+// U output elements at once, in two halves so that a caller can issue the
+// loads early (before the accumulators are ready) and keep them in registers:
+// epi_load fetches what the outputs depend on besides the accumulators (bias,
+// residual, row metadata), epi_store combines and writes.  The elements are
+// distinct, so no store can feed a later load.
 template <int MODE, int U>
-__device__ __forceinline__ void epi_batch(const Epi& e, const int* m, const int* n, const float* v,
-                                          const bool* ok) {
-  if constexpr (MODE == EPI_RESID) {
-    float old[U], bias[U];
+struct EpiPre {
+  float bias[U];
+  float old[U];   // EPI_RESID: x before the update
+  int rb[U], rp[U];   // EPI_QKV: utterance and position of the row
+};
+
+template <int MODE, int U>
+__device__ __forceinline__ void epi_load(const Epi& e, const int* m, const int* n, const bool* ok,
+                                         EpiPre<MODE, U>& p) {
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      old[u] = ok[u] ? e.x[(size_t)n[u] * e.d + m[u]] : 0.f;
-      bias[u] = ok[u] ? e.bias[m[u]] : 0.f;
+  for (int u = 0; u < U; ++u) {
+    if constexpr (MODE == EPI_RESID || MODE == EPI_QKV || MODE == EPI_Q || MODE == EPI_GELU)
+      p.bias[u] = ok[u] ? __ldg(e.bias + m[u]) : 0.f;
+    if constexpr (MODE == EPI_RESID) p.old[u] = ok[u] ? e.x[(size_t)n[u] * e.d + m[u]] : 0.f;
+    if constexpr (MODE == EPI_QKV) {
+      p.rb[u] = ok[u] && m[u] >= e.d ? e.row_b[n[u]] : 0;
+      p.rp[u] = ok[u] && m[u] >= e.d ? e.row_pos[n[u]] : 0;
     }
+  }
+}
+
+template <int MODE, int U>
+__device__ __forceinline__ void epi_store(const Epi& e, const int* m, const int* n, const float* v, const bool* ok,
+                                          const EpiPre<MODE, U>& p) {
 #pragma unroll
-    for (int u = 0; u < U; ++u)
-      if (ok[u]) e.x[(size_t)n[u] * e.d + m[u]] = old[u] + (v[u] + bias[u]);
-  } else if constexpr (MODE == EPI_QKV) {
-    // row metadata and biases first, then the stores
-    float bias[U];
-    int rb[U], rp[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      bias[u] = ok[u] ? e.bias[m[u]] : 0.f;
-      rb[u] = ok[u] && m[u] >= e.d ? e.row_b[n[u]] : 0;
-      rp[u] = ok[u] && m[u] >= e.d ? e.row_pos[n[u]] : 0;
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (!ok[u]) continue;
-      const float val = v[u] + bias[u];
+  for (int u = 0; u < U; ++u) {
+    if (!ok[u]) continue;
+    if constexpr (MODE == EPI_RESID) {
+      e.x[(size_t)n[u] * e.d + m[u]] = p.old[u] + (v[u] + p.bias[u]);
+    } else if constexpr (MODE == EPI_QKV) {
+      const float val = v[u] + p.bias[u];
       if (m[u] < e.d) {
         e.out_f32[(size_t)n[u] * e.d + m[u]] = val;
       } else {
         const int which = (m[u] - e.d) / e.d;
         const int f = (m[u] - e.d) - which * e.d;
-        const size_t idx = (((size_t)rb[u] * e.n_heads + (f >> 6)) * e.max_pos + rp[u]) * 64 + (f & 63);
+        const size_t idx = (((size_t)p.rb[u] * e.n_heads + (f >> 6)) * e.max_pos + p.rp[u]) * 64 + (f & 63);
         void* base = which == 0 ? e.kcache : e.vcache;
         if (e.kv_bf16) store_as<__nv_bfloat16>(base, idx, val);
         else store_as<float>(base, idx, val);
       }
-    }
-  } else if constexpr (MODE == EPI_Q) {
-    float bias[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) bias[u] = ok[u] ? e.bias[m[u]] : 0.f;
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-      if (ok[u]) e.out_f32[(size_t)n[u] * e.d + m[u]] = v[u] + bias[u];
-  } else if constexpr (MODE == EPI_GELU) {
-    float bias[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) bias[u] = ok[u] ? e.bias[m[u]] : 0.f;
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (!ok[u]) continue;
-      const float g = gelu_erf(v[u] + bias[u]);
+    } else if constexpr (MODE == EPI_Q) {
+      e.out_f32[(size_t)n[u] * e.d + m[u]] = v[u] + p.bias[u];
+    } else if constexpr (MODE == EPI_GELU) {
+      const float g = gelu_erf(v[u] + p.bias[u]);
       const size_t idx = (size_t)n[u] * e.M + m[u];
       if (e.act_bf16) store_as<__nv_bfloat16>(e.act, idx, g);
       else store_as<float>(e.act, idx, g);
+    } else {
+      epi_apply<MODE>(e, m[u], n[u], v[u]);
     }
-  } else {
+  }
+}
+
+template <int MODE, int U>
+__device__ __forceinline__ void epi_batch(const Epi& e, const int* m, const int* n, const float* v,
+                                          const bool* ok) {
+  EpiPre<MODE, U> p;
+  epi_load<MODE, U>(e, m, n, ok, p);
+  epi_store<MODE, U>(e, m, n, v, ok, p);
+}
+
+// Row-wise epilogue over a tile staged in shared memory as stg[n_local][m_local]
+// (leading dimension lds): lane l of warp w covers features m = mq .. mq + 3
+// (mq = tile m0 + 4 l) of rows n_local = w, w + 4, ...  Each row is written
+// with one 16-byte (fp32) or 8-byte (bf16) store per lane, so a warp writes
+// whole 512- or 256-byte runs; bias and the feature's role are per lane, the
+// row metadata per row.  Modes: F32 (any M), Q, RESID, GELU, QKV (M, d, and
+// the leading dimensions multiples of 4).
+template <int MODE>
+__host__ __device__ constexpr bool rowwise_mode() {
+  return MODE == EPI_F32 || MODE == EPI_Q || MODE == EPI_RESID || MODE == EPI_GELU || MODE == EPI_QKV;
+}
+
+template <int MODE>
+__device__ __forceinline__ void epi_rows(const Epi& e, const float* stg, int lds, int mq, int m_local, int n0,
+                                         int warp, int rows) {
+  const bool mok = mq < e.M;
+  float4 bias = make_float4(0.f, 0.f, 0.f, 0.f);
+  if constexpr (MODE != EPI_F32)
+    if (mok) bias = __ldg(reinterpret_cast<const float4*>(e.bias + mq));
+  int kind = 0, head = 0, c = 0;   // EPI_QKV: 0 query, 1 key, 2 value
+  if constexpr (MODE == EPI_QKV) {
+    if (mq >= e.d) {
+      const int f = mq - e.d;
+      kind = f >= e.d ? 2 : 1;
+      const int g = f - (kind - 1) * e.d;
+      head = g >> 6;
+      c = g & 63;
+    }
+  }
+  constexpr int RB = 4;   // rows per batch, their loads in flight together
+  for (int j0 = warp; j0 < rows; j0 += 4 * RB) {
+    float4 a[RB], old[RB];
+    int rb[RB], rp[RB];
+    bool ok[RB];
 #pragma unroll
-    for (int u = 0; u < U; ++u)
-      if (ok[u]) epi_apply<MODE>(e, m[u], n[u], v[u]);
+    for (int r = 0; r < RB; ++r) {
+      const int nl = j0 + 4 * r;
+      ok[r] = nl < rows && mok;
+      const int n = n0 + (nl < rows ? nl : 0);
+      a[r] = ok[r] ? *reinterpret_cast<const float4*>(stg + nl * lds + m_local) : make_float4(0.f, 0.f, 0.f, 0.f);
+      if constexpr (MODE == EPI_RESID)
+        old[r] = ok[r] ? *reinterpret_cast<const float4*>(e.x + (size_t)n * e.d + mq) : make_float4(0.f, 0.f, 0.f, 0.f);
+      if constexpr (MODE == EPI_QKV) {
+        rb[r] = ok[r] && kind ? e.row_b[n] : 0;
+        rp[r] = ok[r] && kind ? e.row_pos[n] : 0;
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+      if (!ok[r]) continue;
+      const int n = n0 + j0 + 4 * r;
+      float4 v = a[r];
+      if constexpr (MODE == EPI_F32) {
+        float* o = e.out_f32 + (size_t)n * e.ld;
+        if (mq + 0 < e.M) o[mq + 0] = v.x;
+        if (mq + 1 < e.M) o[mq + 1] = v.y;
+        if (mq + 2 < e.M) o[mq + 2] = v.z;
+        if (mq + 3 < e.M) o[mq + 3] = v.w;
+        continue;
+      }
+      v.x += bias.x; v.y += bias.y; v.z += bias.z; v.w += bias.w;
+      if constexpr (MODE == EPI_Q) {
+        *reinterpret_cast<float4*>(e.out_f32 + (size_t)n * e.d + mq) = v;
+      } else if constexpr (MODE == EPI_RESID) {
+        const float4 o = old[r];
+        *reinterpret_cast<float4*>(e.x + (size_t)n * e.d + mq) = make_float4(o.x + v.x, o.y + v.y, o.z + v.z, o.w + v.w);
+      } else if constexpr (MODE == EPI_GELU) {
+        v = make_float4(gelu_erf(v.x), gelu_erf(v.y), gelu_erf(v.z), gelu_erf(v.w));
+        const size_t idx = (size_t)n * e.M + mq;
+        if (e.act_bf16) {
+          __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
+          *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(e.act) + idx) =
+              make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
+        } else {
+          *reinterpret_cast<float4*>(static_cast<float*>(e.act) + idx) = v;
+        }
+      } else if constexpr (MODE == EPI_QKV) {
+        if (kind == 0) {
+          *reinterpret_cast<float4*>(e.out_f32 + (size_t)n * e.d + mq) = v;
+        } else {
+          const size_t idx = (((size_t)rb[r] * e.n_heads + head) * e.max_pos + rp[r]) * 64 + c;
+          void* base = kind == 1 ? e.kcache : e.vcache;
+          if (e.kv_bf16) {
+            __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
+            *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(base) + idx) =
+                make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
+          } else {
+            *reinterpret_cast<float4*>(static_cast<float*>(base) + idx) = v;
+          }
+        }
+      }
+    }
   }
 }
 

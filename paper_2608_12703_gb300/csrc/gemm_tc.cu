@@ -90,6 +90,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   unsigned long long* tr = epi.trace ? epi.trace + 8ull * (blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z))
                                      : nullptr;
   if (tr && threadIdx.x == 0) tr[0] = global_ns();
+  tl_mark(epi.tl, TL_ENTRY);
   const int n_valid = epi.n_valid ? *epi.n_valid : epi.N;
   const int nkb_total = K / TC_BK;
   const int kb0 = (nkb_total * split) / splits;
@@ -105,6 +106,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   const uint16_t mc_mask = (uint16_t)((1u << mc_size) - 1u);
 
   if (warp == 0) {
+    __syncwarp();   // warp-aligned allocation
     tmem_alloc(tmem_slot, C::TMEM_COLS);
     tmem_relinquish();
   }
@@ -148,6 +150,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       }
     }
     pdl_wait();
+    tl_mark(epi.tl, TL_WORK);
     if constexpr (!LNB)
       for (int i = 0; i < first; ++i) tma_load_2d(sB + i * C::B_BYTES, &mapB, &full[i], (kb0 + i) * TC_BK, n0);
     pdl_launch();
@@ -270,16 +273,61 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     pdl_wait();
     pdl_launch();
   }
+  // Push split: this thread's first-pass outputs of the owner's slice, and
+  // their other operands (bias, residual, row metadata) loaded now, while the
+  // MMAs run.  Item it = (row r of the slice, 4 columns c4).
+  constexpr int EM = MODE == EPI_ARGMAX ? EPI_F32 : MODE;
+  constexpr int IU = 4;
+  const int rows_per = TC_BM / splits;
+  const int r_first = split * rows_per;
+  const int items = rows_per * (BN / 4);
+  auto item_coords = [&](int base, int* mm, int* nn, bool* ok) {
+#pragma unroll
+    for (int u = 0; u < IU; ++u) {
+      const int it = base + u * (int)blockDim.x;
+      const int r = it % rows_per, c4 = it / rows_per;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        mm[4 * u + i] = m0 + r_first + r;
+        nn[4 * u + i] = n0 + 4 * c4 + i;
+        ok[4 * u + i] = it < items && m0 + r_first + r < epi.M && n0 + 4 * c4 + i < n_valid;
+      }
+    }
+  };
+  int pm[4 * IU], pn[4 * IU];
+  bool pok[4 * IU];
+  EpiPre<EM, 4 * IU> pre;
+  if constexpr (PUSH) {
+    item_coords(threadIdx.x, pm, pn, pok);
+    epi_load<EM, 4 * IU>(epi, pm, pn, pok, pre);
+  }
   __syncwarp();
   mbar_wait(done, 0, status);
   if (tr && threadIdx.x == 0) tr[3] = global_ns();
+  tl_mark(epi.tl, TL_MID);
   __syncwarp();   // the warp leaves the wait together: the TMEM loads below are warp-aligned
   tc_fence_after();
 
   const int m = m0 + warp * 32 + lane;
   const uint32_t t_lane = tmem + ((uint32_t)(warp * 32) << 16);
 
-  if (splits == 1) {
+  if (rowwise_mode<MODE>() && splits == 1) {
+    // Stage the tile as [n][m] in the pipeline buffers (every copy has landed
+    // and every MMA retired), then write whole rows.
+    constexpr int LDS = TC_BM + 4;
+    float* stg = reinterpret_cast<float*>(smem);
+    const int ml = warp * 32 + lane;
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(t_lane + c0, v);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) stg[(c0 + i) * LDS + ml] = v[i];
+    }
+    __syncthreads();
+    const int rows = n_valid - n0 < BN ? n_valid - n0 : BN;
+    epi_rows<MODE>(epi, stg, LDS, m0 + 4 * lane, 4 * lane, n0, warp, rows);
+  } else if (splits == 1) {
 #pragma unroll 1
     for (int c0 = 0; c0 < BN; c0 += 16) {
       float v[16];
@@ -316,7 +364,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     }
   } else if constexpr (PUSH) {
     cluster_wait();   // every peer's receive barrier is initialised
-    const int rows_per = TC_BM / splits;
     const int ml = warp * 32 + lane;
     const uint32_t owner = (uint32_t)(ml / rows_per);
     // this split's copy of row ml sits at the same offset in the owner's buffer
@@ -340,13 +387,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     mbar_wait(recv_bar, 0, status);     // the peers' slices
     if (tr && threadIdx.x == 0) tr[6] = global_ns();
     // sum rows [split * rows_per, (split + 1) * rows_per) over the splits, in split order
-    const int r_first = split * rows_per;
-    const int items = rows_per * (BN / 4);
-    constexpr int IU = 4;
     for (int base = threadIdx.x; base < items; base += IU * blockDim.x) {
       int mm[4 * IU], nn[4 * IU];
       bool ok[4 * IU];
       float vals[4 * IU];
+      item_coords(base, mm, nn, ok);
 #pragma unroll
       for (int u = 0; u < IU; ++u) {
         const int it = base + u * blockDim.x;
@@ -354,6 +399,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
         if (it < items) {
           const float* src = recv + r * C::RECV_LD + 4 * c4;
+#pragma unroll 4
           for (int s2 = 0; s2 < splits; ++s2) {
             const float4 p = *reinterpret_cast<const float4*>(src + s2 * rows_per * C::RECV_LD);
             acc.x += p.x; acc.y += p.y; acc.z += p.z; acc.w += p.w;
@@ -363,14 +409,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
         vals[4 * u + 1] = acc.y;
         vals[4 * u + 2] = acc.z;
         vals[4 * u + 3] = acc.w;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          mm[4 * u + i] = m0 + r_first + r;
-          nn[4 * u + i] = n0 + 4 * c4 + i;
-          ok[4 * u + i] = it < items && m0 + r_first + r < epi.M && n0 + 4 * c4 + i < n_valid;
-        }
       }
-      epi_batch<MODE == EPI_ARGMAX ? EPI_F32 : MODE, 4 * IU>(epi, mm, nn, vals, ok);
+      if (base == (int)threadIdx.x) epi_store<EM, 4 * IU>(epi, mm, nn, vals, ok, pre);
+      else epi_batch<EM, 4 * IU>(epi, mm, nn, vals, ok);
     }
     if (tr && threadIdx.x == 0) tr[7] = global_ns();
   } else if constexpr (CLU) {
@@ -389,11 +430,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     if (tr && threadIdx.x == 0) tr[5] = global_ns();
     cluster_sync();
     if (tr && threadIdx.x == 0) tr[6] = global_ns();
-    // this CTA sums rows [rank * 128 / splits, (rank + 1) * 128 / splits) over all splits
-    const int rows_per = TC_BM / splits;
-    const int r_first = split * rows_per;
-    const int items = rows_per * (BN / 4);
-    constexpr int IU = 4;   // items per pass: IU float4 loads from every split in flight
+    // this CTA sums rows [rank * 128 / splits, (rank + 1) * 128 / splits) over all
+    // splits, IU float4 loads from every split in flight per pass
     for (int base = threadIdx.x; base < items; base += IU * blockDim.x) {
       float4 acc[IU];
       const float* local[IU];
@@ -516,6 +554,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
+  tl_mark(epi.tl, TL_EXIT);
 }
 
 // ---------------------------------------------------------------------------

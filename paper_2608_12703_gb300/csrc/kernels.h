@@ -61,14 +61,14 @@ struct TrafficArgs {
 // Validate the step's inputs, lay out the rows and reset the argmax keys.
 void launch_plan_verify(const int* draft, const int* lens, int k, int B, int vocab, int max_pos, const int* kv_len,
                         const int* pending, const int* ready, RowPlan plan, unsigned long long* row_key,
-                        int* status, const TrafficArgs& tr, cudaStream_t st);
+                        int* status, const TrafficArgs& tr, cudaStream_t st, unsigned long long* tl = nullptr);
 void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,
                                RowPlan plan, int* status, cudaStream_t st);
 void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
-                  cudaStream_t st, bool pdl = false);
+                  cudaStream_t st, bool pdl = false, unsigned long long* tl = nullptr);
 // y = LN(x) * g + b over rows < n_rows, written as bf16 or fp32.
 void launch_layernorm(const float* x, const float* g, const float* b, void* y, int y_bf16, const int* n_rows,
-                      int R_max, int d, cudaStream_t st, bool pdl = false);
+                      int R_max, int d, cudaStream_t st, bool pdl = false, unsigned long long* tl = nullptr);
 
 // ---- Attention ---------------------------------------------------------------
 struct AttnArgs {
@@ -98,6 +98,7 @@ struct AttnArgs {
   int rows_max = 0;        // most rows of one utterance in this call
   int splits = 1;          // CTAs (one cluster) per (utterance, head)
   bool pdl = false;        // programmatic dependent launch
+  unsigned long long* tl = nullptr;   // launch timeline slot (tl_mark), or null
 };
 void launch_attention(const AttnArgs& a, cudaStream_t st);
 void launch_attention_tc(const AttnArgs& a, int* status, cudaStream_t st);
@@ -119,7 +120,9 @@ struct AcceptAnchorArgs {
   const int* enc_len;
   unsigned long long* frame_key;    // [B_max], zero between calls
   int* tickets;                     // [B_max], zero between calls
+  int* status;                      // wait time-outs (ST_WAIT_TIMEOUT)
   bool pdl;
+  unsigned long long* tl = nullptr;   // launch timeline slot (tl_mark), or null
 };
 void launch_accept_anchor(const AcceptAnchorArgs& a, cudaStream_t st);
 

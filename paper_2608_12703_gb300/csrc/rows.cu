@@ -40,9 +40,12 @@ __device__ int block_excl_scan(int v, int* total) {
 __global__ void __launch_bounds__(PLAN_THREADS)
 plan_verify_kernel(const int* __restrict__ draft, const int* __restrict__ lens, int k, int B, int vocab, int max_pos,
                    const int* __restrict__ kv_len, const int* __restrict__ pending, const int* __restrict__ ready,
-                   RowPlan plan, unsigned long long* row_key, int* status, TrafficArgs tr) {
+                   RowPlan plan, unsigned long long* row_key, int* status, TrafficArgs tr,
+                   unsigned long long* tl) {
   __shared__ int s_err;
   __shared__ unsigned long long s_cnt[4];
+  tl_mark(tl, TL_ENTRY);
+  tl_mark(tl, TL_WORK);
   if (threadIdx.x == 0) s_err = 0;
   if (threadIdx.x < 4) s_cnt[threadIdx.x] = 0;
   __syncthreads();
@@ -101,6 +104,7 @@ plan_verify_kernel(const int* __restrict__ draft, const int* __restrict__ lens, 
       for (int c = 0; c < 4; ++c) atomicAdd(tr.counters + 1 + c, s_cnt[c]);
     }
   }
+  tl_mark(tl, TL_EXIT);
 }
 
 // Prefill rows: prompt tokens p0 .. p0+c-1 of every utterance at positions p0 + i.
@@ -144,9 +148,9 @@ plan_prefill_kernel(const int* __restrict__ prompt, int P0, int p0, int c, int B
 
 void launch_plan_verify(const int* draft, const int* lens, int k, int B, int vocab, int max_pos, const int* kv_len,
                         const int* pending, const int* ready, RowPlan plan, unsigned long long* row_key,
-                        int* status, const TrafficArgs& tr, cudaStream_t st) {
+                        int* status, const TrafficArgs& tr, cudaStream_t st, unsigned long long* tl) {
   plan_verify_kernel<<<1, PLAN_THREADS, 0, st>>>(draft, lens, k, B, vocab, max_pos, kv_len, pending, ready, plan,
-                                                 row_key, status, tr);
+                                                 row_key, status, tr, tl);
 }
 
 void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,
@@ -157,24 +161,27 @@ void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, 
 // x[r] = tok_emb[token] + pos_emb[position]  (fp32 residual stream)
 template <typename T>
 __global__ void embed_kernel(const T* __restrict__ tok_emb, const T* __restrict__ pos_emb, RowPlan plan, int d,
-                             float* __restrict__ x) {
+                             float* __restrict__ x, unsigned long long* tl) {
+  tl_mark(tl, TL_ENTRY);
   pdl_wait();
+  tl_mark(tl, TL_WORK);
   pdl_launch();
   const int r = blockIdx.x;
   if (r >= *plan.n_rows) return;
   const int t = plan.row_tok[r], p = plan.row_pos[r];
   for (int c = threadIdx.x; c < d; c += blockDim.x)
     x[(size_t)r * d + c] = to_f<T>(tok_emb[(size_t)t * d + c]) + to_f<T>(pos_emb[(size_t)p * d + c]);
+  tl_mark(tl, TL_EXIT);
 }
 
 void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
-                  cudaStream_t st, bool pdl) {
+                  cudaStream_t st, bool pdl, unsigned long long* tl) {
   if (w_bf16)
     launch_ex(embed_kernel<__nv_bfloat16>, dim3(R_max), dim3(128), 0, st, pdl, 1,
-              static_cast<const __nv_bfloat16*>(tok_emb), static_cast<const __nv_bfloat16*>(pos_emb), plan, d, x);
+              static_cast<const __nv_bfloat16*>(tok_emb), static_cast<const __nv_bfloat16*>(pos_emb), plan, d, x, tl);
   else
     launch_ex(embed_kernel<float>, dim3(R_max), dim3(128), 0, st, pdl, 1, static_cast<const float*>(tok_emb),
-              static_cast<const float*>(pos_emb), plan, d, x);
+              static_cast<const float*>(pos_emb), plan, d, x, tl);
 }
 
 // LayerNorm for any d % 4 == 0: a sum pass, a centred sum-of-squares pass over the
@@ -182,8 +189,10 @@ void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan 
 template <typename TO>
 __global__ void __launch_bounds__(256)
 layernorm_any_kernel(const float* __restrict__ x, const float* __restrict__ g, const float* __restrict__ bta,
-                 TO* __restrict__ y, const int* __restrict__ n_rows, int d) {
+                 TO* __restrict__ y, const int* __restrict__ n_rows, int d, unsigned long long* tl) {
+  tl_mark(tl, TL_ENTRY);
   pdl_wait();
+  tl_mark(tl, TL_WORK);
   pdl_launch();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = blockIdx.x * 8 + warp;
@@ -213,18 +222,28 @@ layernorm_any_kernel(const float* __restrict__ x, const float* __restrict__ g, c
     yr[4 * i + 2] = from_f<TO>((v.z - mean) * rstd * gg.z + bb.z);
     yr[4 * i + 3] = from_f<TO>((v.w - mean) * rstd * gg.w + bb.w);
   }
+  tl_mark(tl, TL_EXIT);
 }
 
-// LayerNorm, one warp per row, statistics in fp32.  The row is read once into
+// LayerNorm, one warp per row, statistics in fp32.  The gain and bias (weights)
+// are loaded before the wait on the previous kernel; the row is read once into
 // registers (N4 float4 per lane), then mean, centred variance and the affine
 // write come from the registers.
 template <typename TO, int N4>
 __global__ void __launch_bounds__(256)
 layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const float* __restrict__ bta,
-                 TO* __restrict__ y, const int* __restrict__ n_rows, int d) {
-  pdl_wait();
-  pdl_launch();
+                 TO* __restrict__ y, const int* __restrict__ n_rows, int d, unsigned long long* tl) {
+  tl_mark(tl, TL_ENTRY);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float4 gw[N4], bw[N4];
+#pragma unroll
+  for (int i = 0; i < N4; ++i) {
+    gw[i] = __ldg(reinterpret_cast<const float4*>(g) + lane + 32 * i);
+    bw[i] = __ldg(reinterpret_cast<const float4*>(bta) + lane + 32 * i);
+  }
+  pdl_wait();
+  tl_mark(tl, TL_WORK);
+  pdl_launch();
   const int r = blockIdx.x * 8 + warp;
   if (r >= *n_rows) return;
   const float4* xr = reinterpret_cast<const float4*>(x + (size_t)r * d);
@@ -247,48 +266,48 @@ layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g, const
 #pragma unroll
   for (int i = 0; i < N4; ++i) {
     const int c4 = lane + 32 * i;
-    const float4 gg = reinterpret_cast<const float4*>(g)[c4];
-    const float4 bb = reinterpret_cast<const float4*>(bta)[c4];
+    const float4 gg = gw[i], bb = bw[i];
     yr[4 * c4 + 0] = from_f<TO>((v[i].x - mean) * rstd * gg.x + bb.x);
     yr[4 * c4 + 1] = from_f<TO>((v[i].y - mean) * rstd * gg.y + bb.y);
     yr[4 * c4 + 2] = from_f<TO>((v[i].z - mean) * rstd * gg.z + bb.z);
     yr[4 * c4 + 3] = from_f<TO>((v[i].w - mean) * rstd * gg.w + bb.w);
   }
+  tl_mark(tl, TL_EXIT);
 }
 
 template <typename TO>
 static void launch_ln_t(const float* x, const float* g, const float* b, TO* y, const int* n_rows, int R_max, int d,
-                        cudaStream_t st, bool pdl) {
+                        cudaStream_t st, bool pdl, unsigned long long* tl) {
   const dim3 grid((R_max + 7) / 8), block(256);
   switch (d / 128) {   // d is a multiple of 64; d % 128 == 64 rounds up with a guarded tail
-    case 1: launch_ex(layernorm_kernel<TO, 1>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    case 2: launch_ex(layernorm_kernel<TO, 2>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    case 3: launch_ex(layernorm_kernel<TO, 3>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    case 4: launch_ex(layernorm_kernel<TO, 4>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    case 5: launch_ex(layernorm_kernel<TO, 5>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    case 6: launch_ex(layernorm_kernel<TO, 6>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    case 8: launch_ex(layernorm_kernel<TO, 8>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    case 10: launch_ex(layernorm_kernel<TO, 10>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    case 12: launch_ex(layernorm_kernel<TO, 12>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    case 16: launch_ex(layernorm_kernel<TO, 16>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
-    default: launch_ex(layernorm_any_kernel<TO>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d); break;
+    case 1: launch_ex(layernorm_kernel<TO, 1>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    case 2: launch_ex(layernorm_kernel<TO, 2>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    case 3: launch_ex(layernorm_kernel<TO, 3>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    case 4: launch_ex(layernorm_kernel<TO, 4>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    case 5: launch_ex(layernorm_kernel<TO, 5>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    case 6: launch_ex(layernorm_kernel<TO, 6>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    case 8: launch_ex(layernorm_kernel<TO, 8>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    case 10: launch_ex(layernorm_kernel<TO, 10>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    case 12: launch_ex(layernorm_kernel<TO, 12>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    case 16: launch_ex(layernorm_kernel<TO, 16>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
+    default: launch_ex(layernorm_any_kernel<TO>, grid, block, 0, st, pdl, 1, x, g, b, y, n_rows, d, tl); break;
   }
 }
 
 void launch_layernorm(const float* x, const float* g, const float* b, void* y, int y_bf16, const int* n_rows,
-                      int R_max, int d, cudaStream_t st, bool pdl) {
+                      int R_max, int d, cudaStream_t st, bool pdl, unsigned long long* tl) {
   if (d % 128) {   // widths that are not a whole number of float4 per lane
     const dim3 grid((R_max + 7) / 8);
     if (y_bf16)
       launch_ex(layernorm_any_kernel<__nv_bfloat16>, grid, dim3(256), 0, st, pdl, 1, x, g, b,
-                static_cast<__nv_bfloat16*>(y), n_rows, d);
+                static_cast<__nv_bfloat16*>(y), n_rows, d, tl);
     else
       launch_ex(layernorm_any_kernel<float>, grid, dim3(256), 0, st, pdl, 1, x, g, b, static_cast<float*>(y),
-                n_rows, d);
+                n_rows, d, tl);
     return;
   }
-  if (y_bf16) launch_ln_t(x, g, b, static_cast<__nv_bfloat16*>(y), n_rows, R_max, d, st, pdl);
-  else launch_ln_t(x, g, b, static_cast<float*>(y), n_rows, R_max, d, st, pdl);
+  if (y_bf16) launch_ln_t(x, g, b, static_cast<__nv_bfloat16*>(y), n_rows, R_max, d, st, pdl, tl);
+  else launch_ln_t(x, g, b, static_cast<float*>(y), n_rows, R_max, d, st, pdl, tl);
 }
 
 // After a prefill chunk: the rows' K/V are cached, so the committed length moves on.

@@ -24,6 +24,38 @@ if ROOT not in sys.path:
 import workload as W  # noqa: E402
 
 
+def timeline_summary(ns, kinds, rounds):
+    """Per launch kind: launches per round, mean busy time (end - past the wait),
+    its part up to the kernel's midpoint (GEMM: MMAs done; attention: key loop
+    done), the mean gap from the previous launch's end to this one's
+    past-the-wait point, and the shares of the recorded span."""
+    from paper_2608_12703_gb300 import asrspec as A
+    ns = ns.astype(np.int64)
+    ok = ns[:, 3] > 0
+    t0 = ns[ok, 0].min() if ok.any() else 0
+    span = (ns[ok, 3].max() - t0) / 1e3 if ok.any() else 0.0
+    rows = {}
+    prev_end = None
+    for (s, w, m, e), k in zip(ns, kinds):
+        if e == 0:
+            continue
+        w = w or s
+        r = rows.setdefault(int(k), [0, 0.0, 0.0, 0.0])
+        r[0] += 1
+        r[1] += (e - w) / 1e3
+        r[2] += (m - w) / 1e3 if m else 0.0
+        if prev_end is not None:
+            r[3] += (w - prev_end) / 1e3
+        prev_end = e
+    lines = [f"  launch timeline over {rounds} rounds: span {span:.1f} us ({span / max(rounds, 1):.1f} us per round), "
+             f"{int(ok.sum())} launches recorded"]
+    lines.append(f"  {'kind':<20}{'per round':>10}{'busy us':>10}{'to mid':>9}{'gap us':>9}{'busy %':>9}{'gap %':>8}")
+    for k, (n, busy, mid, gap) in sorted(rows.items(), key=lambda kv: -(kv[1][1] + kv[1][3])):
+        lines.append(f"  {A.tl_kind_name(k):<20}{n / rounds:>10.1f}{busy / n:>10.2f}{mid / n:>9.2f}{gap / n:>9.2f}"
+                     f"{100 * busy / span:>9.1f}{100 * gap / span:>8.1f}")
+    return "\n".join(lines)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--config", default="large-bf16-b1-k8", choices=sorted(W.CONFIGS))
@@ -32,6 +64,8 @@ def main():
     ap.add_argument("--no-graphs", action="store_true")
     ap.add_argument("--classes", action="store_true",
                     help="also time each kernel class with CUDA events (direct launches)")
+    ap.add_argument("--timeline", action="store_true",
+                    help="also record the launch timeline of the rounds (direct launches) and summarise it per kind")
     args = ap.parse_args()
 
     import torch
@@ -75,6 +109,13 @@ def main():
         A.asr_spec_profile(sess.h, False)
         print("  per round (us, event-bracketed direct launches): " + ", ".join(
             f"{n} {1e3 * m / args.rounds:.0f}" for n, m in zip(A.PROF_CLASSES, ms)))
+    if args.timeline:
+        A.asr_spec_timeline(sess.h, True)
+        for i in range(args.rounds):
+            sess.verify_device(drafts[i], lens, wl.k)
+        ns, kinds = A.asr_spec_timeline_read(sess.h)
+        A.asr_spec_timeline(sess.h, False)
+        print(timeline_summary(ns, kinds, args.rounds))
     sess.close()
     if st:
         sys.exit(1)

@@ -138,3 +138,45 @@ def test_graph_replay_matches_direct_launch_and_profile(built_lib, cuda):
         assert s.status() == 0
         s.close()
     assert outs[0] == outs[1] == outs[2]
+
+
+def test_timeline_records_every_launch_in_order(built_lib, cuda):
+    """The launch timeline: one record per kernel of the verify chain, in
+    launch order and of the expected kind; every record starts, passes its
+    wait on the previous kernel and ends in that order, and no kernel passes
+    its wait before the previous kernel has ended (dependent launches really
+    wait).  Recording changes no result."""
+    from paper_2608_12703_gb300 import asrspec as A
+    from paper_2608_12703_gb300.session import Session
+    blob = W.make_weights(DIMS, std=0.1)
+    outs, records = [], None
+    for timeline in (False, True):
+        s = Session(DIMS, blob, max_batch=3, max_draft=4)
+        _ready(s)
+        A.asr_spec_timeline(s.h, timeline)
+        res = []
+        for r in range(3):
+            o = s.verify(np.array([[r, 2, 3, 4]] * 3), np.array([4, 2, r % 2 - 1]))
+            res.append((list(o.accepted), list(o.bonus), list(o.kv_len), list(o.anchor)))
+        if timeline:
+            records = A.asr_spec_timeline_read(s.h)
+            ns2, _ = A.asr_spec_timeline_read(s.h)
+            assert len(ns2) == 0                       # a read clears the record
+        outs.append(res)
+        assert s.status() == 0
+        s.close()
+    assert outs[0] == outs[1]
+    ns, kinds = records
+    g, ln = A.TL_GEMM, 3   # LayerNorm as its own launch (the default)
+    layer = [ln, g + 1, 4, g + 2, ln, g + 3, 5, g + 2, ln, g + 4, g + 2]
+    one = [1, 2] + layer * DIMS.n_layers + [ln, g + 6, 6]
+    assert list(kinds) == one * 3
+    ns = ns.astype(np.int64)
+    start, work, mid, end = ns[:, 0], ns[:, 1], ns[:, 2], ns[:, 3]
+    assert np.all(end > 0)
+    assert np.all(start <= work) and np.all(work <= end)
+    has_mid = np.array([k >= g or k in (4, 5) for k in kinds])
+    assert np.all(mid[has_mid] > 0) and np.all(mid[~has_mid] == 0)
+    assert np.all(mid[has_mid] <= end[has_mid])
+    slack = 2000   # ns: the timer is global, CTAs on different SMs read it
+    assert np.all(work[1:] >= end[:-1] - slack)
