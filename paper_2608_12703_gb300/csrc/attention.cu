@@ -203,9 +203,9 @@ constexpr int ANCHOR_HMAX = 32;   // heads (d_model <= 2048)
 
 template <typename T>
 struct AnchorCfg {
-  static constexpr int FB = sizeof(T) == 2 ? 32 : 16;   // frames per CTA
+  static constexpr int FB = sizeof(T) == 2 ? 16 : 8;   // frames per CTA (40 KB of keys for 20 heads)
   static constexpr int ROW_BYTES = 64 * (int)sizeof(T);
-  static constexpr int SMEM = ANCHOR_HMAX * FB * ROW_BYTES;   // keys [H][FB][64]; <= 128 KB
+  static constexpr int SMEM = ANCHOR_HMAX * FB * ROW_BYTES;   // keys [H][FB][64]; <= 64 KB
 };
 
 template <typename T>

@@ -5,8 +5,10 @@
 // block-causal, cross-attention covers the utterance's encoder frames), laid
 // out for GB300:
 //   * one CTA = one (utterance, head, split); it streams every S-th 128-key
-//     chunk of the utterance's K and V through a 3-deep ring of TMA tile loads
-//     into 128-byte-swizzled shared memory (one mbarrier per slot);
+//     chunk of the utterance's K and V through a ring of TMA tile loads into
+//     128-byte-swizzled shared memory (one mbarrier per slot): 2 deep (three
+//     CTAs share an SM) for self-attention and for unsplit cross-attention,
+//     3 deep when the encoder keys are split over a cluster;
 //   * the utterance's rows (up to 16 per m-tile) are the M side of
 //     mma.sync m16n8k16 (bf16 in, fp32 accumulate): S = Q K^T, then an online
 //     softmax on the accumulator fragments (quad shuffles), then O = P V with
@@ -49,14 +51,13 @@ __device__ __forceinline__ uint32_t sw128(int row, int chunk16) {
 }
 
 constexpr int TCA_CH = 128;        // keys per chunk (one TMA tile of K and one of V)
-constexpr int TCA_STAGES = 3;      // chunks in flight per CTA
 constexpr int TCA_TILE = TCA_CH * 128;
 
-template <int MT>
+template <int MT, int STAGES>
 struct TcaCfg {
   static constexpr int KW = TCA_CH / 4;       // keys per warp per chunk
   static constexpr int NT = KW / 8;           // n-tiles of keys per warp
-  static constexpr int RING = TCA_STAGES * 2 * TCA_TILE;
+  static constexpr int RING = STAGES * 2 * TCA_TILE;
   static constexpr int OW = 4 * MT * 16 * 64 * 4;
   static constexpr int PART = (32 * 64 + 64) * 4;   // this CTA's (max, sum, output) per row
   static constexpr int SMEM = 1024 + (RING > OW ? RING : OW) + PART;
@@ -67,11 +68,11 @@ struct TcaCfg {
 // keeping a running (max, sum, output) per row (online softmax).  With S > 1
 // the S splits of a (utterance, head) form one cluster and merge their
 // results through distributed shared memory, in split order.
-template <int MT>
+template <int MT, int TCA_STAGES>
 __global__ void __launch_bounds__(TCA_THREADS)
 attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, AttnArgs a,
                int* status) {
-  using C = TcaCfg<MT>;
+  using C = TcaCfg<MT, TCA_STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   float* Ow = reinterpret_cast<float*>(smem);                  // warp partials, after the ring is drained
@@ -315,31 +316,41 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
   tl_mark(a.tl, TL_EXIT);
 }
 
-template <int MT>
+template <int MT, int ST>
 static void configure_one() {
-  cudaFuncSetAttribute(attn_tc_kernel<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcaCfg<MT>::SMEM);
+  cudaFuncSetAttribute(attn_tc_kernel<MT, ST>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcaCfg<MT, ST>::SMEM);
 }
 
 void configure_attention_tc() {
   static std::once_flag once;
   std::call_once(once, [] {
-    configure_one<1>();
-    configure_one<2>();
+    configure_one<1, 2>();
+    configure_one<2, 2>();
+    configure_one<1, 3>();
+    configure_one<2, 3>();
   });
 }
 
-template <int MT>
+template <int MT, int ST>
 static void launch_one(const AttnArgs& a, int splits, int* status, cudaStream_t st) {
-  launch_ex(attn_tc_kernel<MT>, dim3(splits, a.H, a.B), dim3(TCA_THREADS), TcaCfg<MT>::SMEM, st, a.pdl, splits,
-            *a.kmap, *a.vmap, a, status);
+  launch_ex(attn_tc_kernel<MT, ST>, dim3(splits, a.H, a.B), dim3(TCA_THREADS), TcaCfg<MT, ST>::SMEM, st, a.pdl,
+            splits, *a.kmap, *a.vmap, a, status);
 }
 
 // a.splits CTAs (1, 2, 4 or 8; one cluster) per (utterance, head);
 // rows_max > 16 takes two m-tiles.
 void launch_attention_tc(const AttnArgs& a, int* status, cudaStream_t st) {
   configure_attention_tc();
-  if (a.rows_max > 16) launch_one<2>(a, a.splits, status, st);
-  else launch_one<1>(a, a.splits, status, st);
+  if (a.causal) {
+    if (a.rows_max > 16) launch_one<2, 2>(a, a.splits, status, st);
+    else launch_one<1, 2>(a, a.splits, status, st);
+  } else if (a.splits == 1) {   // many utterances: more CTAs per SM (54 vs 56 us at batch 64)
+    if (a.rows_max > 16) launch_one<2, 2>(a, a.splits, status, st);
+    else launch_one<1, 2>(a, a.splits, status, st);
+  } else {                      // few utterances, keys split over a cluster: deeper ring per CTA
+    if (a.rows_max > 16) launch_one<2, 3>(a, a.splits, status, st);
+    else launch_one<1, 3>(a, a.splits, status, st);
+  }
 }
 
 bool make_tmap_cache(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {

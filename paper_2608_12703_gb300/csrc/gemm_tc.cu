@@ -81,10 +81,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   __shared__ int s_last;
   __shared__ float ln_mean[LNB ? BN : 1], ln_rstd[LNB ? BN : 1];
 
-  // cluster split: the splits of a tile are consecutive CTAs along x (one cluster)
-  const int tile_m = CLU ? (int)blockIdx.x / splits : (int)blockIdx.x;
+  // Grid: cluster split: (M tiles x splits, N tiles), the splits of a tile
+  // consecutive along x (one cluster); multicast: (M tiles, N tiles), the N
+  // tiles of an M tile one cluster; otherwise (N tiles, M tiles, splits), so
+  // that the CTAs sharing a weight tile run together and read it from HBM once.
+  const int tile_m = CLU ? (int)blockIdx.x / splits : MC ? (int)blockIdx.x : (int)blockIdx.y;
   const int split = CLU ? (int)blockIdx.x % splits : (int)blockIdx.z;
-  const int tile_n = blockIdx.y;
+  const int tile_n = (CLU || MC) ? (int)blockIdx.y : (int)blockIdx.x;
   const int m0 = tile_m * TC_BM, n0 = tile_n * BN;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   unsigned long long* tr = epi.trace ? epi.trace + 8ull * (blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z))
@@ -472,7 +475,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     if (tr && threadIdx.x == 0) tr[7] = global_ns();
     cluster_sync();   // no CTA leaves while another may still read its shared memory
   } else {
-    const int tile = tile_n * gridDim.x + tile_m;
+    const int tile = tile_n * ((epi.M + TC_BM - 1) / TC_BM) + tile_m;
     float* my = ws + ((size_t)(tile * splits + split) * TC_BM + warp * 32 + lane) * BN;
 #pragma unroll 1
     for (int c0 = 0; c0 < BN; c0 += 16) {
@@ -654,7 +657,7 @@ static void launch_tc_ln(const TcGemm& g, const Epi& epi, int* status, cudaStrea
       return;
     }
   }
-  launch_ex(gemm_tc_kernel<BN, MODE, false, LNB, false>, dim3(mt, nt, g.splits), dim3(128), TcCfg<BN>::SMEM, st,
+  launch_ex(gemm_tc_kernel<BN, MODE, false, LNB, false>, dim3(nt, mt, g.splits), dim3(128), TcCfg<BN>::SMEM, st,
             g.pdl, 1, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
 }
 

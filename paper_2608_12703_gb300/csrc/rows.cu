@@ -406,4 +406,5 @@ void launch_mark_ready(const int* enc_len, int B, int t_max, int* ready, int* kv
   mark_ready_kernel<<<(B + 127) / 128, 128, 0, st>>>(enc_len, B, t_max, ready, kv_len, pending, status);
 }
 
+
 }  // namespace asrspec
