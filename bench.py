@@ -9,7 +9,7 @@ value = emitted tokens (accepted drafts + bonus tokens) per second over the
 timed steps, with weights and encoder states resident in HBM.
 
 Also reported, on the same workload: per-verify-call latency (CUDA events),
-the dominant kernel class against its roofline, an end-to-end number through
+the dominant kernel against its roofline, an end-to-end number through
 host buffers, the CPU oracle on a bounded sample, and the batch-1 workload.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
@@ -255,6 +255,15 @@ class GpuRun:
                     verify_us=dict(median=float(np.median(per_call)), p10=float(np.percentile(per_call, 10)),
                                    p90=float(np.percentile(per_call, 90)), calls=int(len(per_call))))
 
+    def launch_timeline(self):
+        """One decode with the launch timeline recorded (direct launches)."""
+        A = self.A
+        A.asr_spec_timeline(self.sess.h, True)
+        self.decode()
+        tl = A.asr_spec_timeline_read(self.sess.h)
+        A.asr_spec_timeline(self.sess.h, False)
+        return tl
+
     def profile(self):
         """One decode with per-kernel-class CUDA events (direct launches)."""
         A = self.A
@@ -300,41 +309,94 @@ class GpuRun:
                     h2d_bytes_per_step=int(h2d // steps), d2h_bytes_per_step=int(d2h // steps))
 
 
-def roofline(dims, ms, launches, traffic, pk):
-    """Dominant kernel class of one profiled decode against its roofline."""
-    from paper_2608_12703_gb300.asrspec import PROF_CLASSES
-    cls = int(np.argmax(ms[:4]))
-    name = PROF_CLASSES[cls]
+# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one
+# ncu capture of the kernel on the workload, as summarised in profiles/; averaged
+# over the kernel's launches in one layer.  Only valid for the kernel code the
+# capture ran on: drop an entry when that kernel changes.
+NCU_TRAFFIC = {
+    ("large-bf16-b1-k8", "resid"): (6.727e6, "profiles/gemm_tc_kernel_resid_large-bf16-b1-k8.md"),
+    ("large-bf16-b64-k6", "cross_attn"): (337.7e6, "profiles/attn_tc_kernel_large-bf16-b64-k6_dram.md"),
+}
+
+# Launch kinds of the timeline (ASR_TL_*; a LayerNorm-fused GEMM counts with its
+# GEMM) and the profile class (CUDA events) that times the same kernel.
+TL_KIND_CLASS = {17: "qkv", 18: "resid", 19: "query", 20: "mlp_up", 22: "lm_head", 4: "self_attn",
+                 5: "cross_attn", 3: "layernorm"}
+
+
+def kind_class(kind: int):
+    return TL_KIND_CLASS.get(kind - 32 if kind >= 48 else kind)
+
+
+def algorithmic_work(dims, cls, traffic):
+    """(bytes, flops, per-unit statement) of one decode's launches of a kernel class.
+    Bytes are the unique operands a launch must read from HBM: weights for a
+    projection (its activations are L2-resident), the K/V rows for attention."""
     es = 2 if dims.dtype == "bf16" else 4
     d, L, F, V = dims.d_model, dims.n_layers, dims.d_ffn, dims.vocab
-    calls, self_b, cross_b, anchor_b, rows = (int(x) for x in traffic[:5])
-    t = ms[cls] / 1e3
-    n = int(launches[cls])
-    if name == "cross_attn":
-        work, bound, unit, peak = cross_b / t / 1e9, "hbm", "GB/s", pk["hbm"]
-        per_unit = "2 * T_b * d * 2 bytes of encoder K/V per active utterance per layer"
-    elif name == "self_attn":
-        work, bound, unit, peak = self_b / t / 1e9, "hbm", "GB/s", pk["hbm"]
-        per_unit = "2 * (P_b + n_b) * d * 2 bytes of self K/V per active utterance per layer"
+    calls, self_b, cross_b, _, rows = (float(x) for x in traffic[:5])
+    mk = {"qkv": (L * 3 * d * d, "3 d^2 weights per layer"),
+          "resid": (L * (2 * d * d + F * d), "d^2 + d^2 + F d weights per layer (self out, cross out, MLP down)"),
+          "query": (L * d * d, "d^2 weights per layer"),
+          "mlp_up": (L * F * d, "F d weights per layer"),
+          "lm_head": (V * d, "V d weights")}
+    if cls in mk:
+        params, what = mk[cls]
+        return (calls * params * es, 2.0 * rows * params,
+                f"{what} x {es} bytes per verify call; 2 x scored rows x those parameters in flops")
+    if cls == "self_attn":
+        return self_b, 0.0, "2 (K, V) x (P_b + n_b) keys x d x 2 bytes per active utterance per layer"
+    if cls == "cross_attn":
+        return cross_b, 0.0, "2 (K, V) x T_b frames x d x 2 bytes per active utterance per layer"
+    if cls == "layernorm":
+        return rows * (3 * L + 1) * d * (4 + es), 0.0, "rows x d x (4 read + 2 written) bytes per LayerNorm"
+    return 0.0, 0.0, ""
+
+
+def roofline(wl_name, dims, tl, ms, launches, traffic, pk):
+    """The kernel with the largest share of the decode (launch timeline, busy
+    time past the wait on the previous kernel) against its roofline.
+    achieved = algorithmic work / its CUDA-event time (each launch bracketed by
+    events on the library stream, launches one by one: no overlap with the
+    neighbours); the in-chain figure divides by the timeline's busy time of
+    the same launches in the normal (dependent-launch) chain."""
+    from paper_2608_12703_gb300.asrspec import PROF_CLASSES
+    ns, kinds = tl
+    busy = {}
+    count = {}
+    for (s, w, m, e), k in zip(ns.astype(np.int64), kinds):
+        c = kind_class(int(k))
+        if c is None or e == 0:
+            continue
+        busy[c] = busy.get(c, 0.0) + (e - (w or s)) / 1e9
+        count[c] = count.get(c, 0) + 1
+    total = sum(busy.values())
+    name = max(busy, key=busy.get)
+    ci = PROF_CLASSES.index(name)
+    t = ms[ci] / 1e3
+    n = int(launches[ci])
+    nbytes, flops, per_unit = algorithmic_work(dims, name, traffic)
+    balance = pk["bf16_sus"] * 1e12 / (pk["hbm"] * 1e9)
+    if flops > 0 and flops / nbytes > balance:
+        bound, unit, peak, work, scale = "tensor", "TFLOP/s", pk["bf16_sus"], flops, 1e12
     else:
-        if name == "proj_gemm":
-            wbytes = calls * L * (6 * d * d + 2 * F * d) * es
-            flops = 2.0 * rows * L * (6 * d * d + 2 * F * d)
-        else:
-            wbytes = calls * V * d * es
-            flops = 2.0 * rows * V * d
-        intensity = flops / max(wbytes, 1)
-        if intensity > pk["bf16_sus"] * 1e12 / (pk["hbm"] * 1e9):
-            work, bound, unit, peak = flops / t / 1e12, "tensor", "TFLOP/s", pk["bf16_sus"]
-            per_unit = "2 * rows * K * M flops per projection"
-        else:
-            work, bound, unit, peak = wbytes / t / 1e9, "hbm", "GB/s", pk["hbm"]
-            per_unit = "M * K * 2 bytes of weights per projection launch"
-    return {"kernel": name, "bound": bound, "achieved": round(work, 2), "peak": peak, "unit": unit,
-            "frac": round(work / peak, 4), "traffic": None, "launches": n,
-            "ms_per_launch": round(ms[cls] / max(n, 1), 5), "per_unit": per_unit,
+        bound, unit, peak, work, scale = "hbm", "GB/s", pk["hbm"], nbytes, 1e9
+    achieved = work / t / scale
+    chain = work / busy[name] / scale
+    ncu = NCU_TRAFFIC.get((wl_name, name))
+    return {"kernel": name, "bound": bound, "achieved": round(achieved, 2), "peak": peak, "unit": unit,
+            "frac": round(achieved / peak, 4), "traffic": ncu[0] if ncu else None,
+            "traffic_source": ncu[1] if ncu else None,
+            "algorithmic_bytes_per_launch": round(nbytes / max(n, 1), 1), "launches": n,
+            "ms_per_launch": round(ms[ci] / max(n, 1), 5), "per_unit": per_unit,
+            "units": "work summed over the decode's launches of the kernel; per launch = that / launches",
             "peak_source": pk["src"],
-            "class_ms": {PROF_CLASSES[i]: round(float(ms[i]), 3) for i in range(len(ms))}}
+            "share_of_busy_time": round(busy[name] / total, 4),
+            "in_chain": {"achieved": round(chain, 2), "frac": round(chain / peak, 4),
+                         "us_per_launch": round(1e6 * busy[name] / max(count[name], 1), 3),
+                         "timer": "GPU global timer, first CTA past its wait to last CTA exit"},
+            "class_ms": {PROF_CLASSES[i]: round(float(ms[i]), 3) for i in range(len(ms))},
+            "busy_share": {k: round(v / total, 4) for k, v in sorted(busy.items(), key=lambda kv: -kv[1])}}
 
 
 def step_bytes(dims, traffic, calls_override=None):
@@ -496,6 +558,7 @@ def main():
     total_tokens = world * args.steps * run.tokens_per_decode
     value = total_tokens / (ms / 1e3)
     prof_ms, prof_launches, prof_traffic = run.profile()
+    tl = run.launch_timeline()
     line = base_line(args, wl, world)
     bytes_per_call = step_bytes(wl.dims, prof_traffic)
     line.update({
@@ -508,7 +571,7 @@ def main():
                        "frac_nominal_8tbs": bytes_per_call / (res["verify_us"]["median"] * 1e-6) / 8e12},
         "clocks": res["clocks"],
         "gpu_launches": res["launches"] + 0,
-        "roofline": roofline(wl.dims, prof_ms, prof_launches, prof_traffic, pk),
+        "roofline": roofline(wl.name, wl.dims, tl, prof_ms, prof_launches, prof_traffic, pk),
     })
     if not args.no_e2e:
         line["e2e"] = run.e2e(max(1, min(args.steps, 2)))
@@ -526,6 +589,7 @@ def main():
             r1 = GpuRun(wl1)
             b1 = r1.timed(args.steps, args.warmup, None, gpu_index=local)
             pm, pl, pt = r1.profile()
+            tl1 = r1.launch_timeline()
             bpc = step_bytes(wl1.dims, pt)
             line["batch1"] = {
                 "workload": wl1.name, "value": args.steps * r1.tokens_per_decode / (b1["ms"] / 1e3),
@@ -534,7 +598,7 @@ def main():
                 "verify_hbm": {"bytes_per_call": bpc,
                                "frac": bpc / (b1["verify_us"]["median"] * 1e-6) / (pk["hbm"] * 1e9),
                                "frac_nominal_8tbs": bpc / (b1["verify_us"]["median"] * 1e-6) / 8e12},
-                "clocks": b1["clocks"], "roofline": roofline(wl1.dims, pm, pl, pt, pk)}
+                "clocks": b1["clocks"], "roofline": roofline(wl1.name, wl1.dims, tl1, pm, pl, pt, pk)}
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()

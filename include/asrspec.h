@@ -176,12 +176,16 @@ void asr_spec_destroy(asr_spec_handle h);
  * (launches[ASR_PROF_N]), and the algorithmic traffic counters
  * (traffic[8]: verify calls, self K/V bytes, encoder K/V bytes, anchor key
  * bytes, scored rows; weight bytes follow from the dims), then reset all. */
-#define ASR_PROF_PROJ 0    /* decoder projection GEMMs */
-#define ASR_PROF_SELF 1    /* self-attention (chunk + merge kernels) */
-#define ASR_PROF_CROSS 2   /* cross-attention (chunk + merge kernels) */
-#define ASR_PROF_LMHEAD 3  /* LM head with fused argmax */
-#define ASR_PROF_OTHER 4   /* row plan, embedding, LayerNorm, accept, anchor */
-#define ASR_PROF_N 5
+#define ASR_PROF_QKV 0        /* self-attention Q/K/V projection (+ cache append) */
+#define ASR_PROF_RESID 1      /* projections added to the residual: self out, cross out, MLP down */
+#define ASR_PROF_QUERY 2      /* cross-attention query projection */
+#define ASR_PROF_UP 3         /* MLP up projection + GELU */
+#define ASR_PROF_SELF 4       /* self-attention */
+#define ASR_PROF_CROSS 5      /* cross-attention */
+#define ASR_PROF_LMHEAD 6     /* LM head with fused argmax */
+#define ASR_PROF_LAYERNORM 7  /* stand-alone LayerNorm */
+#define ASR_PROF_OTHER 8      /* row plan, embedding, accept + anchor, encoder cache build, prefill steps */
+#define ASR_PROF_N 9
 int asr_spec_set_graphs(asr_spec_handle h, int enable);
 int asr_spec_profile(asr_spec_handle h, int enable);
 int asr_spec_profile_read(asr_spec_handle h, double* ms, int64_t* launches, uint64_t* traffic);
@@ -200,7 +204,7 @@ int asr_spec_profile_read(asr_spec_handle h, double* ms, int64_t* launches, uint
  * launch order: ns[4 * i + 0..3] = (start, past the wait, midpoint, end), 0
  * where nothing was recorded, kind[i] as below; *count = the
  * launches recorded since the last read; then clear.  Host pointers. */
-#define ASR_TL_CAP 8192
+#define ASR_TL_CAP 65536
 #define ASR_TL_OTHER 0
 #define ASR_TL_PLAN 1          /* row plan of a verify step */
 #define ASR_TL_EMBED 2         /* token + position embedding */

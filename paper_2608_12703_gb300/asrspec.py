@@ -29,8 +29,8 @@ EXPORTED = [
     "asr_spec_test_gemm", "asr_spec_set_graphs", "asr_spec_profile", "asr_spec_profile_read",
     "asr_spec_gemm_noalloc", "asr_spec_timeline", "asr_spec_timeline_read",
 ]
-PROF_CLASSES = ["proj_gemm", "self_attn", "cross_attn", "lm_head", "other"]
-TL_CAP = 8192
+PROF_CLASSES = ["qkv", "resid", "query", "mlp_up", "self_attn", "cross_attn", "lm_head", "layernorm", "other"]
+TL_CAP = 65536
 TL_GEMM, TL_LN_FUSED = 16, 32
 TL_KINDS = {0: "other", 1: "plan", 2: "embed", 3: "layernorm", 4: "attn_self", 5: "attn_cross", 6: "accept_anchor"}
 TL_GEMM_EPILOGUES = {0: "plain", 1: "qkv", 2: "residual", 3: "query", 4: "gelu", 5: "cross_kv", 6: "argmax"}

@@ -208,7 +208,12 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   Epi epi = epi_in;
   epi.M = M;
   epi.N = N;
-  Prof p(h, (mode == EPI_ARGMAX || mode == EPI_F32) ? ASR_PROF_LMHEAD : ASR_PROF_PROJ, 1);
+  const int cls = mode == EPI_QKV     ? ASR_PROF_QKV
+                  : mode == EPI_RESID ? ASR_PROF_RESID
+                  : mode == EPI_Q     ? ASR_PROF_QUERY
+                  : mode == EPI_GELU  ? ASR_PROF_UP
+                                      : ASR_PROF_LMHEAD;
+  Prof p(h, cls, 1);
   if (!h->bf16) {
     launch_gemm_simt(W, 0, X, 0, M, N, K, mode, epi, h->st);
     return 0;
@@ -268,7 +273,7 @@ int gemm_rows_ln(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K
     return gemm_rows(h, W, mW, M, K, nullptr, ln_out_id, N, mode, e);
   }
   {
-    Prof p(h, ASR_PROF_OTHER, 1);
+    Prof p(h, ASR_PROF_LAYERNORM, 1);
     Tl t(h, ASR_TL_LAYERNORM);
     launch_layernorm(h->x, g, b, ln_out, h->bf16, h->plan.n_rows, N, K, h->st, h->use_pdl, h->tl_cur);
   }
@@ -730,10 +735,10 @@ int asr_spec_encode_cache(asr_spec_handle h, int32_t B, const void* enc_states, 
     g.splits = 1;
     g.ws = h->ws;
     g.tickets = h->tickets;
-    Prof pg(h, ASR_PROF_PROJ, 1);
+    Prof pg(h, ASR_PROF_OTHER, 1);
     launch_gemm_tc(g, EPI_CROSSKV, e, h->status, h->st);
   } else {
-    Prof pg(h, ASR_PROF_PROJ, 1);
+    Prof pg(h, ASR_PROF_OTHER, 1);
     launch_gemm_simt(enc_states, 0, h->w_cross, 0, M, N, d, EPI_CROSSKV, e, h->st);
   }
   CK(cudaGetLastError());

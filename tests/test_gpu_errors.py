@@ -133,7 +133,7 @@ def test_graph_replay_matches_direct_launch_and_profile(built_lib, cuda):
         ms, launches, traffic = A.asr_spec_profile_read(s.h)
         assert traffic[0] == 5 and launches.sum() > 0
         if prof:
-            assert ms[A.PROF_CLASSES.index("proj_gemm")] > 0
+            assert ms[A.PROF_CLASSES.index("qkv")] > 0 and ms[A.PROF_CLASSES.index("resid")] > 0
         outs.append(res)
         assert s.status() == 0
         s.close()
