@@ -213,7 +213,7 @@ int asr_spec_profile_read(asr_spec_handle h, double* ms, int64_t* launches, uint
 #define ASR_TL_ATTN_CROSS 5    /* cross-attention */
 #define ASR_TL_ACCEPT 6        /* acceptance, commit and anchor readout */
 #define ASR_TL_GEMM 16         /* + epilogue: 0 plain, 1 QKV + cache append, 2 residual, 3 query, 4 GELU, 6 argmax */
-#define ASR_TL_LN_FUSED 32     /* added to a GEMM kind whose B operand is LayerNorm(x), normalised in the GEMM */
+#define ASR_TL_LN_FUSED 32     /* added to a GEMM kind whose input LayerNorm is folded into it (no LayerNorm launch) */
 int asr_spec_timeline(asr_spec_handle h, int32_t enable);
 int asr_spec_timeline_read(asr_spec_handle h, uint64_t* ns, int32_t* kind, int32_t cap, int32_t* count);
 

@@ -20,6 +20,9 @@ struct LayerW {
   void *wqkv, *wo, *wcq, *wco, *w1, *w2;
   float *bqkv, *bo, *bcq, *bco, *b1, *b2;
   float *ln1g, *ln1b, *ln2g, *ln2b, *ln3g, *ln3b;
+  // folded LayerNorm constants (c1 = W g, c2 = W b) of the three projections
+  // whose input is a LayerNorm output
+  float *c1_qkv = nullptr, *c2_qkv = nullptr, *c1_cq = nullptr, *c2_cq = nullptr, *c1_fc1 = nullptr, *c2_fc1 = nullptr;
   CUtensorMap m_wqkv, m_wo, m_wcq, m_wco, m_w1, m_w2;
 };
 
@@ -40,6 +43,7 @@ struct asr_spec {
   std::vector<void*> allocs;
   void *w_tok = nullptr, *w_pos = nullptr, *w_cross = nullptr;
   float *b_cross = nullptr, *lnf_g = nullptr, *lnf_b = nullptr;
+  float *c1_lm = nullptr, *c2_lm = nullptr;   // folded final LayerNorm of the LM head
   CUtensorMap m_tok{};
   std::vector<LayerW> lw;
 
@@ -75,12 +79,14 @@ struct asr_spec {
   // CUDA graphs of the verify body, keyed by (B, k)
   bool use_graphs = true;
   bool use_pdl = true;   // programmatic dependent launch between verify kernels
-  bool lm_ln_fused = false;   // the last verify's LM head normalised x itself (xf not written)
+  // LayerNorm folded into its neighbours (bf16, d % 128 == 0, N tiles <= 64):
+  // the producer of x writes bf16(g * x) into xn and slice statistics into
+  // ln_part; the consumer GEMM corrects its accumulators.  ln_S / ln_c: the
+  // slices of the last producer.
+  bool ln_fold = false;
+  float2* ln_part = nullptr;
+  int ln_S = 0, ln_c = 0;
   bool use_mc = false;        // multicast weight tiles across the row tiles (ASRSPEC_MC=1; slower as measured)
-  // GEMMs over at most this many rows normalise their own B operand
-  // (ASRSPEC_LN_FUSE_MAX, <= 64); off by default: a separate LayerNorm launch
-  // measured faster at batch 1 (1.99 vs 2.48 ms per large-decoder round)
-  int ln_fuse_max = 0;
   int wide_bn = 64;      // N tile for many rows (ASRSPEC_WIDE_BN: 64, 128, 192, 224, 256)
   int wide_target = 2 * 152;   // CTAs a many-row GEMM may fill by splitting K (ASRSPEC_WIDE_TARGET)
   // launch timeline (diagnostics): [ASR_TL_CAP][4] device slots, the kind of
@@ -92,6 +98,7 @@ struct asr_spec {
   struct Graph {
     cudaGraphExec_t exec;
     long long launches[ASR_PROF_N];
+    int ln_S, ln_c;   // the folded LayerNorm slices the captured body leaves (for debug_logits)
   };
   std::map<std::pair<int, int>, Graph> graphs;
 };
@@ -220,7 +227,6 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   }
   TcGemm g{};
   g.mapA = *mW;
-  g.mapB = *mW;   // unused when the B operand is LayerNorm(x) written by the kernel
   // Few rows (batch 1): one narrow N tile and K split across the CTAs of a
   // cluster so that every SM streams weights.  Many rows: 64-wide N tiles
   // (two CTAs per SM; measured best at batch 64 against 128 and 256), K split
@@ -230,11 +236,9 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   // for many rows: its weights are read half as often (measured 95 vs 116 us
   // at 448 rows)
   g.bn = N <= 64 ? tc_pick_bn(N) : (mode == EPI_ARGMAX ? 128 : h->wide_bn);
-  if (!epi.ln_x) {
-    const CUtensorMap* mb = bmap(h, x_id, X, h->R_pad, K, g.bn);
-    if (!mb) return fail(h, ASR_E_CUDA, "tensor map encode failed");
-    g.mapB = *mb;
-  }
+  const CUtensorMap* mb = bmap(h, x_id, X, h->R_pad, K, g.bn);
+  if (!mb) return fail(h, ASR_E_CUDA, "tensor map encode failed");
+  g.mapB = *mb;
   g.M = M;
   g.N = N;
   g.K = K;
@@ -250,27 +254,38 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   g.pdl = h->use_pdl;
   g.ws = h->ws;
   g.tickets = h->tickets;
-  Tl t(h, ASR_TL_GEMM + mode + (epi.ln_x ? ASR_TL_LN_FUSED : 0));
+  Tl t(h, ASR_TL_GEMM + mode + (epi.ln_part ? ASR_TL_LN_FUSED : 0));
   epi.tl = h->tl_cur;
   launch_gemm_tc(g, mode, epi, h->status, h->st);
+  if (epi.xg) {   // the slices the residual epilogue wrote statistics for
+    h->ln_c = g.splits > 1 ? 128 / g.splits : 128;
+    h->ln_S = M / h->ln_c;
+  }
   return 0;
 }
 
 enum BufId { BUF_XN = 1, BUF_ATT = 2, BUF_H = 3, BUF_XF = 4 };
 
-// A projection whose input is LayerNorm(x).  Few rows (bf16): the GEMM
-// normalises its own B tiles from x (no separate LayerNorm launch).  Otherwise
-// a LayerNorm kernel writes `ln_out` and the GEMM loads it by TMA.
+// Folded LayerNorm of a consumer GEMM: B = xn (bf16(g * x), written by the
+// producer of x) and the producer's slice statistics.
+void fold_consumer(asr_spec* h, Epi& e, const float* c1, const float* c2) {
+  e.ln_part = h->ln_part;
+  e.ln_S = h->ln_S;
+  e.ln_c = h->ln_c;
+  e.ln_stride = h->R_pad;
+  e.ln_c1 = c1;
+  e.ln_c2 = c2;
+}
+
+// A projection whose input is LayerNorm(x).  Folded (bf16): no LayerNorm
+// launch; the GEMM reads xn and corrects its accumulators.  Otherwise a
+// LayerNorm kernel writes `ln_out` and the GEMM loads it by TMA.
 int gemm_rows_ln(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, const float* g, const float* b,
-                 void* ln_out, int ln_out_id, int N, int mode, const Epi& epi_in, bool* fused = nullptr) {
+                 const float* c1, const float* c2, void* ln_out, int ln_out_id, int N, int mode, const Epi& epi_in) {
   Epi e = epi_in;
-  const bool fuse = h->bf16 && N <= std::min(h->ln_fuse_max, 64);
-  if (fused) *fused = fuse;
-  if (fuse) {
-    e.ln_x = h->x;
-    e.ln_g = g;
-    e.ln_b = b;
-    return gemm_rows(h, W, mW, M, K, nullptr, ln_out_id, N, mode, e);
+  if (h->ln_fold) {
+    fold_consumer(h, e, c1, c2);
+    return gemm_rows(h, W, mW, M, K, h->xn, BUF_XN, N, mode, e);
   }
   {
     Prof p(h, ASR_PROF_LAYERNORM, 1);
@@ -332,8 +347,23 @@ int run_layers(asr_spec* h, int N) {
   {
     Prof p(h, ASR_PROF_OTHER, 1);
     Tl t(h, ASR_TL_EMBED);
-    launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st, h->use_pdl, h->tl_cur);
+    if (h->ln_fold) {   // the first LayerNorm's operand and statistics (one slice of d features)
+      launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st, h->use_pdl, h->tl_cur,
+                   static_cast<__nv_bfloat16*>(h->xn), h->lw[0].ln1g, h->ln_part);
+      h->ln_S = 1;
+      h->ln_c = d;
+    } else {
+      launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st, h->use_pdl, h->tl_cur);
+    }
   }
+  // a residual projection that also produces the next LayerNorm's folded operand
+  auto producer = [&](Epi& e, const float* next_gain) {
+    if (!h->ln_fold) return;
+    e.xg = static_cast<__nv_bfloat16*>(h->xn);
+    e.xg_gain = next_gain;
+    e.st_part = h->ln_part;
+    e.st_stride = h->R_pad;
+  };
   for (int l = 0; l < h->L; ++l) {
     LayerW& w = h->lw[l];
     char* ks = static_cast<char*>(h->kself) + l * self_layer;
@@ -346,7 +376,8 @@ int run_layers(asr_spec* h, int N) {
     e.out_f32 = h->q;
     e.kcache = ks;
     e.vcache = vs;
-    if (int rc = gemm_rows_ln(h, w.wqkv, &w.m_wqkv, 3 * d, d, w.ln1g, w.ln1b, h->xn, BUF_XN, N, EPI_QKV, e))
+    if (int rc = gemm_rows_ln(h, w.wqkv, &w.m_wqkv, 3 * d, d, w.ln1g, w.ln1b, w.c1_qkv, w.c2_qkv, h->xn, BUF_XN, N,
+                              EPI_QKV, e))
       return rc;
     AttnArgs a{};
     a.q = h->q;
@@ -376,13 +407,15 @@ int run_layers(asr_spec* h, int N) {
     e = base;
     e.bias = w.bo;
     e.x = h->x;
+    producer(e, w.ln2g);
     if (int rc = gemm_rows(h, w.wo, &w.m_wo, d, d, h->att, BUF_ATT, N, EPI_RESID, e)) return rc;
     // cross-attention block
     float* qc = (l == h->anchor) ? h->q_anchor : h->q;
     e = base;
     e.bias = w.bcq;
     e.out_f32 = qc;
-    if (int rc = gemm_rows_ln(h, w.wcq, &w.m_wcq, d, d, w.ln2g, w.ln2b, h->xn, BUF_XN, N, EPI_Q, e)) return rc;
+    if (int rc = gemm_rows_ln(h, w.wcq, &w.m_wcq, d, d, w.ln2g, w.ln2b, w.c1_cq, w.c2_cq, h->xn, BUF_XN, N, EPI_Q, e))
+      return rc;
     a.q = qc;
     a.kc = kx;
     a.vc = vx;
@@ -397,15 +430,19 @@ int run_layers(asr_spec* h, int N) {
     e = base;
     e.bias = w.bco;
     e.x = h->x;
+    producer(e, w.ln3g);
     if (int rc = gemm_rows(h, w.wco, &w.m_wco, d, d, h->att, BUF_ATT, N, EPI_RESID, e)) return rc;
     // MLP block
     e = base;
     e.bias = w.b1;
     e.act = h->hbuf;
-    if (int rc = gemm_rows_ln(h, w.w1, &w.m_w1, h->F, d, w.ln3g, w.ln3b, h->xn, BUF_XN, N, EPI_GELU, e)) return rc;
+    if (int rc = gemm_rows_ln(h, w.w1, &w.m_w1, h->F, d, w.ln3g, w.ln3b, w.c1_fc1, w.c2_fc1, h->xn, BUF_XN, N, EPI_GELU,
+                              e))
+      return rc;
     e = base;
     e.bias = w.b2;
     e.x = h->x;
+    producer(e, l + 1 < h->L ? h->lw[l + 1].ln1g : h->lnf_g);
     if (int rc = gemm_rows(h, w.w2, &w.m_w2, d, h->F, h->hbuf, BUF_H, N, EPI_RESID, e)) return rc;
   }
   return 0;
@@ -445,8 +482,8 @@ int enqueue_verify(asr_spec* h, int k) {
   e.n_valid = h->plan.n_rows;
   e.row_key = h->row_key;
   e.d = h->d;
-  if (int rc = gemm_rows_ln(h, h->w_tok, &h->m_tok, h->V, h->d, h->lnf_g, h->lnf_b, h->xf, BUF_XF, N, EPI_ARGMAX, e,
-                            &h->lm_ln_fused))
+  if (int rc = gemm_rows_ln(h, h->w_tok, &h->m_tok, h->V, h->d, h->lnf_g, h->lnf_b, h->c1_lm, h->c2_lm, h->xf, BUF_XF,
+                            N, EPI_ARGMAX, e))
     return rc;
   Prof p(h, ASR_PROF_OTHER, 1);
   AcceptAnchorArgs A{};
@@ -503,13 +540,14 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   h->bf16 = dims->dtype == 1;
   if (const char* e = std::getenv("ASRSPEC_PDL")) h->use_pdl = std::atoi(e) != 0;
   if (const char* e = std::getenv("ASRSPEC_MC")) h->use_mc = std::atoi(e) != 0;
-  if (const char* e = std::getenv("ASRSPEC_LN_FUSE_MAX")) h->ln_fuse_max = std::atoi(e);
   if (const char* e = std::getenv("ASRSPEC_WIDE_BN")) {
     const int v = std::atoi(e);
     if (v == 64 || v == 128 || v == 192 || v == 224 || v == 256) h->wide_bn = v;
   }
   if (const char* e = std::getenv("ASRSPEC_WIDE_TARGET")) h->wide_target = std::max(1, std::atoi(e));
   h->es = h->bf16 ? 2 : 4;
+  h->ln_fold = h->bf16 && h->d % 128 == 0 && h->wide_bn <= 64;
+  if (const char* e = std::getenv("ASRSPEC_LN_FOLD")) h->ln_fold = h->ln_fold && std::atoi(e) != 0;
   h->st = static_cast<cudaStream_t>(stream);
   if (!h->st) {
     // A blocking stream of our own: ordered with the legacy default stream,
@@ -624,6 +662,23 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   if ((rc = dalloc(h, &h->lnf_b, d * 4)) || (rc = upload_f32(h, h->lnf_b, lnfb, d))) return finish(rc);
   if (h->bf16 && !make_tmap_bf16(&h->m_tok, h->w_tok, h->V, d, 128))
     return finish(fail(h, ASR_E_CUDA, "tensor map encode failed"));
+  if (h->ln_fold) {
+    auto fold = [&](const void* W, const float* g, const float* b, int M, float** c1, float** c2) {
+      int r = dalloc(h, c1, (size_t)M * 4);
+      if (!r) r = dalloc(h, c2, (size_t)M * 4);
+      if (!r) launch_ln_fold(W, g, b, M, d, *c1, *c2, h->st);
+      return r;
+    };
+    for (int l = 0; l < L; ++l) {
+      LayerW& w = h->lw[l];
+      if ((rc = fold(w.wqkv, w.ln1g, w.ln1b, 3 * d, &w.c1_qkv, &w.c2_qkv)) ||
+          (rc = fold(w.wcq, w.ln2g, w.ln2b, d, &w.c1_cq, &w.c2_cq)) ||
+          (rc = fold(w.w1, w.ln3g, w.ln3b, F, &w.c1_fc1, &w.c2_fc1)))
+        return finish(rc);
+    }
+    if ((rc = fold(h->w_tok, h->lnf_g, h->lnf_b, h->V, &h->c1_lm, &h->c2_lm))) return finish(rc);
+    CK(cudaGetLastError());
+  }
 
   // caches
   const size_t self_bytes = (size_t)L * h->Bmax * h->H * h->maxpos * 64 * es;
@@ -652,6 +707,10 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   CK(cudaMemset(h->att, 0, R * d * es));
   CK(cudaMemset(h->hbuf, 0, R * F * es));
   CK(cudaMemset(h->xf, 0, R * d * es));
+  if (h->ln_fold) {   // slices of at least 8 features
+    if ((rc = dalloc(h, &h->ln_part, (size_t)(d / 8) * R * sizeof(float2)))) return finish(rc);
+    CK(cudaMemset(h->ln_part, 0, (size_t)(d / 8) * R * sizeof(float2)));
+  }
   const int chunk = h->bf16 ? 128 : attn_chunk_len(0);   // the finest split either path uses
   const int n_chunks = (std::max(h->maxpos, h->Tmax) + chunk - 1) / chunk;
   if ((rc = dalloc(h, &h->part, (size_t)h->Bmax * h->H * n_chunks * (h->kmax + 1) * 66 * 4))) return finish(rc);
@@ -804,9 +863,13 @@ int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens
       cudaGraphDestroy(graph);
       if (e != cudaSuccess) return fail(h, ASR_E_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(e));
       for (int c = 0; c < ASR_PROF_N; ++c) g.launches[c] = h->cur[c];
+      g.ln_S = h->ln_S;
+      g.ln_c = h->ln_c;
       it = h->graphs.emplace(key, g).first;
     }
     CK(cudaGraphLaunch(it->second.exec, h->st));
+    h->ln_S = it->second.ln_S;
+    h->ln_c = it->second.ln_c;
     for (int c = 0; c < ASR_PROF_N; ++c) h->launches[c] += it->second.launches[c];
   } else {
     if (int rc = enqueue_verify(h, k)) return rc;
@@ -931,12 +994,13 @@ int asr_spec_debug_logits(asr_spec_handle h, float* out, int32_t max_rows) {
   e.out_f32 = dst;
   e.ld = h->V;
   e.n_valid = h->plan.n_rows;
-  if (h->lm_ln_fused && h->bf16) {   // same B operand as the fused argmax: LayerNorm(x) built in the GEMM
-    e.ln_x = h->x;
-    e.ln_g = h->lnf_g;
-    e.ln_b = h->lnf_b;
+  int rc;
+  if (h->ln_fold) {   // the same operand and statistics as the last verify's LM head
+    fold_consumer(h, e, h->c1_lm, h->c2_lm);
+    rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xn, BUF_XN, R, EPI_F32, e);
+  } else {
+    rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, R, EPI_F32, e);
   }
-  int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, R, EPI_F32, e);
   if (!rc && h->host_io) {
     CK(cudaMemcpyAsync(out, tmp, (size_t)R * h->V * 4, cudaMemcpyDeviceToHost, h->st));
   }

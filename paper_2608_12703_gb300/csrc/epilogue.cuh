@@ -48,10 +48,20 @@ struct Epi {
   int b_max = 0;
   // LM head argmax
   unsigned long long* row_key = nullptr;
-  // B operand = LayerNorm(ln_x) (few-row GEMMs): fp32 rows [N][K], gain and bias [K]
-  const float* ln_x = nullptr;
-  const float* ln_g = nullptr;
-  const float* ln_b = nullptr;
+  // LayerNorm folded into the GEMM (consumer).  The B operand is bf16(g * x)
+  // and y = rstd_n (acc - mu_n c1_m) + c2_m (+ bias), with c1 = W g, c2 = W b
+  // and the row statistics combined from ln_S slices of ln_c features each:
+  // ln_part[s * ln_stride + n] = (slice mean, slice sum of squared deviations).
+  const float2* ln_part = nullptr;
+  int ln_S = 0, ln_c = 0, ln_stride = 0;
+  const float* ln_c1 = nullptr;
+  const float* ln_c2 = nullptr;
+  // Producer of the next folded LayerNorm (EPI_RESID): writes xg = bf16(g * x)
+  // [n][d] and its slice statistics st_part[slice * st_stride + n].
+  __nv_bfloat16* xg = nullptr;
+  const float* xg_gain = nullptr;
+  float2* st_part = nullptr;
+  int st_stride = 0;
   // launch timeline slot (see tl_mark), or null
   unsigned long long* tl = nullptr;
   // optional phase timestamps (ns, %globaltimer) per CTA: [CTA][8]
@@ -121,6 +131,8 @@ struct EpiPre {
   float bias[U];
   float old[U];   // EPI_RESID: x before the update
   int rb[U], rp[U];   // EPI_QKV: utterance and position of the row
+  float c1[U], c2[U];   // folded LayerNorm (consumer)
+  float gain[U];        // next LayerNorm's gain (EPI_RESID producer)
 };
 
 template <int MODE, int U>
@@ -135,6 +147,11 @@ __device__ __forceinline__ void epi_load(const Epi& e, const int* m, const int* 
       p.rb[u] = ok[u] && m[u] >= e.d ? e.row_b[n[u]] : 0;
       p.rp[u] = ok[u] && m[u] >= e.d ? e.row_pos[n[u]] : 0;
     }
+    if constexpr (MODE != EPI_RESID && MODE != EPI_CROSSKV) {
+      p.c1[u] = ok[u] && e.ln_part ? __ldg(e.ln_c1 + m[u]) : 0.f;
+      p.c2[u] = ok[u] && e.ln_part ? __ldg(e.ln_c2 + m[u]) : 0.f;
+    }
+    if constexpr (MODE == EPI_RESID) p.gain[u] = ok[u] && e.xg ? __ldg(e.xg_gain + m[u]) : 0.f;
   }
 }
 
@@ -191,13 +208,25 @@ __host__ __device__ constexpr bool rowwise_mode() {
   return MODE == EPI_F32 || MODE == EPI_Q || MODE == EPI_RESID || MODE == EPI_GELU || MODE == EPI_QKV;
 }
 
+// ln_mu / ln_rs: the folded LayerNorm's row statistics of the tile's rows
+// (shared memory, indexed by local row), used when e.ln_part is set.  A
+// residual producer (e.xg set) also writes bf16(g * x) and the statistics of
+// the warp's 128 features (slice m0 / 128) of each row.
 template <int MODE>
 __device__ __forceinline__ void epi_rows(const Epi& e, const float* stg, int lds, int mq, int m_local, int n0,
-                                         int warp, int rows) {
+                                         int warp, int rows, const float* ln_mu, const float* ln_rs) {
   const bool mok = mq < e.M;
   float4 bias = make_float4(0.f, 0.f, 0.f, 0.f);
   if constexpr (MODE != EPI_F32)
     if (mok) bias = __ldg(reinterpret_cast<const float4*>(e.bias + mq));
+  const bool fold = e.ln_part != nullptr && MODE != EPI_RESID;
+  float4 c1 = make_float4(0.f, 0.f, 0.f, 0.f), c2 = c1, gain = c1;
+  if (fold && mok) {
+    c1 = __ldg(reinterpret_cast<const float4*>(e.ln_c1 + mq));
+    c2 = __ldg(reinterpret_cast<const float4*>(e.ln_c2 + mq));
+  }
+  if constexpr (MODE == EPI_RESID)
+    if (e.xg && mok) gain = __ldg(reinterpret_cast<const float4*>(e.xg_gain + mq));
   int kind = 0, head = 0, c = 0;   // EPI_QKV: 0 query, 1 key, 2 value
   if constexpr (MODE == EPI_QKV) {
     if (mq >= e.d) {
@@ -231,6 +260,11 @@ __device__ __forceinline__ void epi_rows(const Epi& e, const float* stg, int lds
       if (!ok[r]) continue;
       const int n = n0 + j0 + 4 * r;
       float4 v = a[r];
+      if (fold) {   // y = rstd (acc - mu c1) + c2
+        const float mu = ln_mu[j0 + 4 * r], rs = ln_rs[j0 + 4 * r];
+        v = make_float4(rs * (v.x - mu * c1.x) + c2.x, rs * (v.y - mu * c1.y) + c2.y, rs * (v.z - mu * c1.z) + c2.z,
+                        rs * (v.w - mu * c1.w) + c2.w);
+      }
       if constexpr (MODE == EPI_F32) {
         float* o = e.out_f32 + (size_t)n * e.ld;
         if (mq + 0 < e.M) o[mq + 0] = v.x;
@@ -244,7 +278,18 @@ __device__ __forceinline__ void epi_rows(const Epi& e, const float* stg, int lds
         *reinterpret_cast<float4*>(e.out_f32 + (size_t)n * e.d + mq) = v;
       } else if constexpr (MODE == EPI_RESID) {
         const float4 o = old[r];
-        *reinterpret_cast<float4*>(e.x + (size_t)n * e.d + mq) = make_float4(o.x + v.x, o.y + v.y, o.z + v.z, o.w + v.w);
+        const float4 xn = make_float4(o.x + v.x, o.y + v.y, o.z + v.z, o.w + v.w);
+        *reinterpret_cast<float4*>(e.x + (size_t)n * e.d + mq) = xn;
+        if (e.xg) {   // the next LayerNorm's operand and this slice's statistics (uniform over the warp)
+          __nv_bfloat162 lo = __floats2bfloat162_rn(gain.x * xn.x, gain.y * xn.y);
+          __nv_bfloat162 hi = __floats2bfloat162_rn(gain.z * xn.z, gain.w * xn.w);
+          *reinterpret_cast<uint2*>(e.xg + (size_t)n * e.d + mq) =
+              make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
+          const float mean = warp_sum((xn.x + xn.y) + (xn.z + xn.w)) * (1.f / 128.f);
+          const float dx = xn.x - mean, dy = xn.y - mean, dz = xn.z - mean, dw = xn.w - mean;
+          const float m2 = warp_sum((dx * dx + dy * dy) + (dz * dz + dw * dw));
+          if ((threadIdx.x & 31) == 0) e.st_part[(size_t)(mq / 128) * e.st_stride + n] = make_float2(mean, m2);
+        }
       } else if constexpr (MODE == EPI_GELU) {
         v = make_float4(gelu_erf(v.x), gelu_erf(v.y), gelu_erf(v.z), gelu_erf(v.w));
         const size_t idx = (size_t)n * e.M + mq;

@@ -53,15 +53,12 @@ struct TcCfg {
   static_assert(B_BYTES % 1024 == 0, "B tile must keep 1024-byte alignment");
 };
 
-// Named barrier of the two B-writer warps (warps 2 and 3) of the LayerNorm path.
-__device__ __forceinline__ void writers_sync() { asm volatile("bar.sync 1, 64;" ::: "memory"); }
-__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 // MC: the N tiles of one M tile form a cluster (grid y = cluster y); each
 // k-block's A tile is loaded once, by CTA (k-block mod cluster size), and
 // multicast to every CTA of the cluster; an MMA commit frees the slot in all
 // of them, so a slot is refilled only after every CTA has consumed it.
-template <int BN, int MODE, bool CLU, bool LNB, bool MC>
+template <int BN, int MODE, bool CLU, bool MC>
 __global__ void __launch_bounds__(128, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, int K, int splits,
                float* __restrict__ ws, int* __restrict__ tickets, Epi epi, int* status) {
@@ -79,7 +76,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   float* recv = reinterpret_cast<float*>(smem + C::RECV_OFF);
   __shared__ unsigned long long red[4][BN];
   __shared__ int s_last;
-  __shared__ float ln_mean[LNB ? BN : 1], ln_rstd[LNB ? BN : 1];
+  __shared__ float ln_mu[BN], ln_rs[BN];   // folded LayerNorm: statistics of the tile's rows
 
   // Grid: cluster split: (M tiles x splits, N tiles), the splits of a tile
   // consecutive along x (one cluster); multicast: (M tiles, N tiles), the N
@@ -115,7 +112,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   }
   if (threadIdx.x == 32) {
     for (int s = 0; s < C::STAGES; ++s) {
-      mbar_init(&full[s], LNB ? 2 : 1);   // LayerNorm path: TMA (A) + the B writers
+      mbar_init(&full[s], 1);
       mbar_init(&empty[s], MC ? mc_size : 1);
     }
     mbar_init(done, 1);
@@ -141,7 +138,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     tma_prefetch_desc(&mapB);
     // The weights (A) do not depend on the previous kernel: fill the ring with
     // them first, then wait for the predecessor before loading activations (B).
-    constexpr uint32_t TX = LNB ? C::A_BYTES : C::STAGE_BYTES;
+    constexpr uint32_t TX = C::STAGE_BYTES;
     const int first = nkb < C::STAGES ? nkb : C::STAGES;
     for (int i = 0; i < first; ++i) {
       mbar_arrive_expect_tx(&full[i], TX);
@@ -154,8 +151,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     }
     pdl_wait();
     tl_mark(epi.tl, TL_WORK);
-    if constexpr (!LNB)
-      for (int i = 0; i < first; ++i) tma_load_2d(sB + i * C::B_BYTES, &mapB, &full[i], (kb0 + i) * TC_BK, n0);
+    for (int i = 0; i < first; ++i) tma_load_2d(sB + i * C::B_BYTES, &mapB, &full[i], (kb0 + i) * TC_BK, n0);
     pdl_launch();
     int issued = first;
     for (int i = first; i < nkb; ++i) {
@@ -169,7 +165,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       } else {
         tma_load_2d(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0);
       }
-      if constexpr (!LNB) tma_load_2d(sB + s * C::B_BYTES, &mapB, &full[s], (kb0 + i) * TC_BK, n0);
+      tma_load_2d(sB + s * C::B_BYTES, &mapB, &full[s], (kb0 + i) * TC_BK, n0);
       issued = i + 1;
     }
     // Drain: every issued copy has landed before this CTA can exit.
@@ -193,88 +189,51 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       else umma_commit(&empty[s]);
     }
     umma_commit(done);
-  } else if (LNB && warp >= 2) {
-    // B = bf16(LayerNorm(x)) rows n0 .. n0 + BN - 1, written straight into the
-    // 128-byte-swizzled K-major tile the MMA reads.  Statistics first: one pass
-    // of shifted sums per row (shift = the row's first element).
-    pdl_wait();
-    pdl_launch();
-    const int t = threadIdx.x - 64;
-    // four rows at a time per warp, all their loads in flight together
-    for (int rb = warp - 2; rb < BN; rb += 8) {
-      constexpr int RI = 4;
-      const float4* x4[RI];
-      float sh[RI], s1[RI], s2[RI];
-      bool ok[RI];
-#pragma unroll
-      for (int j = 0; j < RI; ++j) {
-        const int r = rb + 2 * j, n = n0 + r;
-        ok[j] = r < BN && n < n_valid;
-        const float* xr = epi.ln_x + (size_t)(ok[j] ? n : 0) * K;
-        x4[j] = reinterpret_cast<const float4*>(xr);
-        sh[j] = ok[j] ? __ldg(xr) : 0.f;
-        s1[j] = s2[j] = 0.f;
-      }
-      for (int i = lane; i < K / 4; i += 32) {
-#pragma unroll
-        for (int j = 0; j < RI; ++j) {
-          if (!ok[j]) continue;
-          const float4 v = x4[j][i];
-          const float a = v.x - sh[j], b = v.y - sh[j], c = v.z - sh[j], e = v.w - sh[j];
-          s1[j] += (a + b) + (c + e);
-          s2[j] += (a * a + b * b) + (c * c + e * e);
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < RI; ++j) {
-        const int r = rb + 2 * j;
-        const float a1 = warp_sum(s1[j]), a2 = warp_sum(s2[j]);
-        const float m1 = a1 / (float)K;
-        if (lane == 0 && r < BN) {
-          ln_mean[r] = ok[j] ? sh[j] + m1 : 0.f;
-          ln_rstd[r] = ok[j] ? rsqrtf(fmaxf(a2 / (float)K - m1 * m1, 0.f) + 1e-5f) : 0.f;
-        }
-      }
-    }
-    writers_sync();
-    for (int i = 0; i < nkb; ++i) {
-      const int s = i % C::STAGES;
-      const uint32_t ph = (i / C::STAGES) & 1;
-      if (!mbar_wait(&empty[s], ph ^ 1, status)) break;
-      const int k0 = (kb0 + i) * TC_BK;
-      uint8_t* bt = sB + s * C::B_BYTES;
-      for (int id = t; id < BN * 4; id += 64) {      // BN rows x 4 runs of 16 columns
-        const int r = id >> 2, c0 = (id & 3) * 16, n = n0 + r;
-        uint32_t w[8];
-        if (n < n_valid) {
-          const float4* x4 = reinterpret_cast<const float4*>(epi.ln_x + (size_t)n * K + k0 + c0);
-          const float4* g4 = reinterpret_cast<const float4*>(epi.ln_g + k0 + c0);
-          const float4* b4 = reinterpret_cast<const float4*>(epi.ln_b + k0 + c0);
-          const float mu = ln_mean[r], rs = ln_rstd[r];
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const float4 v = x4[q], gg = __ldg(g4 + q), bb = __ldg(b4 + q);
-            __nv_bfloat162 lo = __floats2bfloat162_rn((v.x - mu) * rs * gg.x + bb.x, (v.y - mu) * rs * gg.y + bb.y);
-            __nv_bfloat162 hi = __floats2bfloat162_rn((v.z - mu) * rs * gg.z + bb.z, (v.w - mu) * rs * gg.w + bb.w);
-            w[2 * q] = *reinterpret_cast<uint32_t*>(&lo);
-            w[2 * q + 1] = *reinterpret_cast<uint32_t*>(&hi);
-          }
-        } else {
-#pragma unroll
-          for (int q = 0; q < 8; ++q) w[q] = 0u;
-        }
-        const int ch = c0 >> 3;   // first 16-byte chunk of this run
-        *reinterpret_cast<uint4*>(bt + r * 128 + (((ch) ^ (r & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
-        *reinterpret_cast<uint4*>(bt + r * 128 + (((ch + 1) ^ (r & 7)) << 4)) = make_uint4(w[4], w[5], w[6], w[7]);
-      }
-      fence_async_smem();   // make the generic-proxy writes visible to the tensor core
-      writers_sync();
-      if (t == 0) mbar_arrive(&full[s]);
-    }
   }
-  if (!(warp == 0 && lane == 0) && !(LNB && warp >= 2)) {
+  if (!(warp == 0 && lane == 0)) {
     pdl_wait();
     pdl_launch();
+  }
+  // Folded LayerNorm: warps 2-3 (idle during the main loop) combine the row
+  // statistics of the tile's rows from the producer's slices (equal slice
+  // sizes: mean = average of slice means, M2 = sum of slice M2 + c * sum of
+  // squared deviations of the slice means), 64 / BN threads per row.
+  if (epi.ln_part != nullptr && warp >= 2) {
+    const int t = threadIdx.x - 64;
+    constexpr int TPR = BN >= 64 ? 1 : 64 / BN;   // threads per row (a power of two)
+    const int S = epi.ln_S;
+    for (int rl = t / TPR; rl < BN; rl += 64 / TPR) {
+      const int n = n0 + rl;
+      const int sub = t % TPR;
+      const bool ok = n < n_valid;
+      const float2* pr = epi.ln_part + (ok ? n : 0);
+      // one pass, shifted by the first slice's mean (well conditioned when the
+      // slice means are close to the row mean): with e_s = mean_s - shift,
+      // mean = shift + E/S and M2 = sum M2_s + c (sum e_s^2 - E^2 / S)
+      const float shift = ok ? pr[0].x : 0.f;
+      float e1 = 0.f, e2 = 0.f, m2 = 0.f;
+      if (ok)
+#pragma unroll 8
+        for (int j = sub; j < S; j += TPR) {
+          const float2 p = pr[(size_t)j * epi.ln_stride];
+          const float es = p.x - shift;
+          e1 += es;
+          e2 += es * es;
+          m2 += p.y;
+        }
+#pragma unroll
+      for (int o = TPR / 2; o > 0; o >>= 1) {
+        e1 += __shfl_xor_sync(0xffffffffu, e1, o);
+        e2 += __shfl_xor_sync(0xffffffffu, e2, o);
+        m2 += __shfl_xor_sync(0xffffffffu, m2, o);
+      }
+      const float mean = shift + e1 / (float)S;
+      const float q = m2 + (float)epi.ln_c * fmaxf(e2 - e1 * e1 / (float)S, 0.f);
+      if (sub == 0) {
+        ln_mu[rl] = ok ? mean : 0.f;
+        ln_rs[rl] = ok ? rsqrtf(q / (float)(S * epi.ln_c) + 1e-5f) : 0.f;
+      }
+    }
   }
   // Push split: this thread's first-pass outputs of the owner's slice, and
   // their other operands (bias, residual, row metadata) loaded now, while the
@@ -329,12 +288,25 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     }
     __syncthreads();
     const int rows = n_valid - n0 < BN ? n_valid - n0 : BN;
-    epi_rows<MODE>(epi, stg, LDS, m0 + 4 * lane, 4 * lane, n0, warp, rows);
+    epi_rows<MODE>(epi, stg, LDS, m0 + 4 * lane, 4 * lane, n0, warp, rows, ln_mu, ln_rs);
   } else if (splits == 1) {
+    const bool fold = epi.ln_part != nullptr && MODE != EPI_CROSSKV;
+    float c1m = 0.f, c2m = 0.f;
+    if (fold) {
+      __syncthreads();   // the row statistics of warps 2-3
+      if (m < epi.M) {
+        c1m = __ldg(epi.ln_c1 + m);
+        c2m = __ldg(epi.ln_c2 + m);
+      }
+    }
 #pragma unroll 1
     for (int c0 = 0; c0 < BN; c0 += 16) {
       float v[16];
       tmem_ld16(t_lane + c0, v);
+      if (fold) {   // y = rstd (acc - mu c1) + c2
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = ln_rs[c0 + i] * (v[i] - ln_mu[c0 + i] * c1m) + c2m;
+      }
       if constexpr (MODE == EPI_ARGMAX) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -413,8 +385,56 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
         vals[4 * u + 2] = acc.z;
         vals[4 * u + 3] = acc.w;
       }
-      if (base == (int)threadIdx.x) epi_store<EM, 4 * IU>(epi, mm, nn, vals, ok, pre);
-      else epi_batch<EM, 4 * IU>(epi, mm, nn, vals, ok);
+      // the first pass's operands were loaded during the main loop; later passes load theirs now
+      if (base != (int)threadIdx.x) epi_load<EM, 4 * IU>(epi, mm, nn, ok, pre);
+      const EpiPre<EM, 4 * IU>& op = pre;
+      if constexpr (EM != EPI_RESID) {
+        if (epi.ln_part != nullptr) {   // folded LayerNorm: y = rstd (acc - mu c1) + c2
+#pragma unroll
+          for (int k = 0; k < 4 * IU; ++k) {
+            if (!ok[k]) continue;
+            const int nl = nn[k] - n0;
+            vals[k] = ln_rs[nl] * (vals[k] - ln_mu[nl] * op.c1[k]) + op.c2[k];
+          }
+        }
+      }
+      epi_store<EM, 4 * IU>(epi, mm, nn, vals, ok, op);
+      if constexpr (EM == EPI_RESID) {
+        if (epi.xg != nullptr) {
+          // the next LayerNorm's operand bf16(g * x), and x staged as [feature
+          // of the slice][row] in the pipeline buffers (free since the MMAs
+          // retired) for the slice statistics below
+          float* xt = reinterpret_cast<float*>(smem);
+#pragma unroll
+          for (int k = 0; k < 4 * IU; ++k) {
+            if (!ok[k]) continue;
+            const float xn = op.old[k] + (vals[k] + op.bias[k]);   // the value just stored
+            epi.xg[(size_t)nn[k] * epi.d + mm[k]] = __float2bfloat16_rn(op.gain[k] * xn);
+            xt[(mm[k] - m0 - r_first) * (BN + 4) + (nn[k] - n0)] = xn;
+          }
+        }
+      }
+    }
+    if constexpr (EM == EPI_RESID) {
+      if (epi.xg != nullptr) {
+        // Statistics of this owner's slice (rows_per features) of every row:
+        // one thread per row sums its column of the staged tile.
+        const float* xt = reinterpret_cast<const float*>(smem);
+        __syncthreads();
+        for (int c = threadIdx.x; c < BN; c += blockDim.x) {
+          const int n = n0 + c;
+          if (n >= n_valid) continue;
+          float sm = 0.f;
+          for (int r = 0; r < rows_per; ++r) sm += xt[r * (BN + 4) + c];
+          const float mean = sm / (float)rows_per;
+          float q = 0.f;
+          for (int r = 0; r < rows_per; ++r) {
+            const float dv = xt[r * (BN + 4) + c] - mean;
+            q += dv * dv;
+          }
+          epi.st_part[(size_t)((m0 + r_first) / rows_per) * epi.st_stride + n] = make_float2(mean, q);
+        }
+      }
     }
     if (tr && threadIdx.x == 0) tr[7] = global_ns();
   } else if constexpr (CLU) {
@@ -629,47 +649,29 @@ int tc_pick_bn_wide(int n) {
   return best;
 }
 
-// LayerNorm-fused B operand exists for the few-row tiles (BN <= 64) of the
-// modes whose input is a LayerNorm output.
-template <int BN, int MODE>
-constexpr bool ln_capable() {
-  return BN <= 64 && (MODE == EPI_QKV || MODE == EPI_Q || MODE == EPI_GELU || MODE == EPI_ARGMAX || MODE == EPI_F32);
-}
-
 template <int BN>
 constexpr bool mc_capable() {
   return BN == 64 || BN == 128;
 }
 
-template <int BN, int MODE, bool LNB>
-static void launch_tc_ln(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
+template <int BN, int MODE>
+static void launch_tc_t(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
   const int mt = (g.M + TC_BM - 1) / TC_BM, nt = (g.N + BN - 1) / BN;
   if (g.cluster && g.splits > 1) {
-    launch_ex(gemm_tc_kernel<BN, MODE, true, LNB, false>, dim3(mt * g.splits, nt, 1), dim3(128),
+    launch_ex(gemm_tc_kernel<BN, MODE, true, false>, dim3(mt * g.splits, nt, 1), dim3(128),
               TcCfg<BN, (BN <= 64)>::SMEM, st, g.pdl, g.splits, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi,
               status);
     return;
   }
-  if constexpr (!LNB && mc_capable<BN>()) {
+  if constexpr (mc_capable<BN>()) {
     if (g.mc && g.splits == 1 && nt >= 2 && nt <= 8) {
-      launch_ex2(gemm_tc_kernel<BN, MODE, false, false, true>, dim3(mt, nt, 1), dim3(128), TcCfg<BN>::SMEM, st,
-                 g.pdl, 1, nt, g.mapA, g.mapB, g.K, 1, g.ws, g.tickets, epi, status);
+      launch_ex2(gemm_tc_kernel<BN, MODE, false, true>, dim3(mt, nt, 1), dim3(128), TcCfg<BN>::SMEM, st, g.pdl, 1,
+                 nt, g.mapA, g.mapB, g.K, 1, g.ws, g.tickets, epi, status);
       return;
     }
   }
-  launch_ex(gemm_tc_kernel<BN, MODE, false, LNB, false>, dim3(nt, mt, g.splits), dim3(128), TcCfg<BN>::SMEM, st,
-            g.pdl, 1, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
-}
-
-template <int BN, int MODE>
-static void launch_tc_t(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
-  if constexpr (ln_capable<BN, MODE>()) {
-    if (epi.ln_x) {
-      launch_tc_ln<BN, MODE, true>(g, epi, status, st);
-      return;
-    }
-  }
-  launch_tc_ln<BN, MODE, false>(g, epi, status, st);
+  launch_ex(gemm_tc_kernel<BN, MODE, false, false>, dim3(nt, mt, g.splits), dim3(128), TcCfg<BN>::SMEM, st, g.pdl,
+            1, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
 }
 
 template <int MODE>
@@ -685,22 +687,16 @@ static void launch_tc_mode(const TcGemm& g, const Epi& epi, int* status, cudaStr
   }
 }
 
-template <int BN, int MODE, bool LNB>
-static void configure_ln() {
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, LNB, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       TcCfg<BN>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, LNB, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       TcCfg<BN, (BN <= 64)>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, LNB, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if constexpr (!LNB && mc_capable<BN>())
-    cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         TcCfg<BN>::SMEM);
-}
-
 template <int BN, int MODE>
 static void configure_one() {
-  configure_ln<BN, MODE, false>();
-  if constexpr (ln_capable<BN, MODE>()) configure_ln<BN, MODE, true>();
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       TcCfg<BN>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       TcCfg<BN, (BN <= 64)>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if constexpr (mc_capable<BN>())
+    cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         TcCfg<BN>::SMEM);
 }
 
 template <int MODE>

@@ -64,8 +64,14 @@ void launch_plan_verify(const int* draft, const int* lens, int k, int B, int voc
                         int* status, const TrafficArgs& tr, cudaStream_t st, unsigned long long* tl = nullptr);
 void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,
                                RowPlan plan, int* status, cudaStream_t st);
+// xg / gain / st_part: the folded first LayerNorm's operand bf16(gain * x) [R][d]
+// and the rows' statistics (one slice of d features), or null.
 void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
-                  cudaStream_t st, bool pdl = false, unsigned long long* tl = nullptr);
+                  cudaStream_t st, bool pdl = false, unsigned long long* tl = nullptr, __nv_bfloat16* xg = nullptr,
+                  const float* gain = nullptr, float2* st_part = nullptr);
+// c1[m] = sum_k W[m][k] g[k], c2[m] = sum_k W[m][k] b[k] for a bf16 W [M][K].
+void launch_ln_fold(const void* W, const float* g, const float* b, int M, int K, float* c1, float* c2,
+                    cudaStream_t st);
 // y = LN(x) * g + b over rows < n_rows, written as bf16 or fp32.
 void launch_layernorm(const float* x, const float* g, const float* b, void* y, int y_bf16, const int* n_rows,
                       int R_max, int d, cudaStream_t st, bool pdl = false, unsigned long long* tl = nullptr);

@@ -158,30 +158,94 @@ void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, 
   plan_prefill_kernel<<<1, PLAN_THREADS, 0, st>>>(prompt, P0, p0, c, B, vocab, ready, plan, status);
 }
 
-// x[r] = tok_emb[token] + pos_emb[position]  (fp32 residual stream)
+// x[r] = tok_emb[token] + pos_emb[position]  (fp32 residual stream).  With a
+// folded first LayerNorm (xg set) also bf16(g * x) and the row's statistics as
+// one slice of d features: st_part[r] = (mean, sum of squared deviations).
+// One CTA of 128 threads per row (d <= 2048: 16 values per thread).
 template <typename T>
-__global__ void embed_kernel(const T* __restrict__ tok_emb, const T* __restrict__ pos_emb, RowPlan plan, int d,
-                             float* __restrict__ x, unsigned long long* tl) {
+__global__ void __launch_bounds__(128)
+embed_kernel(const T* __restrict__ tok_emb, const T* __restrict__ pos_emb, RowPlan plan, int d,
+             float* __restrict__ x, __nv_bfloat16* __restrict__ xg, const float* __restrict__ gain,
+             float2* __restrict__ st_part, unsigned long long* tl) {
+  __shared__ float red[4];
   tl_mark(tl, TL_ENTRY);
   pdl_wait();
   tl_mark(tl, TL_WORK);
   pdl_launch();
   const int r = blockIdx.x;
-  if (r >= *plan.n_rows) return;
+  if (r >= *plan.n_rows) return;   // uniform over the CTA
   const int t = plan.row_tok[r], p = plan.row_pos[r];
-  for (int c = threadIdx.x; c < d; c += blockDim.x)
-    x[(size_t)r * d + c] = to_f<T>(tok_emb[(size_t)t * d + c]) + to_f<T>(pos_emb[(size_t)p * d + c]);
+  float v[16];
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const int c = threadIdx.x + 128 * i;
+    v[i] = c < d ? to_f<T>(tok_emb[(size_t)t * d + c]) + to_f<T>(pos_emb[(size_t)p * d + c]) : 0.f;
+    if (c < d) x[(size_t)r * d + c] = v[i];
+    s += v[i];
+  }
+  if (xg != nullptr) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    s = warp_sum(s);
+    if (lane == 0) red[warp] = s;
+    __syncthreads();
+    const float mean = ((red[0] + red[1]) + (red[2] + red[3])) / (float)d;
+    __syncthreads();
+    float q = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int c = threadIdx.x + 128 * i;
+      if (c < d) {
+        const float dv = v[i] - mean;
+        q += dv * dv;
+        xg[(size_t)r * d + c] = __float2bfloat16_rn(gain[c] * v[i]);
+      }
+    }
+    q = warp_sum(q);
+    if (lane == 0) red[warp] = q;
+    __syncthreads();
+    if (threadIdx.x == 0) st_part[r] = make_float2(mean, (red[0] + red[1]) + (red[2] + red[3]));
+  }
   tl_mark(tl, TL_EXIT);
 }
 
+// Folded-LayerNorm constants of a projection W [M][K] (bf16) whose input is
+// LayerNorm(x) with gain g and bias b: c1[m] = sum_k W[m][k] g[k],
+// c2[m] = sum_k W[m][k] b[k].  One warp per row, fp32 sums.
+__global__ void __launch_bounds__(256)
+ln_fold_kernel(const __nv_bfloat16* __restrict__ W, const float* __restrict__ g, const float* __restrict__ b, int M,
+               int K, float* __restrict__ c1, float* __restrict__ c2) {
+  const int m = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const __nv_bfloat16* w = W + (size_t)m * K;
+  float s1 = 0.f, s2 = 0.f;
+  for (int k = lane; k < K; k += 32) {
+    const float wk = bf2f(w[k]);
+    s1 = fmaf(wk, g[k], s1);
+    s2 = fmaf(wk, b[k], s2);
+  }
+  s1 = warp_sum(s1);
+  s2 = warp_sum(s2);
+  if (lane == 0) {
+    c1[m] = s1;
+    c2[m] = s2;
+  }
+}
+void launch_ln_fold(const void* W, const float* g, const float* b, int M, int K, float* c1, float* c2,
+                    cudaStream_t st) {
+  ln_fold_kernel<<<(M + 7) / 8, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(W), g, b, M, K, c1, c2);
+}
+
 void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
-                  cudaStream_t st, bool pdl, unsigned long long* tl) {
+                  cudaStream_t st, bool pdl, unsigned long long* tl, __nv_bfloat16* xg, const float* gain,
+                  float2* st_part) {
   if (w_bf16)
     launch_ex(embed_kernel<__nv_bfloat16>, dim3(R_max), dim3(128), 0, st, pdl, 1,
-              static_cast<const __nv_bfloat16*>(tok_emb), static_cast<const __nv_bfloat16*>(pos_emb), plan, d, x, tl);
+              static_cast<const __nv_bfloat16*>(tok_emb), static_cast<const __nv_bfloat16*>(pos_emb), plan, d, x, xg,
+              gain, st_part, tl);
   else
     launch_ex(embed_kernel<float>, dim3(R_max), dim3(128), 0, st, pdl, 1, static_cast<const float*>(tok_emb),
-              static_cast<const float*>(pos_emb), plan, d, x, tl);
+              static_cast<const float*>(pos_emb), plan, d, x, xg, gain, st_part, tl);
 }
 
 // LayerNorm for any d % 4 == 0: a sum pass, a centred sum-of-squares pass over the

@@ -167,9 +167,9 @@ def test_timeline_records_every_launch_in_order(built_lib, cuda):
         s.close()
     assert outs[0] == outs[1]
     ns, kinds = records
-    g, ln = A.TL_GEMM, 3   # LayerNorm as its own launch (the default)
-    layer = [ln, g + 1, 4, g + 2, ln, g + 3, 5, g + 2, ln, g + 4, g + 2]
-    one = [1, 2] + layer * DIMS.n_layers + [ln, g + 6, 6]
+    g, f = A.TL_GEMM, A.TL_LN_FUSED   # LayerNorm folded into its neighbours (the default)
+    layer = [g + 1 + f, 4, g + 2, g + 3 + f, 5, g + 2, g + 4 + f, g + 2]
+    one = [1, 2] + layer * DIMS.n_layers + [g + 6 + f, 6]
     assert list(kinds) == one * 3
     ns = ns.astype(np.int64)
     start, work, mid, end = ns[:, 0], ns[:, 1], ns[:, 2], ns[:, 3]

@@ -49,12 +49,12 @@ def test_tiny_fp32_full_workload(built_lib, cuda):
     assert st.near_ties == 0
 
 
-@pytest.mark.parametrize("std,ln_fused", [(0.02, False), (0.05, False), (0.02, True)])
-def test_small_bf16_ragged_batch(built_lib, cuda, monkeypatch, std, ln_fused):
-    """ln_fused: the GEMMs after a LayerNorm normalise their own B operand
-    (the optional fused path, read from the environment at create time)."""
-    if ln_fused:
-        monkeypatch.setenv("ASRSPEC_LN_FUSE_MAX", "64")
+@pytest.mark.parametrize("std,ln_kernel", [(0.02, False), (0.05, False), (0.02, True)])
+def test_small_bf16_ragged_batch(built_lib, cuda, monkeypatch, std, ln_kernel):
+    """ln_kernel: LayerNorm as its own launch instead of folded into its
+    neighbouring GEMMs (read from the environment at create time)."""
+    if ln_kernel:
+        monkeypatch.setenv("ASRSPEC_LN_FOLD", "0")
     dims = W.SMALL
     blob = _blob(dims, std)
     enc_lens = [1500, 777, 250, 1023, 1]
@@ -65,7 +65,7 @@ def test_small_bf16_ragged_batch(built_lib, cuda, monkeypatch, std, ln_fused):
     prompt = W.make_prompt(dims, 5)
     st, _ = run_decode(dims, blob, enc, enc_lens, prompt, total, 8, W.make_corruption(wl),
                        _session(dims, blob, 5, 8), scale=scale_for(dims, std))
-    _report(f"small std={std}{' ln-fused' if ln_fused else ''}", st)
+    _report(f"small std={std}{' ln-kernel' if ln_kernel else ''}", st)
     assert st.rows > 50
 
 
