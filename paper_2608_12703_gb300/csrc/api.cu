@@ -89,6 +89,7 @@ struct asr_spec {
   bool use_mc = false;        // multicast weight tiles across the row tiles (ASRSPEC_MC=1; slower as measured)
   int wide_bn = 64;      // N tile for many rows (ASRSPEC_WIDE_BN: 64, 128, 192, 224, 256)
   int wide_target = 2 * 152;   // CTAs a many-row GEMM may fill by splitting K (ASRSPEC_WIDE_TARGET)
+  int few_target = 2 * 152;    // the same for few rows (ASRSPEC_FEW_TARGET)
   // launch timeline (diagnostics): [ASR_TL_CAP][4] device slots, the kind of
   // each recorded launch, and the slot of the launch being enqueued
   bool tl_on = false;
@@ -244,7 +245,7 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   g.K = K;
   const int tiles = ((M + 127) / 128) * ((N + g.bn - 1) / g.bn);
   const int nkb = K / 64;
-  const int target = N <= 64 ? 2 * NUM_SMS_TARGET : h->wide_target;
+  const int target = N <= 64 ? h->few_target : h->wide_target;
   g.splits = 1;
   if (mode != EPI_ARGMAX && mode != EPI_F32)
     while (g.splits < 16 && tiles * g.splits * 2 <= target && g.splits * 2 <= (N <= 64 ? nkb : nkb / 4))
@@ -545,6 +546,7 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
     if (v == 64 || v == 128 || v == 192 || v == 224 || v == 256) h->wide_bn = v;
   }
   if (const char* e = std::getenv("ASRSPEC_WIDE_TARGET")) h->wide_target = std::max(1, std::atoi(e));
+  if (const char* e = std::getenv("ASRSPEC_FEW_TARGET")) h->few_target = std::max(1, std::atoi(e));
   h->es = h->bf16 ? 2 : 4;
   h->ln_fold = h->bf16 && h->d % 128 == 0 && h->wide_bn <= 64;
   if (const char* e = std::getenv("ASRSPEC_LN_FOLD")) h->ln_fold = h->ln_fold && std::atoi(e) != 0;
