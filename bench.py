@@ -8,7 +8,9 @@ commit, re-anchoring) until every utterance has its target length.
 value = emitted tokens (accepted drafts + bonus tokens) per second over the
 timed steps, with weights and encoder states resident in HBM.
 
-Also reported, on the same workload: per-verify-call latency (CUDA events),
+Also reported, on the same workload: per-verify-call latency (CUDA events) over
+the decode and at a fixed state (verify, rollback, verify: 20 + 100 calls), the
+encoder-cache build alone,
 the dominant kernel against its roofline, an end-to-end number through
 host buffers, the CPU oracle on a bounded sample, and the batch-1 workload.
 
@@ -254,6 +256,51 @@ class GpuRun:
         return dict(ms=ms, launches=int(launches.sum()) + 0, traffic=traffic, clocks=clk.summary(),
                     verify_us=dict(median=float(np.median(per_call)), p10=float(np.percentile(per_call, 10)),
                                    p90=float(np.percentile(per_call, 90)), calls=int(len(per_call))))
+
+    def fixed_state(self, reps=100, warm=20):
+        """The paper's per-step protocol: one verify call repeated at a fixed
+        committed state (verify, rollback to the state, verify again), here the
+        state after half of the decode's rounds.  Per-call CUDA-event times of
+        `reps` calls after `warm` warm-up calls."""
+        torch, A, s = self.torch, self.A, self.sess
+        self._begin()
+        for _ in range(self.rounds // 2):
+            d, l = self.drafts.next()
+            s.verify_device(d, l, self.wl.k)
+        d, l = self.drafts.next()
+        with torch.cuda.stream(s.stream):
+            kv = torch.zeros(self.wl.batch, dtype=torch.int32, device="cuda")
+            pe = torch.zeros(self.wl.batch, dtype=torch.int32, device="cuda")
+        A.asr_spec_state(s.h, kv, pe)
+        ev = []
+        for i in range(warm + reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(s.stream)
+            s.verify_device(d, l, self.wl.k)
+            e1.record(s.stream)
+            A.asr_spec_rollback(s.h, kv, pe)
+            if i >= warm:
+                ev.append((e0, e1))
+        torch.cuda.synchronize()
+        us = np.array([a.elapsed_time(b) for a, b in ev]) * 1e3
+        assert s.status() == 0
+        return {"median": float(np.median(us)), "p10": float(np.percentile(us, 10)),
+                "p90": float(np.percentile(us, 90)), "reps": reps, "warmup": warm,
+                "state": f"after {self.rounds // 2} of {self.rounds} rounds"}
+
+    def encode_ms(self, reps=5):
+        """asr_spec_encode_cache alone (all layers' encoder K/V), CUDA events."""
+        torch, A, s = self.torch, self.A, self.sess
+        ev = []
+        for i in range(reps + 1):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(s.stream)
+            A.asr_spec_encode_cache(s.h, self.wl.batch, self.enc, self.wl.t_max, self.enc_lens_d)
+            e1.record(s.stream)
+            if i:
+                ev.append((e0, e1))
+        torch.cuda.synchronize()
+        return float(np.mean([a.elapsed_time(b) for a, b in ev]))
 
     def launch_timeline(self):
         """One decode with the launch timeline recorded (direct launches)."""
@@ -559,11 +606,15 @@ def main():
     value = total_tokens / (ms / 1e3)
     prof_ms, prof_launches, prof_traffic = run.profile()
     tl = run.launch_timeline()
+    fixed = run.fixed_state()
+    enc_ms = run.encode_ms()
     line = base_line(args, wl, world)
     bytes_per_call = step_bytes(wl.dims, prof_traffic)
     line.update({
         "value": value, "ms_per_step": ms / args.steps,
         "verify_us": res["verify_us"],
+        "fixed_state_verify_us": fixed,
+        "encode_cache_ms": enc_ms,
         "verify_rounds_per_step": run.rounds,
         "transcript_tokens_changed_by_batching": run.changed_tokens,
         "verify_hbm": {"bytes_per_call": bytes_per_call,
@@ -590,10 +641,13 @@ def main():
             b1 = r1.timed(args.steps, args.warmup, None, gpu_index=local)
             pm, pl, pt = r1.profile()
             tl1 = r1.launch_timeline()
+            fixed1 = r1.fixed_state()
+            enc1 = r1.encode_ms()
             bpc = step_bytes(wl1.dims, pt)
             line["batch1"] = {
                 "workload": wl1.name, "value": args.steps * r1.tokens_per_decode / (b1["ms"] / 1e3),
                 "unit": "tokens/s", "ms_per_step": b1["ms"] / args.steps, "verify_us": b1["verify_us"],
+                "fixed_state_verify_us": fixed1, "encode_cache_ms": enc1,
                 "verify_rounds_per_step": r1.rounds,
                 "verify_hbm": {"bytes_per_call": bpc,
                                "frac": bpc / (b1["verify_us"]["median"] * 1e-6) / (pk["hbm"] * 1e9),

@@ -64,6 +64,9 @@ struct Epi {
   int st_stride = 0;
   // launch timeline slot (see tl_mark), or null
   unsigned long long* tl = nullptr;
+  // > 0: one-dimensional grid walked in bands of group_m M tiles, each band
+  // sweeping every N tile (L2 reuse when both operands exceed the L2)
+  int group_m = 0;
   // optional phase timestamps (ns, %globaltimer) per CTA: [CTA][8]
   // (entry, set-up done, first stage full, MMAs done, end; cluster split:
   // partials staged, first cluster barrier passed, reduction done)

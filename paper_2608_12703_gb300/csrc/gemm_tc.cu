@@ -82,9 +82,17 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   // consecutive along x (one cluster); multicast: (M tiles, N tiles), the N
   // tiles of an M tile one cluster; otherwise (N tiles, M tiles, splits), so
   // that the CTAs sharing a weight tile run together and read it from HBM once.
-  const int tile_m = CLU ? (int)blockIdx.x / splits : MC ? (int)blockIdx.x : (int)blockIdx.y;
+  int tile_m = CLU ? (int)blockIdx.x / splits : MC ? (int)blockIdx.x : (int)blockIdx.y;
   const int split = CLU ? (int)blockIdx.x % splits : (int)blockIdx.z;
-  const int tile_n = (CLU || MC) ? (int)blockIdx.y : (int)blockIdx.x;
+  int tile_n = (CLU || MC) ? (int)blockIdx.y : (int)blockIdx.x;
+  if (!CLU && !MC && epi.group_m > 0) {   // grouped order: a band of group_m M tiles sweeps the N tiles
+    const int mt = (epi.M + TC_BM - 1) / TC_BM, nt = (epi.N + BN - 1) / BN;
+    const int band = (int)blockIdx.x / (epi.group_m * nt);
+    const int r = (int)blockIdx.x - band * epi.group_m * nt;
+    const int gm = min(epi.group_m, mt - band * epi.group_m);
+    tile_m = band * epi.group_m + r % gm;
+    tile_n = r / gm;
+  }
   const int m0 = tile_m * TC_BM, n0 = tile_n * BN;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   unsigned long long* tr = epi.trace ? epi.trace + 8ull * (blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z))
@@ -96,7 +104,19 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   const int kb0 = (nkb_total * split) / splits;
   const int kb1 = (nkb_total * (split + 1)) / splits;
   const int nkb = kb1 - kb0;
-  if (!MC && (n0 >= n_valid || nkb <= 0)) {   // uniform over the CTA and over all splits of a tile
+  bool dead = false;   // encoder-cache build: every frame of the tile is padding
+  if constexpr (MODE == EPI_CROSSKV) {
+    dead = true;
+    for (int mr = m0; mr < m0 + TC_BM && mr < epi.M;) {   // one segment per utterance in the tile
+      const int b = mr / epi.t_max, t = mr - b * epi.t_max;
+      if (t < epi.enc_len[b]) {
+        dead = false;
+        break;
+      }
+      mr = (b + 1) * epi.t_max;
+    }
+  }
+  if (!MC && (n0 >= n_valid || nkb <= 0 || dead)) {   // uniform over the CTA and over all splits of a tile
     pdl_wait();
     return;
   }
@@ -290,6 +310,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     const int rows = n_valid - n0 < BN ? n_valid - n0 : BN;
     epi_rows<MODE>(epi, stg, LDS, m0 + 4 * lane, 4 * lane, n0, warp, rows, ln_mu, ln_rs);
   } else if (splits == 1) {
+    // encoder-cache build: this thread's frame (utterance fb, frame ft) and whether it is real
+    const int fb = MODE == EPI_CROSSKV ? m / epi.t_max : 0, ft = MODE == EPI_CROSSKV ? m - fb * epi.t_max : 0;
+    const bool frame_ok = MODE == EPI_CROSSKV && m < epi.M && ft < epi.enc_len[fb];
     const bool fold = epi.ln_part != nullptr && MODE != EPI_CROSSKV;
     float c1m = 0.f, c2m = 0.f;
     if (fold) {
@@ -314,6 +337,40 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
           unsigned long long key = (m < epi.M && n < n_valid) ? argmax_key(v[i], (uint32_t)m) : 0ull;
           key = warp_max_u64(key);
           if (lane == 0) red[warp][c0 + i] = key;
+        }
+      } else if constexpr (MODE == EPI_CROSSKV) {
+        // 16 consecutive features of one frame lie in one head: one index, two
+        // 16-byte stores (bf16) per thread
+        if (frame_ok && n0 + c0 < n_valid) {
+          const int n = n0 + c0, two_d = 2 * epi.d;
+          const int l = n / two_d, r = n - l * two_d;
+          const int which = r / epi.d, f = r - which * epi.d;
+          const size_t idx =
+              (((((size_t)l * 2 + which) * epi.b_max + fb) * epi.n_heads + (f >> 6)) * epi.max_enc + ft) * 64 + (f & 63);
+          float w[16];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float4 bq = __ldg(reinterpret_cast<const float4*>(epi.bias + n) + q);
+            w[4 * q + 0] = v[4 * q + 0] + bq.x;
+            w[4 * q + 1] = v[4 * q + 1] + bq.y;
+            w[4 * q + 2] = v[4 * q + 2] + bq.z;
+            w[4 * q + 3] = v[4 * q + 3] + bq.w;
+          }
+          if (epi.kv_bf16) {
+            uint32_t pk[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              __nv_bfloat162 t2 = __floats2bfloat162_rn(w[2 * q], w[2 * q + 1]);
+              pk[q] = *reinterpret_cast<uint32_t*>(&t2);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(epi.kcache) + idx);
+            dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          } else {
+            float4* dst = reinterpret_cast<float4*>(static_cast<float*>(epi.kcache) + idx);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) dst[q] = make_float4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+          }
         }
       } else {
         int mm[16], nn[16];
@@ -670,8 +727,9 @@ static void launch_tc_t(const TcGemm& g, const Epi& epi, int* status, cudaStream
       return;
     }
   }
-  launch_ex(gemm_tc_kernel<BN, MODE, false, false>, dim3(nt, mt, g.splits), dim3(128), TcCfg<BN>::SMEM, st, g.pdl,
-            1, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi, status);
+  const dim3 grid = epi.group_m > 0 ? dim3(nt * mt, 1, g.splits) : dim3(nt, mt, g.splits);
+  launch_ex(gemm_tc_kernel<BN, MODE, false, false>, grid, dim3(128), TcCfg<BN>::SMEM, st, g.pdl, 1, g.mapA, g.mapB,
+            g.K, g.splits, g.ws, g.tickets, epi, status);
 }
 
 template <int MODE>
