@@ -361,7 +361,8 @@ class GpuRun:
 # over the kernel's launches in one layer.  Only valid for the kernel code the
 # capture ran on: drop an entry when that kernel changes.
 NCU_TRAFFIC = {
-    ("large-bf16-b1-k8", "resid"): (6.727e6, "profiles/gemm_tc_kernel_resid_large-bf16-b1-k8.md"),
+    ("large-bf16-b1-k8", "resid"): (6.76e6, "profiles/gemm_tc_kernel_resid_large-bf16-b1-k8.md"),
+    ("large-bf16-b64-k6", "resid"): (11.21e6, "profiles/gemm_tc_kernel_large-bf16-b64-k6_tensor.md"),
     ("large-bf16-b64-k6", "cross_attn"): (337.7e6, "profiles/attn_tc_kernel_large-bf16-b64-k6_dram.md"),
 }
 
