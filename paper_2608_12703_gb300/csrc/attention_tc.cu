@@ -15,8 +15,10 @@
 //     P re-used from the S fragments and V fragments from ldmatrix.trans;
 //   * each of the 4 warps takes a quarter of every chunk's keys; the CTA
 //     combines its warps, and the S splits of one (utterance, head) form a
-//     thread-block cluster that merges through distributed shared memory in
-//     split order, so the result does not depend on timing.
+//     thread-block cluster: CTA q owns output columns [64q/S, 64(q+1)/S), every
+//     split pushes its (max, sum, partial output) of those columns into q's
+//     shared memory with st.async (bytes counted on q's mbarrier), and q merges
+//     them in split order, so the result does not depend on timing.
 #include <mutex>
 
 #include "kernels.h"
@@ -53,34 +55,40 @@ __device__ __forceinline__ uint32_t sw128(int row, int chunk16) {
 constexpr int TCA_CH = 128;        // keys per chunk (one TMA tile of K and one of V)
 constexpr int TCA_TILE = TCA_CH * 128;
 
-template <int MT, int STAGES>
+template <int MT, int STAGES, bool PUSH>
 struct TcaCfg {
   static constexpr int KW = TCA_CH / 4;       // keys per warp per chunk
   static constexpr int NT = KW / 8;           // n-tiles of keys per warp
   static constexpr int RING = STAGES * 2 * TCA_TILE;
   static constexpr int OW = 4 * MT * 16 * 64 * 4;
   static constexpr int PART = (32 * 64 + 64) * 4;   // this CTA's (max, sum, output) per row
-  static constexpr int SMEM = 1024 + (RING > OW ? RING : OW) + PART;
+  static constexpr int P_OFF = RING > OW ? RING : OW;
+  // split merge by push: the partials of this CTA's output columns from every
+  // split, [split][row][4 + 64 / S] floats ((max, sum, -, -), output columns)
+  static constexpr int RECV_OFF = P_OFF + PART;
+  static constexpr int RECV = PUSH ? MT * 16 * 96 * 4 : 0;
+  static constexpr int SMEM = 1024 + RECV_OFF + RECV;
 };
 
 // One CTA = one (utterance, head, split).  The CTA streams chunks split,
 // split + S, split + 2S, ... of the utterance's keys through a TMA ring,
 // keeping a running (max, sum, output) per row (online softmax).  With S > 1
 // the S splits of a (utterance, head) form one cluster and merge their
-// results through distributed shared memory, in split order.
-template <int MT, int TCA_STAGES>
+// results by pushing them to the CTA that owns each output column (PUSH).
+template <int MT, int TCA_STAGES, bool PUSH>
 __global__ void __launch_bounds__(TCA_THREADS)
 attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, AttnArgs a,
                int* status) {
-  using C = TcaCfg<MT, TCA_STAGES>;
+  using C = TcaCfg<MT, TCA_STAGES, PUSH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   float* Ow = reinterpret_cast<float*>(smem);                  // warp partials, after the ring is drained
-  float* Pm = reinterpret_cast<float*>(smem + (C::RING > C::OW ? C::RING : C::OW));   // [32] max
+  float* Pm = reinterpret_cast<float*>(smem + C::P_OFF);       // [32] max
   float* Pl = Pm + 32;                                          // [32] sum
   float* Po = Pm + 64;                                          // [32][64] output (relative to max)
   __shared__ float mw[4][MT * 16], lw[4][MT * 16];
   __shared__ __align__(8) uint64_t bar[TCA_STAGES];
+  __shared__ __align__(8) uint64_t rbar;   // PUSH: the other splits' partials have landed
 
   const int S = gridDim.x, split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   tl_mark(a.tl, TL_ENTRY);
@@ -99,9 +107,16 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
 
   if (tid == 0) {
     for (int st = 0; st < TCA_STAGES; ++st) mbar_init(&bar[st], 1);
+    if constexpr (PUSH) {   // (S - 1) messages per row: (max, sum) and 64 / S output columns
+      mbar_init(&rbar, 1);
+      mbar_arrive_expect_tx(&rbar, (uint32_t)((S - 1) * nr * (8 + 4 * (64 / S))));
+    }
     fence_mbar_init();
   }
   __syncthreads();
+  // PUSH: announce this CTA's receive barrier; the matching wait comes just
+  // before the first remote store, long after every split has arrived
+  if constexpr (PUSH) cluster_arrive_relaxed();
   auto issue = [&](int i) {
     const int st = i % TCA_STAGES;
     const int key0 = (split + i * S) * TCA_CH;
@@ -290,66 +305,99 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
   // merge the splits of this (utterance, head) in split order
   tl_mark(a.tl, TL_MID);
   __syncwarp();
-  if (S > 1) cluster_sync();
-  else __syncthreads();
-  for (int e = split * TCA_THREADS + tid; e < nr * 64; e += S * TCA_THREADS) {
-    const int r = e >> 6, c = e & 63;
-    float M = -INFINITY;
-    for (int s = 0; s < S; ++s) M = fmaxf(M, S > 1 ? ld_dsmem_f32(dsmem_addr(Pm + r, s)) : Pm[r]);
-    const float Mu = (M == -INFINITY) ? 0.f : M;
-    float L = 0.f, o = 0.f;
-    for (int s = 0; s < S; ++s) {
-      const float ms = S > 1 ? ld_dsmem_f32(dsmem_addr(Pm + r, s)) : Pm[r];
-      const float ls = S > 1 ? ld_dsmem_f32(dsmem_addr(Pl + r, s)) : Pl[r];
-      const float os = S > 1 ? ld_dsmem_f32(dsmem_addr(Po + r * 64 + c, s)) : Po[r * 64 + c];
-      const float f = __expf(ms - Mu);
-      L += ls * f;
-      o += os * f;
+  if constexpr (PUSH) {
+    __syncthreads();   // this CTA's (max, sum, output) per row are complete
+    cluster_wait();    // every split's receive barrier is initialised
+    const int cw = 64 / S, rs = 4 + cw;   // columns per owner, floats per received row
+    float* recv = reinterpret_cast<float*>(smem + C::RECV_OFF);
+    for (int pr = tid; pr < S * nr; pr += TCA_THREADS) {
+      const int q = pr / nr, r = pr - q * nr;   // owner rank, row
+      float* slot = recv + (split * nr + r) * rs;   // this split's row in q's buffer
+      const float* o = Po + r * 64 + q * cw;
+      if (q == split) {
+        slot[0] = Pm[r];
+        slot[1] = Pl[r];
+        for (int c = 0; c < cw; c += 4) *reinterpret_cast<float4*>(slot + 4 + c) = *reinterpret_cast<const float4*>(o + c);
+      } else {
+        const uint32_t dst = dsmem_addr(slot, (uint32_t)q), rb_q = dsmem_addr(&rbar, (uint32_t)q);
+        st_async_f2(dst, Pm[r], Pl[r], rb_q);
+        for (int c = 0; c < cw; c += 4)
+          st_async_f4(dst + (uint32_t)(4 + c) * 4u, *reinterpret_cast<const float4*>(o + c), rb_q);
+      }
     }
-    reinterpret_cast<__nv_bfloat16*>(a.out)[(size_t)(row0 + r) * a.d + h * 64 + c] = f2bf(o / L);
-    if (a.ml_out && c == 0) {
-      a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 0] = M;
-      a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 1] = L;
+    __syncthreads();                 // this CTA's own rows
+    mbar_wait(&rbar, 0, status);     // the other splits' rows
+    for (int e = tid; e < nr * cw; e += TCA_THREADS) {
+      const int r = e / cw, c = e - r * cw;
+      float M = -INFINITY;
+      for (int s2 = 0; s2 < S; ++s2) M = fmaxf(M, recv[(s2 * nr + r) * rs]);
+      const float Mu = (M == -INFINITY) ? 0.f : M;
+      float L = 0.f, o = 0.f;
+      for (int s2 = 0; s2 < S; ++s2) {
+        const float* row = recv + (s2 * nr + r) * rs;
+        const float f = __expf(row[0] - Mu);
+        L += row[1] * f;
+        o += row[4 + c] * f;
+      }
+      reinterpret_cast<__nv_bfloat16*>(a.out)[(size_t)(row0 + r) * a.d + h * 64 + split * cw + c] = f2bf(o / L);
+      if (a.ml_out && split == 0 && c == 0) {
+        a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 0] = M;
+        a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 1] = L;
+      }
+    }
+  } else {
+    __syncthreads();
+    for (int e = tid; e < nr * 64; e += TCA_THREADS) {
+      const int r = e >> 6, c = e & 63;
+      const float M = Pm[r];
+      reinterpret_cast<__nv_bfloat16*>(a.out)[(size_t)(row0 + r) * a.d + h * 64 + c] = f2bf(Po[r * 64 + c] / Pl[r]);
+      if (a.ml_out && c == 0) {
+        a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 0] = M;
+        a.ml_out[((size_t)(row0 + r) * a.H + h) * 2 + 1] = Pl[r];
+      }
     }
   }
-  if (S > 1) cluster_sync();   // no CTA leaves while another may still read its shared memory
   tl_mark(a.tl, TL_EXIT);
 }
 
-template <int MT, int ST>
+template <int MT, int ST, bool PUSH>
 static void configure_one() {
-  cudaFuncSetAttribute(attn_tc_kernel<MT, ST>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcaCfg<MT, ST>::SMEM);
+  cudaFuncSetAttribute(attn_tc_kernel<MT, ST, PUSH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       TcaCfg<MT, ST, PUSH>::SMEM);
+  if constexpr (PUSH) cudaFuncSetAttribute(attn_tc_kernel<MT, ST, PUSH>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
 
 void configure_attention_tc() {
   static std::once_flag once;
   std::call_once(once, [] {
-    configure_one<1, 2>();
-    configure_one<2, 2>();
-    configure_one<1, 3>();
-    configure_one<2, 3>();
+    configure_one<1, 2, false>();
+    configure_one<2, 2, false>();
+    configure_one<1, 2, true>();
+    configure_one<2, 2, true>();
+    configure_one<1, 3, true>();
+    configure_one<2, 3, true>();
   });
 }
 
-template <int MT, int ST>
+template <int MT, int ST, bool PUSH>
 static void launch_one(const AttnArgs& a, int splits, int* status, cudaStream_t st) {
-  launch_ex(attn_tc_kernel<MT, ST>, dim3(splits, a.H, a.B), dim3(TCA_THREADS), TcaCfg<MT, ST>::SMEM, st, a.pdl,
-            splits, *a.kmap, *a.vmap, a, status);
+  launch_ex(attn_tc_kernel<MT, ST, PUSH>, dim3(splits, a.H, a.B), dim3(TCA_THREADS), TcaCfg<MT, ST, PUSH>::SMEM, st,
+            a.pdl, splits, *a.kmap, *a.vmap, a, status);
 }
 
 // a.splits CTAs (1, 2, 4 or 8; one cluster) per (utterance, head);
 // rows_max > 16 takes two m-tiles.
 void launch_attention_tc(const AttnArgs& a, int* status, cudaStream_t st) {
   configure_attention_tc();
-  if (a.causal) {
-    if (a.rows_max > 16) launch_one<2, 2>(a, a.splits, status, st);
-    else launch_one<1, 2>(a, a.splits, status, st);
-  } else if (a.splits == 1) {   // many utterances: more CTAs per SM (54 vs 56 us at batch 64)
-    if (a.rows_max > 16) launch_one<2, 2>(a, a.splits, status, st);
-    else launch_one<1, 2>(a, a.splits, status, st);
-  } else {                      // few utterances, keys split over a cluster: deeper ring per CTA
-    if (a.rows_max > 16) launch_one<2, 3>(a, a.splits, status, st);
-    else launch_one<1, 3>(a, a.splits, status, st);
+  if (a.splits == 1) {   // one CTA per (utterance, head): 2-deep ring, three CTAs per SM (54 vs 56 us at batch 64)
+    if (a.rows_max > 16) launch_one<2, 2, false>(a, a.splits, status, st);
+    else launch_one<1, 2, false>(a, a.splits, status, st);
+  } else if (a.causal) {   // self-attention keys split over a cluster (at most max_pos keys)
+    if (a.rows_max > 16) launch_one<2, 2, true>(a, a.splits, status, st);
+    else launch_one<1, 2, true>(a, a.splits, status, st);
+  } else {                 // encoder keys split over a cluster: deeper ring per CTA
+    if (a.rows_max > 16) launch_one<2, 3, true>(a, a.splits, status, st);
+    else launch_one<1, 3, true>(a, a.splits, status, st);
   }
 }
 

@@ -346,6 +346,11 @@ __device__ __forceinline__ void st_async_f4(uint32_t addr, float4 v, uint32_t re
                ::"r"(addr), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(remote_bar)
                : "memory");
 }
+__device__ __forceinline__ void st_async_f2(uint32_t addr, float a, float b, uint32_t remote_bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];"
+               ::"r"(addr), "f"(a), "f"(b), "r"(remote_bar)
+               : "memory");
+}
 // shared::cluster address of the same shared variable in CTA `rank` of this cluster
 __device__ __forceinline__ uint32_t dsmem_addr(const void* local, uint32_t rank) {
   uint32_t out;
