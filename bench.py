@@ -369,7 +369,7 @@ NCU_TRAFFIC = {
 # Launch kinds of the timeline (ASR_TL_*; a LayerNorm-fused GEMM counts with its
 # GEMM) and the profile class (CUDA events) that times the same kernel.
 TL_KIND_CLASS = {17: "qkv", 18: "resid", 19: "query", 20: "mlp_up", 22: "lm_head", 4: "self_attn",
-                 5: "cross_attn", 3: "layernorm"}
+                 5: "cross_attn", 3: "layernorm", 7: "fused"}
 
 
 def kind_class(kind: int):
@@ -396,6 +396,11 @@ def algorithmic_work(dims, cls, traffic):
         return self_b, 0.0, "2 (K, V) x (P_b + n_b) keys x d x 2 bytes per active utterance per layer"
     if cls == "cross_attn":
         return cross_b, 0.0, "2 (K, V) x T_b frames x d x 2 bytes per active utterance per layer"
+    if cls == "fused":
+        params = L * (6 * d * d + 2 * F * d) + V * d
+        return (calls * params * es + self_b + cross_b, 2.0 * rows * params,
+                "all projection and LM-head weights x %d bytes per verify call + the self and cross K/V rows read "
+                "(2 x keys x d x %d bytes per active utterance per layer); 2 x scored rows x weights in flops" % (es, es))
     if cls == "layernorm":
         return rows * (3 * L + 1) * d * (4 + es), 0.0, "rows x d x (4 read + 2 written) bytes per LayerNorm"
     return 0.0, 0.0, ""

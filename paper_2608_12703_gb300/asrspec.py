@@ -28,11 +28,14 @@ EXPORTED = [
     "asr_spec_status", "asr_spec_last_error", "asr_spec_destroy", "asr_spec_synth_drafts",
     "asr_spec_test_gemm", "asr_spec_set_graphs", "asr_spec_profile", "asr_spec_profile_read",
     "asr_spec_gemm_noalloc", "asr_spec_timeline", "asr_spec_timeline_read",
+    "asr_spec_fused_trace", "asr_spec_fused_trace_read",
 ]
-PROF_CLASSES = ["qkv", "resid", "query", "mlp_up", "self_attn", "cross_attn", "lm_head", "layernorm", "other"]
+PROF_CLASSES = ["qkv", "resid", "query", "mlp_up", "self_attn", "cross_attn", "lm_head", "layernorm", "other",
+                "fused"]
 TL_CAP = 65536
 TL_GEMM, TL_LN_FUSED = 16, 32
-TL_KINDS = {0: "other", 1: "plan", 2: "embed", 3: "layernorm", 4: "attn_self", 5: "attn_cross", 6: "accept_anchor"}
+TL_KINDS = {0: "other", 1: "plan", 2: "embed", 3: "layernorm", 4: "attn_self", 5: "attn_cross", 6: "accept_anchor",
+            7: "fused_verify"}
 TL_GEMM_EPILOGUES = {0: "plain", 1: "qkv", 2: "residual", 3: "query", 4: "gelu", 5: "cross_kv", 6: "argmax"}
 
 
@@ -92,6 +95,8 @@ def lib():
     L.asr_spec_gemm_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
     L.asr_spec_timeline.argtypes = [vp, i32]
     L.asr_spec_timeline_read.argtypes = [vp, vp, vp, i32, vp]
+    L.asr_spec_fused_trace.argtypes = [vp, i32]
+    L.asr_spec_fused_trace_read.argtypes = [vp, vp, ctypes.c_int64, vp, vp]
     for name in EXPORTED:
         if name not in ("asr_spec_last_error", "asr_spec_destroy"):
             getattr(L, name).restype = ctypes.c_int
@@ -213,6 +218,21 @@ def asr_spec_timeline_read(h):
            "asr_spec_timeline_read")
     n = min(count.value, TL_CAP)
     return ns[:n].copy(), kinds[:n].copy()
+
+
+def asr_spec_fused_trace(h, enable: bool):
+    return _check(h, lib().asr_spec_fused_trace(h, 1 if enable else 0), "asr_spec_fused_trace")
+
+
+def asr_spec_fused_trace_read(h):
+    """Per-CTA stage timestamps (ns) of the last traced fused verify, [n_cta][16 L + 2]."""
+    per, n = ctypes.c_int32(0), ctypes.c_int32(0)
+    _check(h, lib().asr_spec_fused_trace_read(h, None, 0, ctypes.byref(per), ctypes.byref(n)),
+           "asr_spec_fused_trace_read")
+    out = np.zeros((n.value, per.value), dtype=np.uint64)
+    _check(h, lib().asr_spec_fused_trace_read(h, out.ctypes.data, out.size, ctypes.byref(per), ctypes.byref(n)),
+           "asr_spec_fused_trace_read")
+    return out
 
 
 def asr_spec_gemm_noalloc(A, B, C, M, N, K, splits, stream=None):

@@ -86,6 +86,20 @@ struct asr_spec {
   bool ln_fold = false;
   float2* ln_part = nullptr;
   int ln_S = 0, ln_c = 0;
+  // fused verify for steps of at most VF_ROWS rows (ASRSPEC_FUSED=1 turns it
+  // on; off by default: 2.04 against 1.84 ms per batch-1 round of the large
+  // decoder, as measured): the grid (one CTA per SM, 0 = unavailable), the
+  // layer table, the grid barrier counter, the split-merge tickets and
+  // partials of its attention
+  bool use_fused = false;
+  int vf_G = 0, vf_bmax = 0;
+  VfLayer* vf_layers = nullptr;
+  unsigned* vf_bar = nullptr;
+  int* vf_tickets = nullptr;
+  float* vf_part = nullptr;
+  bool last_fused = false;    // the last verify ran the fused kernel (LM-head input in xf)
+  unsigned long long* vf_trace = nullptr;   // per-stage timestamps of the fused kernel (diagnostics)
+  bool vf_trace_on = false;
   bool use_mc = false;        // multicast weight tiles across the row tiles (ASRSPEC_MC=1; slower as measured)
   int wide_bn = 64;      // N tile for many rows (ASRSPEC_WIDE_BN: 64, 128, 192, 224, 256)
   int wide_target = 2 * 152;   // CTAs a many-row GEMM may fill by splitting K (ASRSPEC_WIDE_TARGET)
@@ -105,6 +119,7 @@ struct asr_spec {
     cudaGraphExec_t exec;
     long long launches[ASR_PROF_N];
     int ln_S, ln_c;   // the folded LayerNorm slices the captured body leaves (for debug_logits)
+    bool fused;       // the body is the fused verify kernel
   };
   std::map<std::pair<int, int>, Graph> graphs;
 };
@@ -483,14 +498,58 @@ int enqueue_verify(asr_spec* h, int k) {
                        h->row_key, h->status, tr, h->st, h->tl_cur);
   }
   const int N = B * (k + 1);
-  if (int rc = run_layers(h, N)) return rc;
-  Epi e{};
-  e.n_valid = h->plan.n_rows;
-  e.row_key = h->row_key;
-  e.d = h->d;
-  if (int rc = gemm_rows_ln(h, h->w_tok, &h->m_tok, h->V, h->d, h->lnf_g, h->lnf_b, h->c1_lm, h->c2_lm, h->xf, BUF_XF,
-                            N, EPI_ARGMAX, e))
-    return rc;
+  h->last_fused = h->vf_G > 0 && N <= VF_ROWS && B <= h->vf_bmax;
+  if (h->last_fused) {   // few rows: one persistent kernel for the layers and the LM head
+    CK(cudaMemsetAsync(h->vf_bar, 0, 4, h->st));
+    VfArgs a{};
+    a.layers = h->vf_layers;
+    a.L = h->L;
+    a.d = h->d;
+    a.H = h->H;
+    a.F = h->F;
+    a.V = h->V;
+    a.max_pos = h->maxpos;
+    a.t_alloc = h->Tmax;
+    a.b_max = h->Bmax;
+    a.anchor = h->anchor;
+    a.B = B;
+    a.S = std::max(1, std::min(16, h->vf_G / (B * h->H)));
+    int total = 0;
+    vf_layout(h->d, h->F, h->L, &a.a_bytes, &a.slot_bytes, &total);
+    a.tok_emb = static_cast<const __nv_bfloat16*>(h->w_tok);
+    a.pos_emb = static_cast<const __nv_bfloat16*>(h->w_pos);
+    a.lnf_g = h->lnf_g;
+    a.lnf_b = h->lnf_b;
+    a.plan = h->plan;
+    a.kv_len = h->kv_len;
+    a.enc_len = h->enc_len;
+    a.x = h->x;
+    a.q = h->q;
+    a.q_anchor = h->q_anchor;
+    a.ml = h->ml;
+    a.part = h->vf_part;
+    a.att = static_cast<__nv_bfloat16*>(h->att);
+    a.hbuf = static_cast<__nv_bfloat16*>(h->hbuf);
+    a.xf = static_cast<__nv_bfloat16*>(h->xf);
+    a.row_key = h->row_key;
+    a.bar_ctr = h->vf_bar;
+    a.tickets = h->vf_tickets;
+    a.status = h->status;
+    a.trace = h->vf_trace_on ? h->vf_trace : nullptr;
+    Prof p(h, ASR_PROF_FUSED, 1);
+    Tl t(h, ASR_TL_FUSED);
+    a.tl = h->tl_cur;
+    CK(launch_verify_fused(&h->m_xkv[0], a, h->vf_G, h->st));
+  } else {
+    if (int rc = run_layers(h, N)) return rc;
+    Epi e{};
+    e.n_valid = h->plan.n_rows;
+    e.row_key = h->row_key;
+    e.d = h->d;
+    if (int rc = gemm_rows_ln(h, h->w_tok, &h->m_tok, h->V, h->d, h->lnf_g, h->lnf_b, h->c1_lm, h->c2_lm, h->xf,
+                              BUF_XF, N, EPI_ARGMAX, e))
+      return rc;
+  }
   Prof p(h, ASR_PROF_OTHER, 1);
   AcceptAnchorArgs A{};
   A.draft = h->draft_buf;
@@ -767,6 +826,32 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   }
   if ((rc = dalloc(h, &h->counters, 8 * sizeof(unsigned long long)))) return finish(rc);
   CK(cudaMemset(h->counters, 0, 8 * sizeof(unsigned long long)));
+  if (const char* e = std::getenv("ASRSPEC_FUSED")) h->use_fused = std::atoi(e) != 0;
+  if (h->bf16 && h->use_fused && (h->vf_G = vf_grid(d, F, L)) > 0) {
+    std::vector<VfLayer> t(L);
+    for (int l = 0; l < L; ++l) {
+      const LayerW& w = h->lw[l];
+      VfLayer& v = t[l];
+      v.wqkv = static_cast<const __nv_bfloat16*>(w.wqkv);
+      v.wo = static_cast<const __nv_bfloat16*>(w.wo);
+      v.wcq = static_cast<const __nv_bfloat16*>(w.wcq);
+      v.wco = static_cast<const __nv_bfloat16*>(w.wco);
+      v.w1 = static_cast<const __nv_bfloat16*>(w.w1);
+      v.w2 = static_cast<const __nv_bfloat16*>(w.w2);
+      v.bqkv = w.bqkv; v.bo = w.bo; v.bcq = w.bcq; v.bco = w.bco; v.b1 = w.b1; v.b2 = w.b2;
+      v.ln1g = w.ln1g; v.ln1b = w.ln1b; v.ln2g = w.ln2g; v.ln2b = w.ln2b; v.ln3g = w.ln3g; v.ln3b = w.ln3b;
+      const size_t self_layer = (size_t)h->Bmax * h->H * h->maxpos * 64;
+      v.ks = static_cast<__nv_bfloat16*>(h->kself) + l * self_layer;
+      v.vs = static_cast<__nv_bfloat16*>(h->vself) + l * self_layer;
+    }
+    h->vf_bmax = std::min(h->Bmax, VF_ROWS);
+    const size_t part = (size_t)h->vf_bmax * h->H * 16 * VF_ROWS * 66;
+    if ((rc = dalloc(h, &h->vf_layers, L * sizeof(VfLayer))) || (rc = dalloc(h, &h->vf_bar, 4)) ||
+        (rc = dalloc(h, &h->vf_tickets, (size_t)h->vf_bmax * h->H * 4)) || (rc = dalloc(h, &h->vf_part, part * 4)))
+      return finish(rc);
+    CK(cudaMemcpy(h->vf_layers, t.data(), L * sizeof(VfLayer), cudaMemcpyHostToDevice));
+    CK(cudaMemset(h->vf_tickets, 0, (size_t)h->vf_bmax * h->H * 4));
+  }
   configure_gemm_tc();
   configure_attention();
   CK(cudaDeviceSynchronize());
@@ -865,7 +950,7 @@ int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens
   }
   if (int rc = copy_in(h, h->lens_buf, lens, B)) return rc;
   for (int c = 0; c < ASR_PROF_N; ++c) h->cur[c] = 0;
-  if (h->use_graphs && !h->prof && !h->tl_on) {
+  if (h->use_graphs && !h->prof && !h->tl_on && !h->vf_trace_on) {
     auto key = std::make_pair(B, (int)k);
     auto it = h->graphs.find(key);
     if (it == h->graphs.end()) {
@@ -884,11 +969,13 @@ int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens
       for (int c = 0; c < ASR_PROF_N; ++c) g.launches[c] = h->cur[c];
       g.ln_S = h->ln_S;
       g.ln_c = h->ln_c;
+      g.fused = h->last_fused;
       it = h->graphs.emplace(key, g).first;
     }
     CK(cudaGraphLaunch(it->second.exec, h->st));
     h->ln_S = it->second.ln_S;
     h->ln_c = it->second.ln_c;
+    h->last_fused = it->second.fused;
     for (int c = 0; c < ASR_PROF_N; ++c) h->launches[c] += it->second.launches[c];
   } else {
     if (int rc = enqueue_verify(h, k)) return rc;
@@ -975,6 +1062,29 @@ int asr_spec_timeline_read(asr_spec_handle h, uint64_t* ns, int32_t* kind, int32
   return ASR_OK;
 }
 
+int asr_spec_fused_trace(asr_spec_handle h, int32_t enable) {
+  if (!h) return ASR_E_INVAL;
+  if (enable && h->vf_G == 0) return fail(h, ASR_E_INVAL, "the fused verify is not available for this model");
+  if (enable && !h->vf_trace) {
+    const size_t n = (size_t)h->vf_G * vf_trace_points(h->L);
+    int rc = dalloc(h, &h->vf_trace, n * sizeof(unsigned long long));
+    if (rc) return rc;
+    CK(cudaMemset(h->vf_trace, 0, n * sizeof(unsigned long long)));
+  }
+  h->vf_trace_on = enable != 0;
+  return ASR_OK;
+}
+
+int asr_spec_fused_trace_read(asr_spec_handle h, uint64_t* out, int64_t cap, int32_t* per_cta, int32_t* n_cta) {
+  if (!h || !per_cta || !n_cta || cap < 0 || (cap > 0 && !out)) return ASR_E_INVAL;
+  *per_cta = vf_trace_points(h->L);
+  *n_cta = h->vf_trace ? h->vf_G : 0;
+  const size_t n = std::min((size_t)cap, (size_t)(*n_cta) * (size_t)(*per_cta));
+  CK(cudaStreamSynchronize(h->st));
+  if (n > 0) CK(cudaMemcpy(out, h->vf_trace, n * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
+  return ASR_OK;
+}
+
 int asr_spec_rollback(asr_spec_handle h, const int32_t* new_len, const int32_t* new_pending) {
   if (!h) return ASR_E_INVAL;
   if (h->state < 2) return fail(h, ASR_E_STATE, "rollback before prefill");
@@ -1014,7 +1124,7 @@ int asr_spec_debug_logits(asr_spec_handle h, float* out, int32_t max_rows) {
   e.ld = h->V;
   e.n_valid = h->plan.n_rows;
   int rc;
-  if (h->ln_fold) {   // the same operand and statistics as the last verify's LM head
+  if (h->ln_fold && !h->last_fused) {   // the same operand and statistics as the last verify's LM head
     fold_consumer(h, e, h->c1_lm, h->c2_lm);
     rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xn, BUF_XN, R, EPI_F32, e);
   } else {

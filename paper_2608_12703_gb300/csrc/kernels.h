@@ -132,6 +132,50 @@ struct AcceptAnchorArgs {
 };
 void launch_accept_anchor(const AcceptAnchorArgs& a, cudaStream_t st);
 
+// ---- Fused verify for few rows ----------------------------------------------------
+// One persistent cooperative kernel (one CTA per SM) runs the decoder layers and
+// the LM head of a verify step whose rows all fit one 16-row MMA tile
+// (VF_ROWS): the stages are separated by grid-wide barriers, and a producer
+// warp streams every projection's weight slice through a shared-memory ring
+// independently of them, so the next stage's weights load while the current
+// stage waits.  Writes what the multi-kernel chain writes (residual, caches,
+// q_anchor, ml, argmax keys); the accept + anchor kernel follows it.
+constexpr int VF_ROWS = 9;
+struct VfLayer {
+  const __nv_bfloat16 *wqkv, *wo, *wcq, *wco, *w1, *w2;
+  const float *bqkv, *bo, *bcq, *bco, *b1, *b2;
+  const float *ln1g, *ln1b, *ln2g, *ln2b, *ln3g, *ln3b;
+  __nv_bfloat16 *ks, *vs;   // this layer's self K/V cache [B_max][H][max_pos][64]
+};
+struct VfArgs {
+  const VfLayer* layers;    // [L], device memory
+  int L, d, H, F, V, max_pos, t_alloc, b_max, anchor, B;
+  int S;                    // cross-attention splits per (utterance, head)
+  int a_bytes, slot_bytes;  // shared-memory layout (vf_layout)
+  const __nv_bfloat16 *tok_emb, *pos_emb;
+  const float *lnf_g, *lnf_b;
+  RowPlan plan;
+  const int* kv_len;
+  const int* enc_len;
+  float *x, *q, *q_anchor, *ml, *part;
+  __nv_bfloat16 *att, *hbuf, *xf;
+  unsigned long long* row_key;
+  unsigned* bar_ctr;        // grid barrier counter, zeroed before the launch
+  int* tickets;             // [B_max * H] split merge tickets, zero between uses
+  int* status;
+  unsigned long long* tl;
+  unsigned long long* trace;   // per-stage timestamps [CTA][vf_trace_points(L)], or null
+};
+// Timestamps per CTA of a traced fused verify: 16 per layer (layer start, then
+// the end of each stage and of each grid barrier that follows it) + 2 (LM head
+// start and end).
+__host__ __device__ inline int vf_trace_points(int L) { return 16 * L + 2; }
+// Shared-memory layout for (d, F, L): activation/attention region, ring slot, total bytes.
+void vf_layout(int d, int F, int L, int* a_bytes, int* slot_bytes, int* total);
+// 0 when the kernel cannot run for these dimensions on this device.
+int vf_grid(int d, int F, int L);
+cudaError_t launch_verify_fused(const CUtensorMap* xmap, const VfArgs& a, int grid, cudaStream_t st);
+
 // ---- Accept / commit ------------------------------------------------------------
 void launch_prefill_advance(int B, int c, const int* n_utt_rows, int* kv_len, cudaStream_t st);
 void launch_prefill_finish(const int* prompt, int P0, int B, int* pending, const int* ready, cudaStream_t st);

@@ -56,6 +56,37 @@ def timeline_summary(ns, kinds, rounds):
     return "\n".join(lines)
 
 
+FUSED_INTERVALS = ["qkv", "barrier", "self_attn", "barrier", "self_out", "barrier", "cross_q", "barrier",
+                   "cross_attn", "barrier", "cross_out", "barrier", "mlp_up", "barrier", "mlp_down", "barrier"]
+
+
+def fused_trace_summary(tr):
+    """Per interval of a layer of the fused verify (trace [CTA][16 L + 2]):
+    the per-CTA duration (median and max over CTAs, mean over layers) and the
+    advance of the last CTA (max over CTAs of the end stamp minus that of the
+    start stamp, mean over layers), in us; then the LM head."""
+    tr = tr.astype(np.int64)
+    n_cta, per = tr.shape
+    L = (per - 2) // 16
+    lines = [f"  fused verify trace: {n_cta} CTAs, {L} layers, span {(tr.max() - tr[:, 0].min()) / 1e3:.1f} us"]
+    lines.append(f"  {'interval':<12}{'cta med':>9}{'cta max':>9}{'last->last':>12}")
+    tot = 0.0
+    for j in range(16):
+        med, mx, ll = [], [], []
+        for l in range(L):
+            a, b = tr[:, 16 * l + j], tr[:, 16 * l + j + 1]
+            dur = (b - a) / 1e3
+            med.append(np.median(dur))
+            mx.append(dur.max())
+            ll.append((b.max() - a.max()) / 1e3)
+        tot += np.mean(ll)
+        lines.append(f"  {FUSED_INTERVALS[j]:<12}{np.mean(med):>9.2f}{np.mean(mx):>9.2f}{np.mean(ll):>12.2f}")
+    lm = (tr[:, 16 * L + 1] - tr[:, 16 * L]) / 1e3
+    lines.append(f"  per layer (sum of last->last) {tot:.2f} us; LM head per CTA med {np.median(lm):.2f} "
+                 f"max {lm.max():.2f} us")
+    return "\n".join(lines)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--config", default="large-bf16-b1-k8", choices=sorted(W.CONFIGS))
@@ -66,6 +97,8 @@ def main():
                     help="also time each kernel class with CUDA events (direct launches)")
     ap.add_argument("--timeline", action="store_true",
                     help="also record the launch timeline of the rounds (direct launches) and summarise it per kind")
+    ap.add_argument("--fused-trace", action="store_true",
+                    help="also record the per-stage timestamps of one fused verify and summarise them")
     args = ap.parse_args()
 
     import torch
@@ -116,6 +149,12 @@ def main():
         ns, kinds = A.asr_spec_timeline_read(sess.h)
         A.asr_spec_timeline(sess.h, False)
         print(timeline_summary(ns, kinds, args.rounds))
+    if args.fused_trace:
+        A.asr_spec_fused_trace(sess.h, True)
+        sess.verify_device(drafts[0], lens, wl.k)
+        tr = A.asr_spec_fused_trace_read(sess.h)
+        A.asr_spec_fused_trace(sess.h, False)
+        print(fused_trace_summary(tr))
     sess.close()
     if st:
         sys.exit(1)
