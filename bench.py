@@ -41,6 +41,23 @@ BATCH1_CONFIG = "large-bf16-b1-k8"
 METRIC = "accepted tokens/s"
 
 
+def max_over_ranks(dist, x: float, device="cuda") -> float:
+    """The largest value of x over the ranks (every rank gets it): the slowest
+    replica's time bounds the whole job.  dist = torch.distributed or None."""
+    if dist is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, steps: int, tokens_per_step: int, seconds_max: float) -> float:
+    """Tokens of all replicas (weak scaling: each rank decodes its own batch)
+    divided by the slowest rank's time."""
+    return world * steps * tokens_per_step / seconds_max
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -321,14 +338,17 @@ class GpuRun:
         A.asr_spec_profile(self.sess.h, False)
         return ms, launches, traffic
 
-    def e2e(self, steps):
+    def e2e(self, steps, dist=None):
         """The same decodes through host buffers: encoder states copied from pinned
         host memory every step, drafts built on the host and passed with every
-        verify call, outputs read back every round."""
+        verify call, outputs read back every round.  Returns this rank's
+        seconds with the rest; the caller combines the ranks."""
         torch, A = self.torch, self.A
         s = self.sess
         wl = self.wl
         h2d = d2h = 0
+        if dist is not None:
+            dist.barrier()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         for _ in range(steps):
@@ -352,8 +372,10 @@ class GpuRun:
             del enc
         torch.cuda.synchronize()
         dt = time.perf_counter() - t0
+        if dist is not None:
+            dist.barrier()
         return dict(value=steps * self.tokens_per_decode / dt, unit="tokens/s",
-                    h2d_bytes_per_step=int(h2d // steps), d2h_bytes_per_step=int(d2h // steps))
+                    h2d_bytes_per_step=int(h2d // steps), d2h_bytes_per_step=int(d2h // steps), seconds=dt)
 
 
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one
@@ -603,13 +625,8 @@ def main():
     wl = W.CONFIGS[args.config]
     run = GpuRun(wl)
     res = run.timed(args.steps, args.warmup, dist, gpu_index=local)
-    ms = res["ms"]
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    total_tokens = world * args.steps * run.tokens_per_decode
-    value = total_tokens / (ms / 1e3)
+    ms = max_over_ranks(dist, res["ms"])
+    value = whole_job_rate(world, args.steps, run.tokens_per_decode, ms / 1e3)
     prof_ms, prof_launches, prof_traffic = run.profile()
     tl = run.launch_timeline()
     fixed = run.fixed_state()
@@ -631,9 +648,10 @@ def main():
         "roofline": roofline(wl.name, wl.dims, tl, prof_ms, prof_launches, prof_traffic, pk),
     })
     if not args.no_e2e:
-        line["e2e"] = run.e2e(max(1, min(args.steps, 2)))
-        if world > 1:
-            line["e2e"]["value"] *= world
+        e2e_steps = max(1, min(args.steps, 2))
+        e2e = run.e2e(e2e_steps, dist)
+        e2e["value"] = whole_job_rate(world, e2e_steps, run.tokens_per_decode, max_over_ranks(dist, e2e.pop("seconds")))
+        line["e2e"] = e2e
     if rank == 0:
         # CPU oracle on a bounded sample of the same workload
         tokens, dt, rounds, desc = oracle_sample(wl, run.truth, args.cpu_budget)
