@@ -97,6 +97,30 @@ def head_mean_attention(q: np.ndarray, K: np.ndarray, n_heads: int) -> np.ndarra
     return softmax(s).mean(axis=0)
 
 
+def visible_keys(pos: int) -> int:
+    """Self-attention keys a verification row at position pos sees: the
+    committed cache and every row of its own block up to itself (Sec. 3: the
+    target checks the whole block in one pass, each row causally)."""
+    return pos + 1
+
+
+def accepted_prefix(draft_b: np.ndarray, g_b: np.ndarray, lens_b: int) -> int:
+    """Longest prefix of the block kept by the target (Sec. 3 "Speculative
+    Loop"): draft j (0-based) stays while it equals the target's argmax at row
+    j, the row that scored the token before it (the pending token for j = 0)."""
+    n = 0
+    while n < lens_b and draft_b[n] == g_b[n]:
+        n += 1
+    return n
+
+
+def bonus_row(n: int) -> int:
+    """Row of the block whose argmax is the bonus token after n accepted
+    drafts: the row that scored the last accepted token (App. "Correction and
+    Cost": a round advances 1 + L tokens).  The anchor is read at this row."""
+    return n
+
+
 class OracleError(ValueError):
     pass
 
@@ -222,7 +246,8 @@ class Oracle:
                 self.Vs[l][b, ps] = v[r]
             o = np.empty_like(x)
             for r, (b, _, ps) in enumerate(rows):
-                o[r] = attention(q[r], self.Ks[l][b, :ps + 1], self.Vs[l][b, :ps + 1], H)
+                nk = visible_keys(ps)
+                o[r] = attention(q[r], self.Ks[l][b, :nk], self.Vs[l][b, :nk], H)
             x = x + o @ self.W(p + "wo").T + self.W(p + "bo")
             # cross-attention block over the utterance's encoder frames
             h = layer_norm(x, self.W(p + "ln2_g"), self.W(p + "ln2_b"))
@@ -290,15 +315,13 @@ class Oracle:
         for b in range(self.B):
             if lens[b] < 0:
                 continue
-            n = 0
-            # longest prefix: draft j is kept while it equals the argmax of row j-1
-            while n < lens[b] and draft[b, n] == g[r0 + n]:
-                n += 1
+            n = accepted_prefix(draft[b], g[r0:r0 + int(lens[b]) + 1], int(lens[b]))
             acc[b] = n
-            bonus[b] = g[r0 + n]
+            br = r0 + bonus_row(n)
+            bonus[b] = g[br]
             restart[b] = 1 if n < lens[b] else 0
             # re-anchor from the verification row that produced the bonus token
-            pbar = head_mean_attention(q_anchor[r0 + n], self.Kx[d.anchor][b], d.n_heads)
+            pbar = head_mean_attention(q_anchor[br], self.Kx[d.anchor][b], d.n_heads)
             prof[b] = pbar
             anchor[b] = int(np.argmax(pbar))
             self.kv_len[b] = self.kv_len[b] + 1 + n

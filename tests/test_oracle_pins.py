@@ -258,16 +258,47 @@ def _mut_head_mean_logits(q, K, n_heads):
     return D.softmax(s.mean(axis=0))
 
 
-@pytest.mark.parametrize("name,fn", [("gelu", _mut_gelu_tanh), ("layer_norm", _mut_ln_unbiased),
-                                     ("attention", _mut_attention_scale),
-                                     ("head_mean_attention", _mut_head_mean_logits)])
-def test_pins_catch_planted_mistakes(monkeypatch, name, fn):
-    """A plausible mistake planted in the oracle makes the library pins fail."""
+def _mut_prefix_shifted(draft_b, g_b, lens_b):
+    # compares draft j with the argmax of row j + 1 (the row that scored draft j itself)
+    n = 0
+    while n < lens_b and n + 1 < len(g_b) and draft_b[n] == g_b[n + 1]:
+        n += 1
+    return n
+
+
+def _mut_prefix_one_more(draft_b, g_b, lens_b):
+    # keeps the first mismatching draft too
+    n = 0
+    while n < lens_b and draft_b[n] == g_b[n]:
+        n += 1
+    return min(n + 1, lens_b)
+
+
+def _mut_keys_exclusive(pos):
+    return pos          # a row that cannot see its own key
+
+
+def _mut_bonus_row_next(n):
+    return n + 1        # reads the bonus from the row after the last accepted token
+
+
+@pytest.mark.parametrize("name,fn,pin", [
+    ("gelu", _mut_gelu_tanh, "rows"), ("layer_norm", _mut_ln_unbiased, "rows"),
+    ("attention", _mut_attention_scale, "rows"), ("head_mean_attention", _mut_head_mean_logits, "anchor"),
+    ("visible_keys", _mut_keys_exclusive, "rows"),
+    ("accepted_prefix", _mut_prefix_shifted, "accept"), ("accepted_prefix", _mut_prefix_one_more, "accept"),
+    ("bonus_row", _mut_bonus_row_next, "accept")])
+def test_pins_catch_planted_mistakes(monkeypatch, name, fn, pin):
+    """A plausible mistake planted in the oracle makes a pin fail: the library
+    decoder (rows), torch's head-averaged attention (anchor), or brute-force
+    enumeration of every draft block (accept)."""
     import oracle.decoder as D
     monkeypatch.setitem(D.__dict__, "_orig_attention", D.attention)
     monkeypatch.setattr(D, name, fn)
-    with pytest.raises(AssertionError):
-        if name == "head_mean_attention":
+    with pytest.raises((AssertionError, IndexError, ValueError)):
+        if pin == "anchor":
             test_anchor_matches_torch_head_mean_weights()
+        elif pin == "accept":
+            test_accept_brute_force_tiny_vocab()
         else:
             test_verify_rows_match_torch_decoder(0.3)
