@@ -87,6 +87,59 @@ def fused_trace_summary(tr):
     return "\n".join(lines)
 
 
+def batch_sweep(batches, k, rounds, warmup):
+    """Verification cost against batch size on the large decoder: the first B
+    utterances of the 64-utterance workload (ragged encoder lengths), k drafts
+    each, all rows scored; per round the CUDA-event time of the verify call
+    (graph replay) and, from the launch timeline, the time of the acceptance +
+    anchor-readout kernel, whose ratio to the verify call is the runtime
+    correction's cost on the scale of one target verification (the quantity
+    the paper's cost condition compares with the gain in accepted length)."""
+    import torch
+    from paper_2608_12703_gb300 import asrspec as A
+    from paper_2608_12703_gb300.session import Session
+    base = W.CONFIGS["large-bf16-b64-k6"]
+    dims = base.dims
+    blob = W.make_weights(dims)
+    rng = np.random.default_rng(5)
+    lines = [f"  {'batch':>6}{'rows':>6}{'verify us':>11}{'per utt us':>12}{'accept+anchor us':>18}{'readout / verify':>18}"]
+    for B in batches:
+        enc_lens = list(base.enc_lens[:B])
+        t_max = max(enc_lens)
+        sess = Session(dims, blob, max_batch=B, max_draft=k)
+        sess.encode_cache(W.make_encoder_states(dims, enc_lens, t_max), enc_lens)
+        sess.prefill(W.make_prompt(dims, B))
+        with torch.cuda.stream(sess.stream):
+            drafts = [torch.from_numpy(rng.integers(0, dims.vocab, size=(B, k)).astype(np.int32)).cuda()
+                      for _ in range(warmup + rounds)]
+            lens = torch.full((B,), k, dtype=torch.int32, device="cuda")
+        sess.stream.synchronize()
+        times = []
+        for i in range(warmup + rounds):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(sess.stream)
+            sess.verify_device(drafts[i], lens, k)
+            e1.record(sess.stream)
+            if i >= warmup:
+                times.append((e0, e1))
+        torch.cuda.synchronize()
+        us = float(np.median([a.elapsed_time(b) * 1e3 for a, b in times]))
+        A.asr_spec_timeline(sess.h, True)
+        for i in range(rounds):
+            sess.verify_device(drafts[i], lens, k)
+        ns, kinds = A.asr_spec_timeline_read(sess.h)
+        A.asr_spec_timeline(sess.h, False)
+        ns = ns.astype(np.int64)
+        acc = ns[kinds == 6]
+        acc_us = float(np.median((acc[:, 3] - np.where(acc[:, 1] > 0, acc[:, 1], acc[:, 0])) / 1e3))
+        st = sess.status()
+        sess.close()
+        if st:
+            raise RuntimeError(f"status {st} at batch {B}")
+        lines.append(f"  {B:>6}{B * (k + 1):>6}{us:>11.1f}{us / B:>12.1f}{acc_us:>18.2f}{acc_us / us:>18.4f}")
+    return "\n".join(lines)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--config", default="large-bf16-b1-k8", choices=sorted(W.CONFIGS))
@@ -99,7 +152,18 @@ def main():
                     help="also record the launch timeline of the rounds (direct launches) and summarise it per kind")
     ap.add_argument("--fused-trace", action="store_true",
                     help="also record the per-stage timestamps of one fused verify and summarise them")
+    ap.add_argument("--batch-sweep", default="",
+                    help="comma-separated batch sizes: verification cost and anchor-readout share of the large "
+                         "decoder at each (replaces the single-workload run)")
+    ap.add_argument("--k", type=int, default=6, help="drafts per utterance of --batch-sweep")
     args = ap.parse_args()
+    if args.batch_sweep:
+        from paper_2608_12703_gb300 import build as B
+        B.build()
+        batches = [int(b) for b in args.batch_sweep.split(",")]
+        print(f"large decoder, k = {args.k}, median of {args.rounds} verify rounds after {args.warmup} warm-up:")
+        print(batch_sweep(batches, args.k, args.rounds, args.warmup))
+        return
 
     import torch
     from paper_2608_12703_gb300 import asrspec as A
