@@ -104,6 +104,13 @@ def visible_keys(pos: int) -> int:
     return pos + 1
 
 
+def tree_keys(P: int, ancestors: List[int]) -> List[int]:
+    """Cache slots a tree node attends to: the committed cache [0, P) and the
+    slots P + a of its ancestors a (root first, the node itself last); the
+    tree attention mask of the tree decoder control."""
+    return list(range(P)) + [P + a for a in ancestors]
+
+
 def accepted_prefix(draft_b: np.ndarray, g_b: np.ndarray, lens_b: int) -> int:
     """Longest prefix of the block kept by the target (Sec. 3 "Speculative
     Loop"): draft j (0-based) stays while it equals the target's argmax at row
@@ -137,6 +144,7 @@ class VerifyResult:
     argmax: np.ndarray        # [R] greedy token of every row
     top2_gap: np.ndarray      # [R] top-1 minus top-2 logit
     anchor_profile: Dict[int, np.ndarray]  # b -> head-mean attention over frames
+    path: Optional[np.ndarray] = None       # tree verify: [B][n] accepted nodes by depth (-1 past the path)
 
 
 class Oracle:
@@ -222,7 +230,10 @@ class Oracle:
         """Run the decoder on rows (b, token, position), writing each row's
         self-attention K/V at its position first, so that a row attends to the
         committed cache plus every earlier row of its own block and itself:
-        the block-causal mask of one verification pass (Sec. 3).
+        the block-causal mask of one verification pass (Sec. 3).  A row may
+        also be (b, token, position, slot, keys): its K/V go to cache slot
+        `slot` and it attends to the cache slots `keys` (a tree node: the
+        committed cache, its ancestors and itself).
 
         Returns final-LN logits [R, V] (if asked) and each row's cross-attention
         query at the anchor layer.
@@ -231,6 +242,7 @@ class Oracle:
         H = d.n_heads
         tok = np.array([r[1] for r in rows], dtype=np.int64)
         pos = np.array([r[2] for r in rows], dtype=np.int64)
+        slot = [r[3] if len(r) > 3 else r[2] for r in rows]
         bidx = [r[0] for r in rows]
         x = self.W("tok_emb")[tok] + self.W("pos_emb")[pos]
         q_anchor = None
@@ -241,13 +253,18 @@ class Oracle:
             q = h @ self.W(p + "wq").T + self.W(p + "bq")
             k = h @ self.W(p + "wk").T
             v = h @ self.W(p + "wv").T + self.W(p + "bv")
-            for r, (b, _, ps) in enumerate(rows):
-                self.Ks[l][b, ps] = k[r]
-                self.Vs[l][b, ps] = v[r]
+            for r, b in enumerate(bidx):
+                self.Ks[l][b, slot[r]] = k[r]
+                self.Vs[l][b, slot[r]] = v[r]
             o = np.empty_like(x)
-            for r, (b, _, ps) in enumerate(rows):
-                nk = visible_keys(ps)
-                o[r] = attention(q[r], self.Ks[l][b, :nk], self.Vs[l][b, :nk], H)
+            for r, row in enumerate(rows):
+                b = row[0]
+                if len(row) > 3:
+                    keys = row[4]
+                    o[r] = attention(q[r], self.Ks[l][b, keys], self.Vs[l][b, keys], H)
+                else:
+                    nk = visible_keys(row[2])
+                    o[r] = attention(q[r], self.Ks[l][b, :nk], self.Vs[l][b, :nk], H)
             x = x + o @ self.W(p + "wo").T + self.W(p + "bo")
             # cross-attention block over the utterance's encoder frames
             h = layer_norm(x, self.W(p + "ln2_g"), self.W(p + "ln2_b"))
@@ -329,6 +346,93 @@ class Oracle:
             r0 += int(lens[b]) + 1
         return VerifyResult(acc, bonus, self.kv_len.copy(), anchor, restart, row_ids,
                             logits, g, gap, prof)
+
+    def verify_tree(self, tokens, parent, lens) -> VerifyResult:
+        """Score a candidate tree per utterance in one pass under a tree mask
+        (App. "Alternative draft and verification changes", tree decoder):
+        node 0 is the pending token, node i + 1 has token tokens[b][i] and
+        parent parent[b][i] in [0, i]; lens[b] nodes are used (-1: sits out).
+        Node j is scored at position kv_len + depth(j), its K/V in cache slot
+        kv_len + j, attending to the committed cache and to its ancestors
+        (itself included).  The accepted path starts at the root and moves to
+        the first child (lowest index) whose token is the argmax of the current
+        node; the bonus is the argmax of its last node, which is also the
+        anchor row.  The path's K/V move to positions kv_len + 1 .. + n in
+        depth order.  The result carries `path` [B][n] (-1 past the path)."""
+        d = self.dims
+        if self.kv_len is None:
+            raise OracleError("verify before prefill")
+        tokens = np.asarray(tokens, dtype=np.int64).reshape(self.B, -1)
+        parent = np.asarray(parent, dtype=np.int64).reshape(self.B, -1)
+        lens = np.asarray(lens, dtype=np.int64)
+        n_max = tokens.shape[1]
+        if lens.shape != (self.B,) or np.any(lens < -1) or np.any(lens > n_max):
+            raise OracleError("lens out of range")
+        rows, row_ids, kids = [], [], {}
+        for b in range(self.B):
+            if lens[b] < 0:
+                continue
+            l = int(lens[b])
+            if self.kv_len[b] + l + 1 > d.max_pos:
+                raise OracleError("decoder context capacity exceeded")
+            self._check_tokens(tokens[b, :l])
+            par = [-1] + [int(p) for p in parent[b, :l]]
+            if any(par[j] < 0 or par[j] >= j for j in range(1, l + 1)):
+                raise OracleError("a parent outside [0, node)")
+            P = int(self.kv_len[b])
+            depth = [0] * (l + 1)
+            anc = [[0]] + [None] * l
+            for j in range(1, l + 1):
+                depth[j] = depth[par[j]] + 1
+                anc[j] = anc[par[j]] + [j]
+            kids[b] = [[j for j in range(1, l + 1) if par[j] == c] for c in range(l + 1)]
+            for j in range(l + 1):
+                t = int(self.pending[b]) if j == 0 else int(tokens[b, j - 1])
+                keys = tree_keys(P, anc[j])
+                rows.append((b, t, P + depth[j], P + j, keys))
+                row_ids.append((b, j))
+        if rows:
+            logits, q_anchor = self._forward(rows, want_logits=True)
+        else:
+            logits, q_anchor = np.zeros((0, d.vocab)), np.zeros((0, d.d_model))
+        g = np.argmax(logits, axis=1) if rows else np.zeros(0, dtype=np.int64)
+        srt = np.sort(logits, axis=1)[:, -2:] if rows else np.zeros((0, 2))
+        gap = srt[:, 1] - srt[:, 0]
+        acc = np.zeros(self.B, dtype=np.int64)
+        bonus = np.full(self.B, -1, dtype=np.int64)
+        anchor = np.full(self.B, -1, dtype=np.int64)
+        restart = np.zeros(self.B, dtype=np.int64)
+        path = np.full((self.B, n_max), -1, dtype=np.int64)
+        prof: Dict[int, np.ndarray] = {}
+        r0 = 0
+        for b in range(self.B):
+            if lens[b] < 0:
+                continue
+            c, n = 0, 0
+            while True:
+                nxt = [j for j in kids[b][c] if int(tokens[b, j - 1]) == int(g[r0 + c])]
+                if not nxt:
+                    break
+                c = nxt[0]
+                path[b, n] = c
+                n += 1
+            acc[b] = n
+            bonus[b] = g[r0 + c]
+            restart[b] = 1 if kids[b][c] else 0
+            pbar = head_mean_attention(q_anchor[r0 + c], self.Kx[d.anchor][b], d.n_heads)
+            prof[b] = pbar
+            anchor[b] = int(np.argmax(pbar))
+            P = int(self.kv_len[b])
+            for j in range(n):   # the accepted path to consecutive positions, in depth order
+                for l_ in range(d.n_layers):
+                    self.Ks[l_][b, P + j + 1] = self.Ks[l_][b, P + path[b, j]]
+                    self.Vs[l_][b, P + j + 1] = self.Vs[l_][b, P + path[b, j]]
+            self.kv_len[b] = P + 1 + n
+            self.pending[b] = bonus[b]
+            r0 += int(lens[b]) + 1
+        res = VerifyResult(acc, bonus, self.kv_len.copy(), anchor, restart, row_ids, logits, g, gap, prof)
+        res.path = path
+        return res
 
     def rollback(self, new_len, new_pending) -> None:
         """Truncate the committed cache to new_len[b] <= kv_len[b] and set the

@@ -282,12 +282,17 @@ def _mut_bonus_row_next(n):
     return n + 1        # reads the bonus from the row after the last accepted token
 
 
+def _mut_tree_keys_block_causal(P, ancestors):
+    return list(range(P + ancestors[-1] + 1))   # every earlier node, siblings included
+
+
 @pytest.mark.parametrize("name,fn,pin", [
     ("gelu", _mut_gelu_tanh, "rows"), ("layer_norm", _mut_ln_unbiased, "rows"),
     ("attention", _mut_attention_scale, "rows"), ("head_mean_attention", _mut_head_mean_logits, "anchor"),
     ("visible_keys", _mut_keys_exclusive, "rows"),
     ("accepted_prefix", _mut_prefix_shifted, "accept"), ("accepted_prefix", _mut_prefix_one_more, "accept"),
-    ("bonus_row", _mut_bonus_row_next, "accept")])
+    ("bonus_row", _mut_bonus_row_next, "accept"),
+    ("tree_keys", _mut_tree_keys_block_causal, "tree")])
 def test_pins_catch_planted_mistakes(monkeypatch, name, fn, pin):
     """A plausible mistake planted in the oracle makes a pin fail: the library
     decoder (rows), torch's head-averaged attention (anchor), or brute-force
@@ -300,5 +305,116 @@ def test_pins_catch_planted_mistakes(monkeypatch, name, fn, pin):
             test_anchor_matches_torch_head_mean_weights()
         elif pin == "accept":
             test_accept_brute_force_tiny_vocab()
+        elif pin == "tree":
+            test_tree_nodes_equal_linear_branches()
         else:
             test_verify_rows_match_torch_decoder(0.3)
+
+
+# ---- tree verification (App. "Alternative draft and verification changes": the
+# target verifies a candidate tree in one pass under a tree attention mask) ----
+
+def _random_tree(rng, n, vocab):
+    parent = np.array([rng.integers(0, i + 1) for i in range(n)])
+    tokens = rng.integers(0, vocab, size=n)
+    return tokens, parent
+
+
+def _branch(parent, j):
+    """Nodes on the way from the root to node j (excluded root), root first."""
+    out = []
+    while j > 0:
+        out.append(j)
+        j = parent[j - 1]
+    return out[::-1]
+
+
+def test_tree_one_branch_equals_linear_verify():
+    """A one-branch tree reproduces the linear verify token for token: outputs,
+    logits and the committed cache are identical."""
+    o, *_ = _setup()
+    rng = np.random.default_rng(11)
+    for _ in range(3):
+        snap = o.snapshot()
+        draft = rng.integers(0, TINY.vocab, size=(3, 4))
+        lens = np.array([4, 2, -1])
+        lin = o.verify(draft, lens)
+        s_lin = o.snapshot()
+        o.restore(snap)
+        chain = np.tile(np.arange(4), (3, 1))      # parent of node i + 1 is node i
+        tr = o.verify_tree(draft, chain, lens)
+        s_tr = o.snapshot()
+        for f in ("accepted", "bonus", "kv_len", "anchor", "restart"):
+            assert np.array_equal(getattr(lin, f), getattr(tr, f)), f
+        assert np.array_equal(lin.logits, tr.logits)
+        for b in range(3):
+            n = int(lin.accepted[b]) if lens[b] >= 0 else 0
+            assert list(tr.path[b, :n]) == list(range(1, n + 1))
+        for l in range(TINY.n_layers):
+            for b in range(3):
+                kv = int(s_lin[2][b])
+                assert np.array_equal(s_lin[0][l][b, :kv], s_tr[0][l][b, :kv])
+                assert np.array_equal(s_lin[1][l][b, :kv], s_tr[1][l][b, :kv])
+
+
+def test_tree_nodes_equal_linear_branches():
+    """Every node's logits are those of the linear verify of its branch (root to
+    node) from the same state; the accepted path is as long as the longest
+    accepted branch, with its bonus; the committed cache equals the one the
+    linear verify of the accepted path leaves."""
+    o, *_ = _setup()
+    rng = np.random.default_rng(12)
+    for step in range(3):
+        snap = o.snapshot()
+        g = _greedy_continuation(o, 4)             # true continuation, to make paths long
+        n = 11
+        tokens, parent = np.zeros((3, n), dtype=np.int64), np.zeros((3, n), dtype=np.int64)
+        for b in range(3):
+            tokens[b], parent[b] = _random_tree(rng, n, TINY.vocab)
+            parent[b, :3] = [0, 1, 2]              # a branch along the true continuation
+            tokens[b, :3] = g[b, :3]
+            if step == 1:
+                tokens[b, 5] = tokens[b, 1]        # a duplicate of a true token elsewhere
+        lens = np.array([n, 7, n])
+        tr = o.verify_tree(tokens, parent, lens)
+        s_tr = o.snapshot()
+        r0 = 0
+        for b in range(3):
+            l = int(lens[b])
+            best = (-1, None)
+            for j in range(l + 1):
+                nodes = _branch(parent[b], j)
+                o.restore(snap)
+                dr = np.zeros((3, max(len(nodes), 1)), dtype=np.int64)
+                dr[b, :len(nodes)] = tokens[b, np.array(nodes, dtype=int) - 1] if nodes else []
+                ln = np.full(3, -1)
+                ln[b] = len(nodes)
+                lin = o.verify(dr, ln)
+                # (the tree pass multiplies more rows at once: BLAS may sum in another order)
+                np.testing.assert_allclose(tr.logits[r0 + j], lin.logits[len(nodes)], rtol=0, atol=1e-12)
+                if lin.accepted[b] > best[0]:
+                    best = (int(lin.accepted[b]), int(lin.bonus[b]))
+            assert tr.accepted[b] == best[0] and tr.bonus[b] == best[1]
+            # the cache the tree verify committed is the linear verify's of the accepted path
+            path = [int(x) for x in tr.path[b, :tr.accepted[b]]]
+            o.restore(snap)
+            dr = np.zeros((3, max(len(path), 1)), dtype=np.int64)
+            dr[b, :len(path)] = tokens[b, np.array(path, dtype=int) - 1] if path else []
+            ln = np.full(3, -1)
+            ln[b] = len(path)
+            lin = o.verify(dr, ln)
+            assert lin.accepted[b] == len(path) and lin.bonus[b] == tr.bonus[b]
+            s_lin = o.snapshot()
+            kv = int(s_tr[2][b])
+            assert kv == int(s_lin[2][b])
+            for l_ in range(TINY.n_layers):
+                np.testing.assert_allclose(s_lin[0][l_][b, :kv], s_tr[0][l_][b, :kv], rtol=0, atol=1e-12)
+                np.testing.assert_allclose(s_lin[1][l_][b, :kv], s_tr[1][l_][b, :kv], rtol=0, atol=1e-12)
+            r0 += l + 1
+        o.restore(s_tr)
+
+
+def test_tree_errors():
+    o, *_ = _setup()
+    with pytest.raises(OracleError):
+        o.verify_tree(np.zeros((3, 2), dtype=int), np.array([[0, 2], [0, 0], [0, 0]]), np.array([2, 2, 2]))
