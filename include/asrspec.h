@@ -62,6 +62,7 @@ extern "C" {
 #define ASR_ST_CAPACITY 4       /* kv_len[b] + lens[b] + 1 > max_pos, or enc_len out of range */
 #define ASR_ST_WAIT_TIMEOUT 8   /* a bounded pipeline wait gave up; results of that call are invalid */
 #define ASR_ST_NOT_READY 16     /* an utterance slot without an encoder cache or prefill */
+#define ASR_ST_BAD_TREE 32      /* tree verify: a node's parent outside [0, node) */
 
 typedef struct asr_spec* asr_spec_handle;
 
@@ -137,6 +138,31 @@ int asr_spec_prefill(asr_spec_handle h, const int32_t* prompt, int32_t P0);
  * status word. */
 int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens, int32_t k,
                     int32_t* accepted, int32_t* bonus, int32_t* kv_len, int32_t* anchor);
+
+/* One verification round over a candidate tree per utterance (the tree
+ * decoder control of App. "Alternative draft and verification changes": the
+ * target verifies every node in one pass under a tree attention mask).
+ *   tokens [B][n] int32: token of node i + 1 (node 0 is the pending token);
+ *   parent [B][n] int32: parent of node i + 1, in [0, i] (topological order);
+ *   lens   [B] int32: nodes used 0..n, or -1 for an utterance that sits out.
+ * Node i is scored at position kv_len[b] + depth(i) and attends to the
+ * committed cache and to its ancestors (itself included); its K/V go to cache
+ * slot kv_len[b] + i.  With g_i the argmax of node i, the accepted path starts
+ * at the root and moves to the first child (lowest node index) whose token is
+ * g of the current node, while there is one:
+ *   accepted[b] = its length n; bonus[b] = g of its last node;
+ *   path[b][j]  = the node at depth j + 1 (j < n), -1 past it ([B][n] int32);
+ *   the path's K/V move to positions kv_len[b] + 1 .. + n (the committed cache
+ *   is then what the linear verify of that path would leave); kv_len, pending
+ *   and the anchor (read at the path's last node) as asr_spec_verify.
+ * A one-branch tree (parent[b][i] = i) is the linear verify.  n <= 31.
+ * Errors: ASR_E_INVAL (n outside [0, min(max_draft, 31)], fp32 model),
+ * ASR_E_STATE (no prefill).  Data errors (token id, a parent outside
+ * [0, node), lens, capacity kv_len + lens + 1 > max_pos) skip the whole step and
+ * set the status word (ASR_ST_BAD_TREE for a parent). */
+int asr_spec_verify_tree(asr_spec_handle h, const int32_t* tokens, const int32_t* parent, const int32_t* lens,
+                         int32_t n, int32_t* accepted, int32_t* bonus, int32_t* kv_len, int32_t* anchor,
+                         int32_t* path);
 
 /* Roll the committed cache back (App. "Decoding and Intervention Protocol":
  * the cached states of accepted tokens are what the next round reuses):

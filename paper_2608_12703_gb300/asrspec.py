@@ -20,7 +20,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libasrspec.so")
 ASR_OK = 0
 ERRORS = {-1: "ASR_E_INVAL", -2: "ASR_E_STATE", -3: "ASR_E_CAPACITY", -4: "ASR_E_OOM",
           -5: "ASR_E_CUDA", -6: "ASR_E_DEVICE"}
-ST_BAD_TOKEN, ST_BAD_LENS, ST_CAPACITY, ST_WAIT_TIMEOUT, ST_NOT_READY = 1, 2, 4, 8, 16
+ST_BAD_TOKEN, ST_BAD_LENS, ST_CAPACITY, ST_WAIT_TIMEOUT, ST_NOT_READY, ST_BAD_TREE = 1, 2, 4, 8, 16, 32
 
 EXPORTED = [
     "asr_spec_create", "asr_spec_set_host_io", "asr_spec_encode_cache", "asr_spec_prefill",
@@ -28,7 +28,7 @@ EXPORTED = [
     "asr_spec_status", "asr_spec_last_error", "asr_spec_destroy", "asr_spec_synth_drafts",
     "asr_spec_test_gemm", "asr_spec_set_graphs", "asr_spec_profile", "asr_spec_profile_read",
     "asr_spec_gemm_noalloc", "asr_spec_timeline", "asr_spec_timeline_read",
-    "asr_spec_fused_trace", "asr_spec_fused_trace_read",
+    "asr_spec_fused_trace", "asr_spec_fused_trace_read", "asr_spec_verify_tree",
 ]
 PROF_CLASSES = ["qkv", "resid", "query", "mlp_up", "self_attn", "cross_attn", "lm_head", "layernorm", "other",
                 "fused"]
@@ -79,6 +79,7 @@ def lib():
     L.asr_spec_encode_cache.argtypes = [vp, i32, vp, i32, p32]
     L.asr_spec_prefill.argtypes = [vp, p32, i32]
     L.asr_spec_verify.argtypes = [vp, p32, p32, i32, p32, p32, p32, p32]
+    L.asr_spec_verify_tree.argtypes = [vp, p32, p32, p32, i32, p32, p32, p32, p32, p32]
     L.asr_spec_rollback.argtypes = [vp, p32, p32]
     L.asr_spec_state.argtypes = [vp, p32, p32]
     L.asr_spec_debug_logits.argtypes = [vp, vp, i32]
@@ -150,6 +151,11 @@ def asr_spec_prefill(h, prompt, P0):
 def asr_spec_verify(h, draft, lens, k, accepted, bonus, kv_len, anchor):
     return _check(h, lib().asr_spec_verify(h, ptr(draft), ptr(lens), k, ptr(accepted), ptr(bonus),
                                            ptr(kv_len), ptr(anchor)), "asr_spec_verify")
+
+
+def asr_spec_verify_tree(h, tokens, parent, lens, n, accepted, bonus, kv_len, anchor, path):
+    return _check(h, lib().asr_spec_verify_tree(h, ptr(tokens), ptr(parent), ptr(lens), n, ptr(accepted), ptr(bonus),
+                                                ptr(kv_len), ptr(anchor), ptr(path)), "asr_spec_verify_tree")
 
 
 def asr_spec_rollback(h, new_len, new_pending):

@@ -98,6 +98,10 @@ struct asr_spec {
   int* vf_tickets = nullptr;
   float* vf_part = nullptr;
   bool last_fused = false;    // the last verify ran the fused kernel (LM-head input in xf)
+  // tree verify: the nodes' parents and the accepted path ([B_max][max_draft]),
+  // and whether the step being enqueued is one
+  int *parent_buf = nullptr, *path_buf = nullptr;
+  bool cur_tree = false;
   unsigned long long* vf_trace = nullptr;   // per-stage timestamps of the fused kernel (diagnostics)
   bool vf_trace_on = false;
   bool use_mc = false;        // multicast weight tiles across the row tiles (ASRSPEC_MC=1; slower as measured)
@@ -421,10 +425,12 @@ int run_layers(asr_spec* h, int N) {
     a.out_bf16 = h->bf16;
     a.ml_out = nullptr;
     a.rows_max = rows_max;
+    a.tree = h->cur_tree;
     {
       Prof p(h, ASR_PROF_SELF, h->bf16 ? 1 : 2);
       attention(h, a, true, l);
     }
+    a.tree = false;
     e = base;
     e.bias = w.bo;
     e.x = h->x;
@@ -495,10 +501,10 @@ int enqueue_verify(asr_spec* h, int k) {
     Tl t(h, ASR_TL_PLAN);
     TrafficArgs tr{h->counters, h->enc_len, h->L, h->d, (int)h->es};
     launch_plan_verify(h->draft_buf, h->lens_buf, k, B, h->V, h->maxpos, h->kv_len, h->pending, h->ready, h->plan,
-                       h->row_key, h->status, tr, h->st, h->tl_cur);
+                       h->row_key, h->status, tr, h->st, h->tl_cur, h->cur_tree ? h->parent_buf : nullptr);
   }
   const int N = B * (k + 1);
-  h->last_fused = h->vf_G > 0 && N <= VF_ROWS && B <= h->vf_bmax;
+  h->last_fused = h->vf_G > 0 && N <= VF_ROWS && B <= h->vf_bmax && !h->cur_tree;
   if (h->last_fused) {   // few rows: one persistent kernel for the layers and the LM head
     CK(cudaMemsetAsync(h->vf_bar, 0, 4, h->st));
     VfArgs a{};
@@ -576,9 +582,20 @@ int enqueue_verify(asr_spec* h, int k) {
   A.tickets = reinterpret_cast<int*>(h->frame_key + h->Bmax);
   A.status = h->status;
   A.pdl = h->use_pdl;
-  Tl t(h, ASR_TL_ACCEPT);
-  A.tl = h->tl_cur;
-  launch_accept_anchor(A, h->st);
+  if (h->cur_tree) {
+    A.parent = h->parent_buf;
+    A.path = h->path_buf;
+  }
+  {
+    Tl t(h, ASR_TL_ACCEPT);
+    A.tl = h->tl_cur;
+    launch_accept_anchor(A, h->st);
+  }
+  if (h->cur_tree) {   // the accepted path's K/V to consecutive positions
+    Prof p2(h, ASR_PROF_OTHER, 1);
+    launch_tree_commit(h->path_buf, k, h->out4, h->kv_len, B, h->L, h->H, h->maxpos, h->Bmax, h->kself, h->vself,
+                       (int)h->es, h->st);
+  }
   return 0;
 }
 
@@ -793,6 +810,7 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   if ((rc = dalloc(h, &h->part, (size_t)h->Bmax * h->H * n_chunks * (h->kmax + 1) * 66 * 4))) return finish(rc);
   if ((rc = dalloc(h, &h->plan.row_b, R * 4)) || (rc = dalloc(h, &h->plan.row_i, R * 4)) ||
       (rc = dalloc(h, &h->plan.row_pos, R * 4)) || (rc = dalloc(h, &h->plan.row_tok, R * 4)) ||
+      (rc = dalloc(h, &h->plan.row_epos, R * 4)) || (rc = dalloc(h, &h->plan.row_mask, R * 4)) ||
       (rc = dalloc(h, &h->plan.row_start, (h->Bmax + 1) * 4)) || (rc = dalloc(h, &h->plan.n_rows, 4)) ||
       (rc = dalloc(h, &h->plan.n_utt_rows, h->Bmax * 4)))
     return finish(rc);
@@ -801,6 +819,9 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
       (rc = dalloc(h, &h->anchor_row, h->Bmax * 4)))
     return finish(rc);
   CK(cudaMemset(h->frame_key, 0, h->Bmax * 12));
+  if ((rc = dalloc(h, &h->parent_buf, (size_t)h->Bmax * std::max(h->kmax, 1) * 4)) ||
+      (rc = dalloc(h, &h->path_buf, (size_t)h->Bmax * std::max(h->kmax, 1) * 4)))
+    return finish(rc);
   if ((rc = dalloc(h, &h->draft_buf, (size_t)h->Bmax * std::max(h->kmax, 1) * 4)) ||
       (rc = dalloc(h, &h->lens_buf, h->Bmax * 4)) || (rc = dalloc(h, &h->prompt_buf, (size_t)h->Bmax * h->maxpos * 4)) ||
       (rc = dalloc(h, &h->out4, 4 * h->Bmax * 4)) || (rc = dalloc(h, &h->misc, 64 * 4)) ||
@@ -937,21 +958,28 @@ int asr_spec_prefill(asr_spec_handle h, const int32_t* prompt, int32_t P0) {
   return ASR_OK;
 }
 
-int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens, int32_t k, int32_t* accepted,
-                    int32_t* bonus, int32_t* kv_len, int32_t* anchor) {
-  if (!h) return ASR_E_INVAL;
-  if (h->state < 2) return fail(h, ASR_E_STATE, "verify before prefill");
-  if (k < 0 || k > h->kmax) return fail(h, ASR_E_INVAL, "k outside [0, max_draft]");
-  if (!lens || (k > 0 && !draft) || !accepted || !bonus || !kv_len || !anchor)
-    return fail(h, ASR_E_INVAL, "null pointer");
+namespace {
+
+// The verify call: inputs into the internal buffers, the body (a CUDA graph per
+// (B, k, linear or tree), captured on first use), outputs out.
+int verify_call(asr_spec* h, const int32_t* draft, const int32_t* parent, const int32_t* lens, int32_t k,
+                int32_t* accepted, int32_t* bonus, int32_t* kv_len, int32_t* anchor, int32_t* path) {
+  const bool tree = parent != nullptr;
   const int B = h->B;
   if (k > 0) {
     if (int rc = copy_in(h, h->draft_buf, draft, (size_t)B * k)) return rc;
+    if (tree)
+      if (int rc = copy_in(h, h->parent_buf, parent, (size_t)B * k)) return rc;
   }
   if (int rc = copy_in(h, h->lens_buf, lens, B)) return rc;
   for (int c = 0; c < ASR_PROF_N; ++c) h->cur[c] = 0;
+  struct TreeScope {   // the enqueued layers read cur_tree; cleared on every way out
+    asr_spec* h;
+    ~TreeScope() { h->cur_tree = false; }
+  } scope{h};
+  h->cur_tree = tree;
   if (h->use_graphs && !h->prof && !h->tl_on && !h->vf_trace_on) {
-    auto key = std::make_pair(B, (int)k);
+    auto key = std::make_pair(B, tree ? 1000 + (int)k : (int)k);
     auto it = h->graphs.find(key);
     if (it == h->graphs.end()) {
       cudaGraph_t graph;
@@ -986,8 +1014,34 @@ int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens
   if (int rc = copy_out(h, bonus, o + h->Bmax, B)) return rc;
   if (int rc = copy_out(h, kv_len, o + 2 * h->Bmax, B)) return rc;
   if (int rc = copy_out(h, anchor, o + 3 * h->Bmax, B)) return rc;
+  if (tree && path && k > 0)
+    if (int rc = copy_out(h, path, h->path_buf, (size_t)B * k)) return rc;
   if (h->host_io) CK(cudaStreamSynchronize(h->st));
   return ASR_OK;
+}
+
+}  // namespace
+
+int asr_spec_verify(asr_spec_handle h, const int32_t* draft, const int32_t* lens, int32_t k, int32_t* accepted,
+                    int32_t* bonus, int32_t* kv_len, int32_t* anchor) {
+  if (!h) return ASR_E_INVAL;
+  if (h->state < 2) return fail(h, ASR_E_STATE, "verify before prefill");
+  if (k < 0 || k > h->kmax) return fail(h, ASR_E_INVAL, "k outside [0, max_draft]");
+  if (!lens || (k > 0 && !draft) || !accepted || !bonus || !kv_len || !anchor)
+    return fail(h, ASR_E_INVAL, "null pointer");
+  return verify_call(h, draft, nullptr, lens, k, accepted, bonus, kv_len, anchor, nullptr);
+}
+
+int asr_spec_verify_tree(asr_spec_handle h, const int32_t* tokens, const int32_t* parent, const int32_t* lens,
+                         int32_t n, int32_t* accepted, int32_t* bonus, int32_t* kv_len, int32_t* anchor,
+                         int32_t* path) {
+  if (!h) return ASR_E_INVAL;
+  if (h->state < 2) return fail(h, ASR_E_STATE, "verify before prefill");
+  if (!h->bf16) return fail(h, ASR_E_INVAL, "tree verify needs a bf16 model");
+  if (n < 0 || n > h->kmax || n > 31) return fail(h, ASR_E_INVAL, "n outside [0, min(max_draft, 31)]");
+  if (!lens || (n > 0 && (!tokens || !parent || !path)) || !accepted || !bonus || !kv_len || !anchor)
+    return fail(h, ASR_E_INVAL, "null pointer");
+  return verify_call(h, tokens, n > 0 ? parent : nullptr, lens, n, accepted, bonus, kv_len, anchor, path);
 }
 
 int asr_spec_set_graphs(asr_spec_handle h, int enable) {

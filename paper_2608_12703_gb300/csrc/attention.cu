@@ -218,7 +218,7 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
   __shared__ float ph[ANCHOR_HMAX][FB + 1];
   __shared__ float sM[ANCHOR_HMAX], sL[ANCHOR_HMAX];
   __shared__ __align__(8) uint64_t bar;
-  __shared__ int s_n, s_last;
+  __shared__ int s_n, s_node, s_last;
   tl_mark(A.tl, TL_ENTRY);
   const int b = blockIdx.y, f0 = blockIdx.x * FB, tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
@@ -245,6 +245,8 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
   pdl_launch();
   const int nr = A.plan.n_utt_rows[b];
   if (nr == 0) {                                      // uniform over the utterance's CTAs
+    if (blockIdx.x == 0 && tid == 0 && A.path != nullptr)
+      for (int j = 0; j < A.k; ++j) A.path[(size_t)b * A.k + j] = -1;
     if (blockIdx.x == 0 && tid == 0) {
       A.accepted[b] = 0;
       A.bonus[b] = -1;
@@ -256,7 +258,40 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
     return;
   }
   const int r0 = A.plan.row_start[b];
-  if (warp == 0) {
+  if (warp == 0 && A.parent != nullptr) {
+    // tree: from the root, follow the first child whose token is the target's
+    // argmax at its parent; n accepted nodes, the bonus is the argmax at the
+    // last of them (lane j < nr holds node j: its argmax, and for j >= 1 its
+    // token and parent)
+    const int l = nr - 1;
+    const unsigned long long key = lane < nr ? A.row_key[r0 + lane] : 0ull;
+    const int tok = (int)argmax_index(key);
+    const int my_tok = (lane >= 1 && lane <= l) ? A.draft[(size_t)b * A.k + lane - 1] : -1;
+    const int my_par = (lane >= 1 && lane <= l) ? A.parent[(size_t)b * A.k + lane - 1] : -1;
+    int c = 0, n = 0;
+    while (true) {   // at most l steps: every step moves to a deeper node
+      const int g = __shfl_sync(0xffffffffu, tok, c);
+      const unsigned hit = __ballot_sync(0xffffffffu, my_par == c && my_tok == g);
+      if (hit == 0u) break;
+      c = __ffs(hit) - 1;
+      if (lane == 0 && blockIdx.x == 0) A.path[(size_t)b * A.k + n] = c;
+      ++n;
+    }
+    const int g = __shfl_sync(0xffffffffu, tok, c);
+    if (lane == 0) {
+      s_n = n;
+      s_node = c;
+      if (blockIdx.x == 0) {
+        for (int j = n; j < A.k; ++j) A.path[(size_t)b * A.k + j] = -1;
+        const int nl = A.kv_len[b] + 1 + n;
+        A.accepted[b] = n;
+        A.bonus[b] = g;
+        A.kv_len[b] = nl;
+        A.kv_len_out[b] = nl;
+        A.pending[b] = g;
+      }
+    }
+  } else if (warp == 0) {
     // draft i is accepted while it equals the target's argmax at row i (i < nr - 1)
     const int l = nr - 1;
     const unsigned long long key = lane < nr ? A.row_key[r0 + lane] : 0ull;
@@ -267,6 +302,7 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
     const int g = __shfl_sync(0xffffffffu, tok, n);
     if (lane == 0) {
       s_n = n;
+      s_node = n;
       if (blockIdx.x == 0) {
         const int nl = A.kv_len[b] + 1 + n;
         A.accepted[b] = n;
@@ -278,7 +314,7 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
     }
   }
   __syncthreads();
-  const int r = r0 + s_n;
+  const int r = r0 + s_node;   // the row that produced the bonus token
   for (int e = tid; e < H * 64; e += blockDim.x) {
     const float v = A.q_anchor[(size_t)r * A.d + e];
     // the tensor-core attention scored bf16(q / 8) against the bf16 keys
@@ -365,6 +401,40 @@ void launch_accept_anchor(const AcceptAnchorArgs& A, cudaStream_t st) {
     dim3 grid((A.t_alloc + C::FB - 1) / C::FB, A.B);
     launch_ex(accept_anchor_kernel<float>, grid, dim3(256), (size_t)A.H * C::FB * C::ROW_BYTES, st, A.pdl, 1, A);
   }
+}
+
+// Tree verify commit: one warp per (utterance, layer, head) moves the accepted
+// path's K and V rows from the nodes' slots kv_len_old + path[j] to the
+// positions kv_len_old + j + 1, in depth order.  Path nodes have increasing
+// slots, path[j] >= j + 1, so a slot is overwritten only after the copy that
+// reads it (each lane moves the same 4 bytes of every row, in program order).
+__global__ void __launch_bounds__(256)
+tree_commit_kernel(const int* __restrict__ path, int k, const int* __restrict__ accepted,
+                   const int* __restrict__ kv_len, int B, int L, int H, int max_pos, int b_max, uint32_t* kself,
+                   uint32_t* vself) {
+  const int w = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+  if (w >= B * L * H) return;
+  const int b = w / (L * H), rem = w - b * L * H, l = rem / H, h = rem - l * H;
+  const int n = accepted[b];
+  if (n <= 0) return;
+  const int P = kv_len[b] - 1 - n;
+  const size_t head = (((size_t)l * b_max + b) * H + h) * (size_t)max_pos;   // row 0 of (layer, b, head)
+  uint32_t* K = kself + head * 32;   // 64 bf16 = 32 words per row
+  uint32_t* V = vself + head * 32;
+  for (int j = 0; j < n; ++j) {
+    const int src = path[(size_t)b * k + j];
+    if (src == j + 1) continue;
+    K[(size_t)(P + j + 1) * 32 + lane] = K[(size_t)(P + src) * 32 + lane];
+    V[(size_t)(P + j + 1) * 32 + lane] = V[(size_t)(P + src) * 32 + lane];
+  }
+}
+
+void launch_tree_commit(const int* path, int k, const int* accepted, const int* kv_len, int B, int L, int H,
+                        int max_pos, int b_max, void* kself, void* vself, int es, cudaStream_t st) {
+  if (es != 2) return;   // tree verify runs on bf16 caches only (the ABI refuses others)
+  const long long threads = 32ll * B * L * H;
+  tree_commit_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, st>>>(
+      path, k, accepted, kv_len, B, L, H, max_pos, b_max, static_cast<uint32_t*>(kself), static_cast<uint32_t*>(vself));
 }
 
 }  // namespace asrspec

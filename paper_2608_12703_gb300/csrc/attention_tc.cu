@@ -75,7 +75,7 @@ struct TcaCfg {
 // keeping a running (max, sum, output) per row (online softmax).  With S > 1
 // the S splits of a (utterance, head) form one cluster and merge their
 // results by pushing them to the CTA that owns each output column (PUSH).
-template <int MT, int TCA_STAGES, bool PUSH>
+template <int MT, int TCA_STAGES, bool PUSH, bool TREE>
 __global__ void __launch_bounds__(TCA_THREADS)
 attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, AttnArgs a,
                int* status) {
@@ -155,13 +155,21 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
     }
   }
   int lim[MT][2];   // visible keys per fragment row (exclusive bound)
+  unsigned tmask[MT][2];   // TREE: the row's ancestors among the slots from kv_len on
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
       const int r = mt * 16 + g + 8 * e;
-      lim[mt][e] = (a.causal && r < nr) ? min(n_keys, a.plan.row_pos[row0 + r] + 1) : n_keys;
+      if constexpr (TREE) {
+        lim[mt][e] = n_keys;
+        tmask[mt][e] = r < nr ? a.plan.row_mask[row0 + r] : 0u;
+      } else {
+        lim[mt][e] = (a.causal && r < nr) ? min(n_keys, a.plan.row_pos[row0 + r] + 1) : n_keys;
+        tmask[mt][e] = 0u;
+      }
     }
+  const int p_committed = TREE ? a.kv_len[b] : 0;   // TREE: slots below are the committed cache
 
   float m_run[MT][2], l_run[MT][2], O[MT][8][4];
 #pragma unroll
@@ -209,7 +217,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
 #pragma unroll
           for (int j = 0; j < 2; ++j) {
             float& s = Sf[mt][nt][2 * e + j];
-            if (kbase + nt * 8 + 2 * t + j >= lim[mt][e]) s = -INFINITY;
+            const int key = kbase + nt * 8 + 2 * t + j;
+            if (key >= lim[mt][e]) s = -INFINITY;
+            if constexpr (TREE)   // a tree slot is visible to the node's descendants only
+              if (key >= p_committed && !((tmask[mt][e] >> (key - p_committed)) & 1u)) s = -INFINITY;
             cm = fmaxf(cm, s);
           }
         cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, 1));
@@ -360,11 +371,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
   tl_mark(a.tl, TL_EXIT);
 }
 
-template <int MT, int ST, bool PUSH>
+template <int MT, int ST, bool PUSH, bool TREE = false>
 static void configure_one() {
-  cudaFuncSetAttribute(attn_tc_kernel<MT, ST, PUSH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaFuncSetAttribute(attn_tc_kernel<MT, ST, PUSH, TREE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        TcaCfg<MT, ST, PUSH>::SMEM);
-  if constexpr (PUSH) cudaFuncSetAttribute(attn_tc_kernel<MT, ST, PUSH>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if constexpr (PUSH)
+    cudaFuncSetAttribute(attn_tc_kernel<MT, ST, PUSH, TREE>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
 
 void configure_attention_tc() {
@@ -376,28 +388,42 @@ void configure_attention_tc() {
     configure_one<2, 2, true>();
     configure_one<1, 3, true>();
     configure_one<2, 3, true>();
+    configure_one<1, 2, false, true>();
+    configure_one<2, 2, false, true>();
+    configure_one<1, 2, true, true>();
+    configure_one<2, 2, true, true>();
   });
 }
 
-template <int MT, int ST, bool PUSH>
+template <int MT, int ST, bool PUSH, bool TREE = false>
 static void launch_one(const AttnArgs& a, int splits, int* status, cudaStream_t st) {
-  launch_ex(attn_tc_kernel<MT, ST, PUSH>, dim3(splits, a.H, a.B), dim3(TCA_THREADS), TcaCfg<MT, ST, PUSH>::SMEM, st,
-            a.pdl, splits, *a.kmap, *a.vmap, a, status);
+  launch_ex(attn_tc_kernel<MT, ST, PUSH, TREE>, dim3(splits, a.H, a.B), dim3(TCA_THREADS), TcaCfg<MT, ST, PUSH>::SMEM,
+            st, a.pdl, splits, *a.kmap, *a.vmap, a, status);
 }
 
 // a.splits CTAs (1, 2, 4 or 8; one cluster) per (utterance, head);
 // rows_max > 16 takes two m-tiles.
 void launch_attention_tc(const AttnArgs& a, int* status, cudaStream_t st) {
   configure_attention_tc();
+  if (a.tree) {   // self-attention of a tree verify (at most 32 nodes per utterance)
+    if (a.splits == 1) {
+      if (a.rows_max > 16) launch_one<2, 2, false, true>(a, a.splits, status, st);
+      else launch_one<1, 2, false, true>(a, a.splits, status, st);
+    } else {
+      if (a.rows_max > 16) launch_one<2, 2, true, true>(a, a.splits, status, st);
+      else launch_one<1, 2, true, true>(a, a.splits, status, st);
+    }
+    return;
+  }
   if (a.splits == 1) {   // one CTA per (utterance, head): 2-deep ring, three CTAs per SM (54 vs 56 us at batch 64)
-    if (a.rows_max > 16) launch_one<2, 2, false>(a, a.splits, status, st);
-    else launch_one<1, 2, false>(a, a.splits, status, st);
+    if (a.rows_max > 16) launch_one<2, 2, false, false>(a, a.splits, status, st);
+    else launch_one<1, 2, false, false>(a, a.splits, status, st);
   } else if (a.causal) {   // self-attention keys split over a cluster (at most max_pos keys)
-    if (a.rows_max > 16) launch_one<2, 2, true>(a, a.splits, status, st);
-    else launch_one<1, 2, true>(a, a.splits, status, st);
+    if (a.rows_max > 16) launch_one<2, 2, true, false>(a, a.splits, status, st);
+    else launch_one<1, 2, true, false>(a, a.splits, status, st);
   } else {                 // encoder keys split over a cluster: deeper ring per CTA
-    if (a.rows_max > 16) launch_one<2, 3, true>(a, a.splits, status, st);
-    else launch_one<1, 3, true>(a, a.splits, status, st);
+    if (a.rows_max > 16) launch_one<2, 3, true, false>(a, a.splits, status, st);
+    else launch_one<1, 3, true, false>(a, a.splits, status, st);
   }
 }
 

@@ -24,6 +24,7 @@ enum StatusBits : int {
   ST_CAPACITY = 1 << 2,      // kv_len + lens + 1 > max_pos
   ST_WAIT_TIMEOUT = 1 << 3,  // a bounded wait gave up (mbarrier / pipeline)
   ST_NOT_READY = 1 << 4,     // verify on an utterance without encoder cache
+  ST_BAD_TREE = 1 << 5,      // tree verify: a parent outside [0, node)
 };
 
 __device__ __forceinline__ void set_status(int* status, int bits) { atomicOr(status, bits); }

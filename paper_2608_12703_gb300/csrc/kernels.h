@@ -42,7 +42,9 @@ void launch_gemm_simt(const void* A, int a_bf16, const void* B, int b_bf16, int 
 struct RowPlan {
   int* row_b;       // [R_max]
   int* row_i;       // [R_max]
-  int* row_pos;     // [R_max]
+  int* row_pos;     // [R_max] cache slot of the row's K/V (its position, but for tree nodes)
+  int* row_epos;    // [R_max] position of the row's token (positional embedding)
+  unsigned* row_mask;   // [R_max] tree verify: the row's ancestors (bit j = node j of its utterance)
   int* row_tok;     // [R_max]
   int* row_start;   // [B_max + 1]
   int* n_rows;      // [1] rows of this step (0 when the step is refused)
@@ -59,9 +61,13 @@ struct TrafficArgs {
 };
 
 // Validate the step's inputs, lay out the rows and reset the argmax keys.
+// parent (tree verify, else null): [B][k], the parent node of node i + 1 in
+// [0, i] (node 0 is the pending token); node i goes to cache slot kv_len + i
+// at position kv_len + depth(i).
 void launch_plan_verify(const int* draft, const int* lens, int k, int B, int vocab, int max_pos, const int* kv_len,
                         const int* pending, const int* ready, RowPlan plan, unsigned long long* row_key,
-                        int* status, const TrafficArgs& tr, cudaStream_t st, unsigned long long* tl = nullptr);
+                        int* status, const TrafficArgs& tr, cudaStream_t st, unsigned long long* tl = nullptr,
+                        const int* parent = nullptr);
 void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,
                                RowPlan plan, int* status, cudaStream_t st);
 // xg / gain / st_part: the folded first LayerNorm's operand bf16(gain * x) [R][d]
@@ -104,6 +110,7 @@ struct AttnArgs {
   int rows_max = 0;        // most rows of one utterance in this call
   int splits = 1;          // CTAs (one cluster) per (utterance, head)
   bool pdl = false;        // programmatic dependent launch
+  bool tree = false;       // self-attention of a tree verify: slots past kv_len visible by plan.row_mask
   unsigned long long* tl = nullptr;   // launch timeline slot (tl_mark), or null
 };
 void launch_attention(const AttnArgs& a, cudaStream_t st);
@@ -127,10 +134,17 @@ struct AcceptAnchorArgs {
   unsigned long long* frame_key;    // [B_max], zero between calls
   int* tickets;                     // [B_max], zero between calls
   int* status;                      // wait time-outs (ST_WAIT_TIMEOUT)
+  const int* parent = nullptr;      // tree verify: [B][k] parents (as the plan), else null
+  int* path = nullptr;              // tree verify: [B][k] accepted nodes by depth (-1 past the path)
   bool pdl;
   unsigned long long* tl = nullptr;   // launch timeline slot (tl_mark), or null
 };
 void launch_accept_anchor(const AcceptAnchorArgs& a, cudaStream_t st);
+// Tree verify commit: the accepted path's self K/V (every layer and head) from
+// the nodes' slots kv_len_old + path[j] to the positions kv_len_old + j + 1.
+// Reads the new kv_len and the accepted count (kv_len_old = kv_len - 1 - n).
+void launch_tree_commit(const int* path, int k, const int* accepted, const int* kv_len, int B, int L, int H,
+                        int max_pos, int b_max, void* kself, void* vself, int es, cudaStream_t st);
 
 // ---- Fused verify for few rows ----------------------------------------------------
 // One persistent cooperative kernel (one CTA per SM) runs the decoder layers and

@@ -35,13 +35,16 @@ __device__ int block_excl_scan(int v, int* total) {
 }
 
 // Verify rows: utterance b contributes lens[b] + 1 rows (pending, then drafts),
-// at positions kv_len[b] + i.  Any invalid input refuses the whole step
-// (n_rows = 0, nothing is written) and sets the status word.
+// at positions kv_len[b] + i.  A tree verify (parent set) lays out the nodes
+// the same way, node i in cache slot kv_len[b] + i, with its position
+// kv_len[b] + depth(i) and its ancestors (itself included) as a bit mask.  Any
+// invalid input refuses the whole step (n_rows = 0, nothing is written) and
+// sets the status word.
 __global__ void __launch_bounds__(PLAN_THREADS)
 plan_verify_kernel(const int* __restrict__ draft, const int* __restrict__ lens, int k, int B, int vocab, int max_pos,
                    const int* __restrict__ kv_len, const int* __restrict__ pending, const int* __restrict__ ready,
                    RowPlan plan, unsigned long long* row_key, int* status, TrafficArgs tr,
-                   unsigned long long* tl) {
+                   unsigned long long* tl, const int* __restrict__ parent) {
   __shared__ int s_err;
   __shared__ unsigned long long s_cnt[4];
   tl_mark(tl, TL_ENTRY);
@@ -60,6 +63,10 @@ plan_verify_kernel(const int* __restrict__ draft, const int* __restrict__ lens, 
       for (int i = 0; i < l; ++i) {
         const int t = draft[(size_t)b * k + i];
         if (t < 0 || t >= vocab) err |= ST_BAD_TOKEN;
+        if (parent != nullptr) {
+          const int p = parent[(size_t)b * k + i];
+          if (p < 0 || p > i) err |= ST_BAD_TREE;
+        }
       }
       n_b = l + 1;
     }
@@ -75,12 +82,23 @@ plan_verify_kernel(const int* __restrict__ draft, const int* __restrict__ lens, 
   if (b < B) {
     plan.row_start[b] = start;
     plan.n_utt_rows[b] = n_b;
+    int depth[32];
+    unsigned anc[32];
     for (int i = 0; i < n_b; ++i) {
       const int r = start + i;
       plan.row_b[r] = b;
       plan.row_i[r] = i;
       plan.row_pos[r] = kv_len[b] + i;
       plan.row_tok[r] = i == 0 ? pending[b] : draft[(size_t)b * k + i - 1];
+      if (parent != nullptr) {   // n_b <= 32 (k <= 31)
+        const int p = i == 0 ? 0 : parent[(size_t)b * k + i - 1];
+        depth[i] = i == 0 ? 0 : depth[p] + 1;
+        anc[i] = (i == 0 ? 0u : anc[p]) | (1u << i);
+        plan.row_epos[r] = kv_len[b] + depth[i];
+        plan.row_mask[r] = anc[i];
+      } else {
+        plan.row_epos[r] = kv_len[b] + i;
+      }
       row_key[r] = 0ull;
     }
     if (n_b > 0 && tr.counters) {
@@ -137,6 +155,7 @@ plan_prefill_kernel(const int* __restrict__ prompt, int P0, int p0, int c, int B
       plan.row_b[r] = b;
       plan.row_i[r] = i;
       plan.row_pos[r] = p0 + i;
+      plan.row_epos[r] = p0 + i;
       plan.row_tok[r] = prompt[(size_t)b * P0 + p0 + i];
     }
   }
@@ -148,9 +167,10 @@ plan_prefill_kernel(const int* __restrict__ prompt, int P0, int p0, int c, int B
 
 void launch_plan_verify(const int* draft, const int* lens, int k, int B, int vocab, int max_pos, const int* kv_len,
                         const int* pending, const int* ready, RowPlan plan, unsigned long long* row_key,
-                        int* status, const TrafficArgs& tr, cudaStream_t st, unsigned long long* tl) {
+                        int* status, const TrafficArgs& tr, cudaStream_t st, unsigned long long* tl,
+                        const int* parent) {
   plan_verify_kernel<<<1, PLAN_THREADS, 0, st>>>(draft, lens, k, B, vocab, max_pos, kv_len, pending, ready, plan,
-                                                 row_key, status, tr, tl);
+                                                 row_key, status, tr, tl, parent);
 }
 
 void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, int vocab, const int* ready,
@@ -174,7 +194,7 @@ embed_kernel(const T* __restrict__ tok_emb, const T* __restrict__ pos_emb, RowPl
   pdl_launch();
   const int r = blockIdx.x;
   if (r >= *plan.n_rows) return;   // uniform over the CTA
-  const int t = plan.row_tok[r], p = plan.row_pos[r];
+  const int t = plan.row_tok[r], p = plan.row_epos[r];
   float v[16];
   float s = 0.f;
 #pragma unroll

@@ -156,6 +156,9 @@ def main():
                     help="comma-separated batch sizes: verification cost and anchor-readout share of the large "
                          "decoder at each (replaces the single-workload run)")
     ap.add_argument("--k", type=int, default=6, help="drafts per utterance of --batch-sweep")
+    ap.add_argument("--tree-nodes", type=int, default=0,
+                    help="also time tree verifies of this many nodes per utterance (random trees whose first k "
+                         "nodes form one branch) beside the linear verify")
     args = ap.parse_args()
     if args.batch_sweep:
         from paper_2608_12703_gb300 import build as B
@@ -213,6 +216,35 @@ def main():
         ns, kinds = A.asr_spec_timeline_read(sess.h)
         A.asr_spec_timeline(sess.h, False)
         print(timeline_summary(ns, kinds, args.rounds))
+    if args.tree_nodes:
+        n = args.tree_nodes
+        trng = np.random.default_rng(9)
+        tsess = Session(dims, W.make_weights(dims), max_batch=wl.batch, max_draft=max(n, wl.k))
+        tsess.encode_cache(W.make_encoder_states(dims, wl.enc_lens, wl.t_max), list(wl.enc_lens))
+        tsess.prefill(W.make_prompt(dims, wl.batch))
+        parent = np.array([[trng.integers(0, i + 1) if i >= wl.k else i for i in range(n)]
+                           for _ in range(wl.batch)], dtype=np.int32)
+        with torch.cuda.stream(tsess.stream):
+            tok_d = [torch.from_numpy(trng.integers(0, dims.vocab, size=(wl.batch, n)).astype(np.int32)).cuda()
+                     for _ in range(args.warmup + args.rounds)]
+            par_d = torch.from_numpy(parent).cuda()
+            lens_t = torch.full((wl.batch,), n, dtype=torch.int32, device="cuda")
+            path_d = torch.zeros((wl.batch, n), dtype=torch.int32, device="cuda")
+        tsess.stream.synchronize()
+        o = tsess.out[:, :wl.batch]
+        tt = []
+        for i in range(args.warmup + args.rounds):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(tsess.stream)
+            A.asr_spec_verify_tree(tsess.h, tok_d[i], par_d, lens_t, n, o[0], o[1], o[2], o[3], path_d)
+            e1.record(tsess.stream)
+            if i >= args.warmup:
+                tt.append((e0, e1))
+        torch.cuda.synchronize()
+        tus = [a.elapsed_time(b) * 1e3 for a, b in tt]
+        print(f"  tree verify, {n} nodes per utterance: us per round " + " ".join(f"{u:.1f}" for u in tus)
+              + f"; status {tsess.status()}")
+        tsess.close()
     if args.fused_trace:
         A.asr_spec_fused_trace(sess.h, True)
         sess.verify_device(drafts[0], lens, wl.k)

@@ -106,6 +106,24 @@ class Session:
             oh = o.cpu().numpy()
         return StepOut(oh[0].copy(), oh[1].copy(), oh[2].copy(), oh[3].copy())
 
+    def verify_tree(self, tokens, parent, lens):
+        """Tree verify: tokens / parent [B][n] (node i + 1's token and parent),
+        lens [B] nodes used or -1.  Returns the step outputs and path [B][n]."""
+        tokens = np.ascontiguousarray(np.asarray(tokens, dtype=np.int32).reshape(self.B, -1))
+        parent = np.ascontiguousarray(np.asarray(parent, dtype=np.int32).reshape(self.B, -1))
+        n = tokens.shape[1]
+        lens = np.asarray(lens, dtype=np.int32)
+        with torch.cuda.stream(self.stream):
+            t = torch.from_numpy(tokens).to(self.dev)
+            p = torch.from_numpy(parent).to(self.dev)
+            l = torch.from_numpy(lens).to(self.dev)
+            path = torch.full((self.B, max(n, 1)), -1, dtype=torch.int32, device=self.dev)
+            o = self.out[:, :self.B]
+            A.asr_spec_verify_tree(self.h, t, p, l, n, o[0], o[1], o[2], o[3], path)
+            oh = o.cpu().numpy()
+            ph = path.cpu().numpy()[:, :n]
+        return StepOut(oh[0].copy(), oh[1].copy(), oh[2].copy(), oh[3].copy()), ph
+
     def host(self, t) -> np.ndarray:
         """Copy a device tensor written on this session's stream to the host."""
         self.stream.synchronize()
