@@ -156,6 +156,8 @@ def main():
                     help="comma-separated batch sizes: verification cost and anchor-readout share of the large "
                          "decoder at each (replaces the single-workload run)")
     ap.add_argument("--k", type=int, default=6, help="drafts per utterance of --batch-sweep")
+    ap.add_argument("--enc-len", type=int, default=0,
+                    help="encoder frames of every utterance instead of the workload's (long-form audio: > 1500)")
     ap.add_argument("--tree-nodes", type=int, default=0,
                     help="also time tree verifies of this many nodes per utterance (random trees whose first k "
                          "nodes form one branch) beside the linear verify")
@@ -175,6 +177,10 @@ def main():
 
     B.build()
     wl = W.CONFIGS[args.config]
+    if args.enc_len:
+        import dataclasses
+        dims = dataclasses.replace(wl.dims, max_enc=max(wl.dims.max_enc, args.enc_len))
+        wl = dataclasses.replace(wl, dims=dims, enc_lens=(args.enc_len,) * wl.batch, t_max=args.enc_len)
     dims = wl.dims
     sess = Session(dims, W.make_weights(dims), max_batch=wl.batch, max_draft=wl.k)
     if args.no_graphs:

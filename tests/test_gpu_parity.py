@@ -155,3 +155,21 @@ def test_large_bf16_batch64_sampled_utterances(built_lib, cuda):
     _report(wl.name, st)
     assert sess.status() == 0
     sess.close()
+
+
+def test_long_form_encoder_memory(built_lib, cuda):
+    """Encoder memories past Whisper's 30 s window (the paper's long-audio
+    setting, up to about 104 s of concatenated audio = 5200 frames at 20 ms):
+    the small bf16 decoder, two utterances of 5200 and 2100 frames, k = 8."""
+    import dataclasses
+    dims = dataclasses.replace(W.SMALL, max_enc=5200)
+    blob = _blob(W.SMALL)   # the same weights (max_enc sizes only the cache)
+    enc_lens = [5200, 2100]
+    enc = W.make_encoder_states(dims, enc_lens, 5200)
+    prompt = W.make_prompt(dims, 2)
+    total = [W.PROMPT_LEN + 18, W.PROMPT_LEN + 11]
+    wl = W.Workload("long", dims, 2, 8, (18, 11), tuple(enc_lens), (0.2, 0.4), "half", t_max=5200)
+    st, _ = run_decode(dims, blob, enc, enc_lens, prompt, total, 8, W.make_corruption(wl),
+                       _session(dims, blob, 2, 8), max_rounds=6)
+    _report("long-form 5200 + 2100 frames", st)
+    assert st.rows > 20
