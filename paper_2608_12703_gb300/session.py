@@ -113,6 +113,11 @@ class Session:
         parent = np.ascontiguousarray(np.asarray(parent, dtype=np.int32).reshape(self.B, -1))
         n = tokens.shape[1]
         lens = np.asarray(lens, dtype=np.int32)
+        if self.host_io:
+            acc, bon, kvl, anc = (np.zeros(self.B, np.int32) for _ in range(4))
+            path = np.full((self.B, max(n, 1)), -1, dtype=np.int32)
+            A.asr_spec_verify_tree(self.h, tokens, parent, lens, n, acc, bon, kvl, anc, path)
+            return StepOut(acc, bon, kvl, anc), path[:, :n]
         with torch.cuda.stream(self.stream):
             t = torch.from_numpy(tokens).to(self.dev)
             p = torch.from_numpy(parent).to(self.dev)

@@ -163,3 +163,26 @@ def test_tree_bad_parent_refuses_the_step(built_lib, cuda):
     out, path = s.verify_tree(np.ones((2, 3)), np.array([[0, 0, 1], [0, 1, 1]]), np.array([3, 3]))
     assert s.status() == 0 and np.all(out.kv_len > kv0)
     s.close()
+
+
+def test_tree_host_io_matches_device_io(built_lib, cuda):
+    from paper_2608_12703_gb300.session import Session
+    dims = W.ModelDims(n_layers=2, d_model=128, n_heads=2, d_ffn=256, vocab=500, dtype="bf16",
+                       max_pos=32, max_enc=64, anchor_layer=1)
+    blob = W.make_weights(dims, std=0.1)
+    rng = np.random.default_rng(8)
+    trees = [(rng.integers(0, 500, size=(2, 5)), np.array([[0, 0, 1, 2, 2], [0, 1, 1, 0, 4]])) for _ in range(3)]
+    outs = []
+    for host in (False, True):
+        s = Session(dims, blob, max_batch=2, max_draft=5)
+        s.set_host_io(host)
+        s.encode_cache(W.make_encoder_states(dims, [64, 20], 64), [64, 20])
+        s.prefill(W.make_prompt(dims, 2))
+        res = []
+        for tok, par in trees:
+            o, path = s.verify_tree(tok, par, np.array([5, 3]))
+            res.append((list(o.accepted), list(o.bonus), list(o.kv_len), list(o.anchor), path.tolist()))
+        assert s.status() == 0
+        s.close()
+        outs.append(res)
+    assert outs[0] == outs[1]
