@@ -418,3 +418,41 @@ def test_tree_errors():
     o, *_ = _setup()
     with pytest.raises(OracleError):
         o.verify_tree(np.zeros((3, 2), dtype=int), np.array([[0, 2], [0, 0], [0, 0]]), np.array([2, 2, 2]))
+
+
+def test_mean_accepted_length_matches_the_closed_form():
+    """Sec. 3 "Speculative Loop": the mean accepted draft length is
+    L = sum_{k=1..K} s_k with s_k the probability that the first k proposals
+    are accepted.  Drafts that are the target's own greedy continuation with
+    every token replaced independently with probability p by a uniform id
+    (R12; the replacement equals the true token with probability 1/V) are kept
+    up to the first mismatch, so s_k = q^k with q = 1 - p + p/V.  The oracle's
+    accepted lengths over full-width rounds must match that law."""
+    dims = W.ModelDims(n_layers=2, d_model=64, n_heads=2, d_ffn=128, vocab=1000, dtype="fp32",
+                       max_pos=448, max_enc=20, anchor_layer=1)
+    K, p = 4, 0.3
+    B = 3
+    total = [400] * B
+    o, *_ = _setup(dims, enc_lens=[20, 13, 7], std=0.3)
+    snap = o.snapshot()
+    prompt = W.make_prompt(dims, B)
+    truth = greedy_transcript(o, prompt, total)
+    o.restore(snap)
+    wl = W.Workload("acc", dims, B, K, tuple(t - W.PROMPT_LEN for t in total), (20, 13, 7), (p,) * B, "none",
+                    t_max=20)
+    corr = W.make_corruption(wl)
+    ns = []
+    while True:
+        draft, lens = W.make_drafts(truth, total, o.kv_len, K, corr)
+        if np.all(lens < 0):
+            break
+        res = o.verify(draft, lens)
+        ns += [int(res.accepted[b]) for b in range(B) if lens[b] == K]
+    q = 1 - p + p / dims.vocab
+    pmf = np.array([q ** j * (1 - q) for j in range(K)] + [q ** K])
+    mean = float(np.dot(np.arange(K + 1), pmf))
+    var = float(np.dot((np.arange(K + 1) - mean) ** 2, pmf))
+    assert mean == pytest.approx(sum(q ** k for k in range(1, K + 1)))
+    got = float(np.mean(ns))
+    assert len(ns) > 250
+    assert abs(got - mean) < 4 * np.sqrt(var / len(ns)), (got, mean, len(ns))
