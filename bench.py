@@ -133,7 +133,7 @@ def weights(dims):
     return _WEIGHTS[dims]
 
 
-class GpuRun:
+class DecodeRun:
     """One workload resident on one GPU, plus the reference transcript that
     drives the synthetic draft source."""
 
@@ -623,7 +623,7 @@ def main():
     B.build()
     pk = peaks()
     wl = W.CONFIGS[args.config]
-    run = GpuRun(wl)
+    run = DecodeRun(wl)
     res = run.timed(args.steps, args.warmup, dist, gpu_index=local)
     ms = max_over_ranks(dist, res["ms"])
     value = whole_job_rate(world, args.steps, run.tokens_per_decode, ms / 1e3)
@@ -661,7 +661,7 @@ def main():
             del run
             torch.cuda.empty_cache()
             wl1 = W.CONFIGS[args.batch1_config]
-            r1 = GpuRun(wl1)
+            r1 = DecodeRun(wl1)
             b1 = r1.timed(args.steps, args.warmup, None, gpu_index=local)
             pm, pl, pt = r1.profile()
             tl1 = r1.launch_timeline()
