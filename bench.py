@@ -487,9 +487,9 @@ def step_bytes(dims, traffic, calls_override=None):
 # ----------------------------------------------------------------------------
 # CPU oracle arm
 # ----------------------------------------------------------------------------
-def oracle_sample(wl: W.Workload, truth, budget_s: float, utt: int = 0, rounds_cap=None):
+def oracle_sample(wl: W.Workload, truth, seconds: float, utt: int = 0, rounds_cap=None):
     """The oracle on utterance `utt` of the workload: encoder cache, prefill,
-    then verify rounds with the workload's drafts until the budget is spent.
+    then verify rounds with the workload's drafts until that many seconds are spent.
     Returns (tokens emitted, seconds, rounds, description)."""
     from oracle import Oracle
     dims = wl.dims
@@ -505,7 +505,7 @@ def oracle_sample(wl: W.Workload, truth, budget_s: float, utt: int = 0, rounds_c
     sub = W.Corruption(corr.repl[utt:utt + 1], corr.shift[utt:utt + 1])
     total = [wl.total_lens[utt]]
     tokens = rounds = 0
-    while time.perf_counter() - t0 < budget_s and (rounds_cap is None or rounds < rounds_cap):
+    while time.perf_counter() - t0 < seconds and (rounds_cap is None or rounds < rounds_cap):
         draft, lens = W.make_drafts(truth[utt:utt + 1], total, orc.kv_len, wl.k, sub)
         if lens[0] < 0:
             break
@@ -598,7 +598,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-batch1", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--cpu-budget", type=float, default=20.0)
+    ap.add_argument("--cpu-seconds", type=float, default=20.0)
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -654,7 +654,7 @@ def main():
         line["e2e"] = e2e
     if rank == 0:
         # CPU oracle on a bounded sample of the same workload
-        tokens, dt, rounds, desc = oracle_sample(wl, run.truth, args.cpu_budget)
+        tokens, dt, rounds, desc = oracle_sample(wl, run.truth, args.cpu_seconds)
         line["cpu_baseline"] = {"value": tokens / dt, "unit": "tokens/s", "cores": cpu_threads(),
                                 "kind": "oracle", "sample": desc}
         if not args.no_batch1 and args.batch1_config != args.config:
