@@ -45,7 +45,7 @@ from typing import Dict, List, Optional
 import numpy as np
 from scipy.special import erf
 
-from workload import ModelDims, weight_layout
+from workload import ModelDims, draft_taps, weight_layout
 
 LN_EPS = 1e-5
 
@@ -145,6 +145,7 @@ class VerifyResult:
     top2_gap: np.ndarray      # [R] top-1 minus top-2 logit
     anchor_profile: Dict[int, np.ndarray]  # b -> head-mean attention over frames
     path: Optional[np.ndarray] = None       # tree verify: [B][n] accepted nodes by depth (-1 past the path)
+    feats: Optional[np.ndarray] = None      # [R, 4, d] the target's outputs at the draft's tap layers
 
 
 class Oracle:
@@ -192,6 +193,7 @@ class Oracle:
         self.B = B
         self.enc_len = enc_lens.copy()
         E = enc_states.astype(np.float64)
+        self.enc = [E[b, :enc_lens[b]].copy() for b in range(B)]   # the draft reads the encoder states too
         self.Kx, self.Vx = [], []
         for l in range(d.n_layers):
             self.Kx.append([E[b, :enc_lens[b]] @ self.W(f"L{l}.wck").T for b in range(B)])
@@ -214,8 +216,10 @@ class Oracle:
             raise OracleError("bad prompt shape")
         self._check_tokens(prompt)
         rows = [(b, int(prompt[b, i]), i) for b in range(B) for i in range(P0 - 1)]
+        self.prefill_feats = np.zeros((B, max(P0 - 1, 0), 4, self.dims.d_model))
         if rows:
             self._forward(rows)
+            self.prefill_feats[:] = self.last_feats.reshape(B, P0 - 1, 4, self.dims.d_model)
         self.kv_len = np.full(B, P0 - 1, dtype=np.int64)
         self.pending = prompt[:, P0 - 1].copy()
 
@@ -246,6 +250,8 @@ class Oracle:
         bidx = [r[0] for r in rows]
         x = self.W("tok_emb")[tok] + self.W("pos_emb")[pos]
         q_anchor = None
+        taps = draft_taps(d)
+        feats = np.zeros((len(rows), 4, d.d_model))
         for l in range(d.n_layers):
             p = f"L{l}."
             # self-attention block
@@ -279,6 +285,10 @@ class Oracle:
             h = layer_norm(x, self.W(p + "ln3_g"), self.W(p + "ln3_b"))
             f = gelu(h @ self.W(p + "w1").T + self.W(p + "b1"))
             x = x + f @ self.W(p + "w2").T + self.W(p + "b2")
+            for i, t in enumerate(taps):
+                if t == l:
+                    feats[:, i] = x
+        self.last_feats = feats   # the draft's inputs (layer outputs at its tap layers), row order
         logits = None
         if want_logits:
             xf = layer_norm(x, self.W("lnf_g"), self.W("lnf_b"))
@@ -344,8 +354,10 @@ class Oracle:
             self.kv_len[b] = self.kv_len[b] + 1 + n
             self.pending[b] = bonus[b]
             r0 += int(lens[b]) + 1
-        return VerifyResult(acc, bonus, self.kv_len.copy(), anchor, restart, row_ids,
-                            logits, g, gap, prof)
+        res = VerifyResult(acc, bonus, self.kv_len.copy(), anchor, restart, row_ids,
+                           logits, g, gap, prof)
+        res.feats = self.last_feats if rows else np.zeros((0, 4, d.d_model))
+        return res
 
     def verify_tree(self, tokens, parent, lens) -> VerifyResult:
         """Score a candidate tree per utterance in one pass under a tree mask
@@ -432,6 +444,7 @@ class Oracle:
             r0 += int(lens[b]) + 1
         res = VerifyResult(acc, bonus, self.kv_len.copy(), anchor, restart, row_ids, logits, g, gap, prof)
         res.path = path
+        res.feats = self.last_feats if rows else np.zeros((0, 4, d.d_model))
         return res
 
     def rollback(self, new_len, new_pending) -> None:

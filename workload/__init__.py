@@ -17,7 +17,8 @@ available; the shapes below follow its workloads instead:
 * draft blocks of up to K tokens (Sec. 3 "Speculative Loop").
 
 Random streams (numpy PCG64 through ``default_rng``):
-  seed 0 weights, 1 encoder states, 2 draft corruption, 3 prompt, 4 lengths.
+  seed 0 weights, 1 encoder states, 2 draft corruption, 3 prompt, 4 lengths,
+  5 draft-model weights.
 """
 from __future__ import annotations
 
@@ -36,6 +37,7 @@ SEED_ENCODER = 1
 SEED_CORRUPT = 2
 SEED_PROMPT = 3
 SEED_LENGTHS = 4
+SEED_DRAFT = 5
 
 
 @dataclasses.dataclass(frozen=True)
@@ -192,6 +194,64 @@ def make_weights(dims: ModelDims, seed: int = SEED_WEIGHTS, std: float = 0.02) -
         chunk = 1 << 26
         for s in range(0, n, chunk):
             blob[s:s + chunk] = bf16_round(blob[s:s + chunk])
+    return blob
+
+
+# ----------------------------------------------------------------------------
+# The one-block draft (random init): layout and the target layers it reads
+# ----------------------------------------------------------------------------
+
+def draft_taps(dims: ModelDims) -> List[int]:
+    """The four target layers whose outputs (the residual stream after the
+    layer) the draft combines (App. "Draft architecture": four frozen target
+    representations): evenly spaced, the last one the final layer."""
+    L = dims.n_layers
+    return [max(0, (i + 1) * L // 4 - 1) for i in range(4)]
+
+
+def draft_ffn(dims: ModelDims) -> int:
+    """The draft's feed-forward width: twice its hidden width, as both of the
+    paper's draft configurations (1024 / 2048 and 2048 / 4096)."""
+    return 2 * dims.d_model
+
+
+def draft_weight_layout(dims: ModelDims) -> Dict[str, Tuple[int, Tuple[int, ...]]]:
+    """Name -> (offset, shape) of the draft's fp32 blob: the input combination
+    w_in [d, 4d], b_in, one pre-LN decoder block (the target block's tensors,
+    feed-forward width draft_ffn), and its final LayerNorm.  Token and position
+    embeddings and the LM head are the target's (frozen)."""
+    d = dims.d_model
+    ddims = dataclasses.replace(dims, d_ffn=draft_ffn(dims))
+    out: Dict[str, Tuple[int, Tuple[int, ...]]] = {}
+    off = 0
+
+    def put(name, shape):
+        nonlocal off
+        out[name] = (off, shape)
+        off += int(np.prod(shape))
+
+    put("w_in", (d, 4 * d))
+    put("b_in", (d,))
+    for name, shape in layer_tensors(ddims):
+        put(name, shape)
+    put("lnf_g", (d,))
+    put("lnf_b", (d,))
+    out["__total__"] = (off, ())
+    return out
+
+
+def make_draft_weights(dims: ModelDims, seed: int = SEED_DRAFT, std: float = 0.02) -> np.ndarray:
+    """Random-init draft blob, drawn like the target's (std * N(0,1),
+    LayerNorm gains 1 + that, bf16-rounded once for bf16 models)."""
+    lay = draft_weight_layout(dims)
+    n = lay["__total__"][0]
+    rng = np.random.default_rng(seed)
+    blob = rng.standard_normal(n, dtype=np.float32) * np.float32(std)
+    for name, (off, shape) in lay.items():
+        if name.endswith("_g"):
+            blob[off:off + shape[0]] += np.float32(1.0)
+    if dims.dtype == "bf16":
+        blob = bf16_round(blob)
     return blob
 
 
