@@ -115,26 +115,35 @@ class Draft:
         for j in range(1, n + 1):
             self.step(b, int(drafts_b[j - 1]), P_old + j, feats_b[j - 1])
 
-    def propose(self, b: int, pending: int, P: int, feat: np.ndarray, k: int, win=None) -> List[int]:
-        """k proposals from the verified state: the restart at position P (the
-        pending token with the target's representations of the row that scored
-        it), then continuation proposals fed by the draft's own output."""
+    def propose(self, b: int, pending: int, P: int, feat: np.ndarray, k: int, win=None,
+                threshold: float = 0.0) -> List[int]:
+        """Up to k proposals from the verified state: the restart at position P
+        (the pending token with the target's representations of the row that
+        scored it), then continuation proposals fed by the draft's own output.
+        A proposal whose draft probability (softmax of its logits) is below
+        `threshold` ends the block unproposed (App. "Draft length and
+        confidence threshold": the block length varies per utterance)."""
         out, tok, f = [], int(pending), feat
         for i in range(k):
             logits, x = self.step(b, tok, P + i, f, win)
             tok = int(np.argmax(logits))
+            if threshold > 0.0:
+                e = np.exp(logits - logits.max())
+                if 1.0 / e.sum() < threshold:   # the top token's probability
+                    break
             out.append(tok)
             f = np.tile(x, (4, 1))
         return out
 
 
 def speculative_decode(target: Oracle, draft: Draft, prompt, total_lens, k: int, kind: Optional[str] = "anchor",
-                       rng: Optional[np.random.Generator] = None):
+                       rng: Optional[np.random.Generator] = None, threshold: float = 0.0):
     """The real cached loop until every utterance holds total_lens[b] tokens
     (prompt included).  kind: "anchor" (deployed correction), "shifted",
-    "random" (controls) or None (unrestricted audio attention).  Returns the
-    token sequences and, per round, (lens, accepted) of the utterances that
-    took part."""
+    "random" (controls) or None (unrestricted audio attention); threshold: the
+    draft's confidence threshold (0 = always k proposals).  Returns the token
+    sequences and, per round, (lens, accepted) of the utterances (lens -1 for
+    those that sat out)."""
     prompt = np.asarray(prompt, dtype=np.int64)
     B = prompt.shape[0]
     target.prefill(prompt)
@@ -157,8 +166,10 @@ def speculative_decode(target: Oracle, draft: Draft, prompt, total_lens, k: int,
             T = len(target.enc[b])
             win = None if kind is None else window(window_center(kind, anchor[b], T, rng), T)
             if lens[b] > 0:
-                drafts[b, :lens[b]] = draft.propose(b, int(target.pending[b]), int(target.kv_len[b]), feat[b],
-                                                    int(lens[b]), win)
+                props = draft.propose(b, int(target.pending[b]), int(target.kv_len[b]), feat[b], int(lens[b]), win,
+                                      threshold)
+                drafts[b, :len(props)] = props
+                lens[b] = len(props)
             else:   # no proposals: the pending position's entry all the same
                 draft.step(b, int(target.pending[b]), int(target.kv_len[b]), feat[b], win)
         P_old = target.kv_len.copy()
@@ -176,3 +187,25 @@ def speculative_decode(target: Oracle, draft: Draft, prompt, total_lens, k: int,
             r0 += int(lens[b]) + 1
         rounds.append((lens.copy(), res.accepted.copy()))
     return seqs, rounds
+
+
+def acceptance_stats(rounds, k: int) -> Dict[str, float]:
+    """The speculative loop's acceptance metrics (Sec. 3 "Speculative Loop"):
+    s_j, the probability that the first j proposals are accepted, over the
+    rounds that offered at least j proposals (s_0 = 1); restart acceptance
+    a_1 = s_1; continuation acceptance a_j^c = s_j / s_{j-1}; L, the mean
+    accepted length per round (sum_j s_j when every round offers k)."""
+    lens = np.concatenate([np.asarray(l) for l, _ in rounds])
+    acc = np.concatenate([np.asarray(a) for _, a in rounds])
+    live = lens >= 0
+    lens, acc = lens[live], acc[live]
+    s = [1.0]
+    for j in range(1, k + 1):
+        offered = lens >= j
+        s.append(float(np.mean(acc[offered] >= j)) if offered.any() else float("nan"))
+    out = {f"s_{j}": s[j] for j in range(1, k + 1)}
+    out["a_1"] = s[1]
+    for j in range(2, k + 1):
+        out[f"a_{j}^c"] = s[j] / s[j - 1] if s[j - 1] > 0 else float("nan")
+    out["L"] = float(np.mean(acc))
+    return out

@@ -189,3 +189,51 @@ def test_pins_catch_planted_draft_mistakes(monkeypatch, mistake):
         monkeypatch.setattr(D.Draft, "step", _step_without_features(D.Draft.step))
         with pytest.raises(AssertionError):
             test_draft_block_matches_torch_decoder_layer()
+
+
+def test_confidence_threshold_varies_the_block_and_stays_lossless():
+    """Threshold 0 proposes k every round; threshold 1 proposes nothing (plain
+    greedy decoding, one token per round); in between the block length varies
+    per utterance and the output is still the target's greedy transcript."""
+    from oracle.draft import acceptance_stats
+    prompt = W.make_prompt(TINY, 3)
+    total = [30, 22, 27]
+    out = {}
+    for thr in (0.0, 0.4, 1.0):
+        o, dr, blob, enc = _setup()
+        seqs, rounds = speculative_decode(o, dr, prompt, total, 4, "anchor", threshold=thr)
+        out[thr] = (seqs, rounds)
+    ref_t = Oracle(TINY, W.make_weights(TINY, std=0.3))
+    ref_t.encode_cache(W.make_encoder_states(TINY, ENC_LENS, max(ENC_LENS)), ENC_LENS)
+    ref_t.prefill(prompt)
+    truth = greedy_transcript(ref_t, prompt, total)
+    for thr, (seqs, rounds) in out.items():
+        assert all(seqs[b] == list(truth[b, :total[b]]) for b in range(3)), thr
+    l0 = np.concatenate([l for l, _ in out[0.0][1]])
+    l1 = np.concatenate([l for l, _ in out[1.0][1]])
+    lm = np.concatenate([l for l, _ in out[0.4][1]])
+    assert np.all(l1[l1 >= 0] == 0)
+    assert len(out[1.0][1]) == max(total) - prompt.shape[1]      # one token per round
+    full = W.round_lens(total, [prompt.shape[1] - 1] * 3, 4)
+    assert np.all(l0[:3] == full)
+    assert 0 < np.sum(lm[lm >= 0]) < np.sum(l0[l0 >= 0])         # some blocks cut short
+    assert acceptance_stats(out[1.0][1], 4)["L"] == 0.0
+
+
+def test_acceptance_stats_follow_the_definitions():
+    """s_j, a_1, a_j^c and L (Sec. 3) on rounds built by hand, and the closed
+    form under independent per-token corruption: s_j = q^j, a_j^c = q."""
+    from oracle.draft import acceptance_stats
+    rounds = [(np.array([3, 3, -1]), np.array([3, 0, 0])), (np.array([3, 1, 2]), np.array([1, 1, 2]))]
+    st = acceptance_stats(rounds, 3)
+    assert st["s_1"] == pytest.approx(4 / 5) and st["s_2"] == pytest.approx(2 / 4) and st["s_3"] == pytest.approx(1 / 3)
+    assert st["a_1"] == st["s_1"] and st["a_2^c"] == pytest.approx((2 / 4) / (4 / 5))
+    assert st["L"] == pytest.approx((3 + 0 + 1 + 1 + 2) / 5)
+    rng = np.random.default_rng(0)
+    q, K, n = 0.7, 4, 20000
+    hits = rng.random((n, K)) < q
+    acc = np.where(hits.all(axis=1), K, np.argmin(hits, axis=1))
+    st = acceptance_stats([(np.full(n, K), acc)], K)
+    for j in range(1, K + 1):
+        assert st[f"s_{j}"] == pytest.approx(q ** j, abs=0.02)
+    assert st["a_2^c"] == pytest.approx(q, abs=0.02) and st["L"] == pytest.approx(sum(q ** j for j in range(1, K + 1)), abs=0.03)
