@@ -7,7 +7,13 @@ CUDA events on the library's stream.
 
   python -m paper_2608_12703_gb300.profile_run --config large-bf16-b1-k8 --warmup 2 --rounds 3
 
-Kernel launches per round (bf16 decoders): 2 + 12 per layer + 4.
+Options: --classes (CUDA-event time per kernel class), --timeline (the launch
+timeline per launch kind), --fused-trace (per-stage stamps of the opt-in fused
+verify), --tree-nodes N (tree verifies beside the linear one), --enc-len T
+(encoder memories of T frames), --batch-sweep 1,4,16,64 (verification cost and
+anchor-readout share against batch size).
+
+Kernel launches per round (bf16 decoders, LayerNorm folded): 2 + 8 per layer + 2.
 """
 from __future__ import annotations
 
