@@ -198,7 +198,11 @@ int attn_chunk_len(int kv_bf16) { return kv_bf16 ? 256 : 128; }
 // "Verification-Attention Correction"), with the (max, sum) the attention pass
 // left: a fixed-order head sum per frame, an order-free atomicMax of packed
 // (value, frame) keys, and the last CTA of the utterance (ticket) writes the
-// peak frame.  Only CTAs that hold frames (and the first) take part.
+// peak frame.  Only CTAs that hold frames (and the first) take part.  A tree
+// verify (A.parent set; App. tree decoder control) replaces the prefix ballot
+// by a walk: from the root, one ballot per step finds the first child whose
+// token is the current node's argmax; the path goes to A.path and the anchor
+// row is the path's last node.
 constexpr int ANCHOR_HMAX = 32;   // heads (d_model <= 2048)
 
 template <typename T>

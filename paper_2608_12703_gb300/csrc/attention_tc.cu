@@ -18,7 +18,11 @@
 //     thread-block cluster: CTA q owns output columns [64q/S, 64(q+1)/S), every
 //     split pushes its (max, sum, partial output) of those columns into q's
 //     shared memory with st.async (bytes counted on q's mbarrier), and q merges
-//     them in split order, so the result does not depend on timing.
+//     them in split order, so the result does not depend on timing;
+//   * the TREE variant (self-attention of a tree verify) makes a cache slot at
+//     or past kv_len visible to a row only if it holds one of the row's
+//     ancestors (plan.row_mask), the tree attention mask of the tree decoder
+//     control.
 #include <mutex>
 
 #include "kernels.h"
