@@ -278,9 +278,8 @@ int asr_spec_synth_drafts(asr_spec_handle h, const int32_t* truth, const int32_t
 /* ---- Kernel test entry (not part of the paper's method) ------------------
  * C[m][n] = sum_k A[m][k] * B[n][k] through the tcgen05 tensor-core GEMM
  * (impl 0), the same with a 3-way K split over a global workspace (impl 2) or
- * with K split inside a thread-block cluster and wide N tiles (impl 4), with
- * 64-wide N tiles clustered per M tile and A tiles multicast (impl 5; 65 to
- * 512 columns), or the SIMT GEMM (impl 1);
+ * with K split inside a thread-block cluster and wide N tiles (impl 4), or
+ * the SIMT GEMM (impl 1);
  * impl 3 runs the LM-head epilogue instead and writes C[n] = the index m of
  * the largest value of column n (lowest m on ties).  A, B bf16 row-major
  * device arrays, C fp32.  K % 64 == 0.  Synchronous. */

@@ -104,7 +104,6 @@ struct asr_spec {
   bool cur_tree = false;
   unsigned long long* vf_trace = nullptr;   // per-stage timestamps of the fused kernel (diagnostics)
   bool vf_trace_on = false;
-  bool use_mc = false;        // multicast weight tiles across the row tiles (ASRSPEC_MC=1; slower as measured)
   int wide_bn = 64;      // N tile for many rows (ASRSPEC_WIDE_BN: 64, 128, 192, 224, 256)
   int wide_target = 2 * 152;   // CTAs a many-row GEMM may fill by splitting K (ASRSPEC_WIDE_TARGET)
   int few_target = 2 * 152;    // the same for few rows (ASRSPEC_FEW_TARGET)
@@ -275,7 +274,6 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
     while (g.splits < 16 && tiles * g.splits * 2 <= target && g.splits * 2 <= (N <= 64 ? nkb : nkb / 4))
       g.splits *= 2;
   g.cluster = g.splits > 1;
-  g.mc = h->use_mc && N > 64 && g.splits == 1;
   g.pdl = h->use_pdl;
   g.ws = h->ws;
   g.tickets = h->tickets;
@@ -621,7 +619,6 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   h->anchor = dims->anchor_layer >= 0 ? dims->anchor_layer : (3 * h->L) / 4;
   h->bf16 = dims->dtype == 1;
   if (const char* e = std::getenv("ASRSPEC_PDL")) h->use_pdl = std::atoi(e) != 0;
-  if (const char* e = std::getenv("ASRSPEC_MC")) h->use_mc = std::atoi(e) != 0;
   if (const char* e = std::getenv("ASRSPEC_WIDE_BN")) {
     const int v = std::atoi(e);
     if (v == 64 || v == 128 || v == 192 || v == 224 || v == 256) h->wide_bn = v;
@@ -1264,8 +1261,7 @@ int asr_spec_test_gemm(int32_t impl, const void* A, const void* B, float* C, int
     cudaFree(status);
   } else {
     TcGemm g{};
-    g.bn = impl == 4 && N > 64 ? tc_pick_bn_wide(N) : impl == 5 ? 64 : tc_pick_bn(N);
-    g.mc = impl == 5;   // N tiles of an M tile in one cluster, weight tiles multicast
+    g.bn = impl == 4 && N > 64 ? tc_pick_bn_wide(N) : tc_pick_bn(N);
     if (!make_tmap_bf16(&g.mapA, A, M, K, 128) || !make_tmap_bf16(&g.mapB, B, N, K, g.bn)) return ASR_E_INVAL;
     g.M = M;
     g.N = N;

@@ -54,11 +54,7 @@ struct TcCfg {
 };
 
 
-// MC: the N tiles of one M tile form a cluster (grid y = cluster y); each
-// k-block's A tile is loaded once, by CTA (k-block mod cluster size), and
-// multicast to every CTA of the cluster; an MMA commit frees the slot in all
-// of them, so a slot is refilled only after every CTA has consumed it.
-template <int BN, int MODE, bool CLU, bool MC>
+template <int BN, int MODE, bool CLU>
 __global__ void __launch_bounds__(128, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, int K, int splits,
                float* __restrict__ ws, int* __restrict__ tickets, Epi epi, int* status) {
@@ -79,13 +75,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   __shared__ float ln_mu[BN], ln_rs[BN];   // folded LayerNorm: statistics of the tile's rows
 
   // Grid: cluster split: (M tiles x splits, N tiles), the splits of a tile
-  // consecutive along x (one cluster); multicast: (M tiles, N tiles), the N
-  // tiles of an M tile one cluster; otherwise (N tiles, M tiles, splits), so
+  // consecutive along x (one cluster); otherwise (N tiles, M tiles, splits), so
   // that the CTAs sharing a weight tile run together and read it from HBM once.
-  int tile_m = CLU ? (int)blockIdx.x / splits : MC ? (int)blockIdx.x : (int)blockIdx.y;
+  int tile_m = CLU ? (int)blockIdx.x / splits : (int)blockIdx.y;
   const int split = CLU ? (int)blockIdx.x % splits : (int)blockIdx.z;
-  int tile_n = (CLU || MC) ? (int)blockIdx.y : (int)blockIdx.x;
-  if (!CLU && !MC && epi.group_m > 0) {   // grouped order: a band of group_m M tiles sweeps the N tiles
+  int tile_n = CLU ? (int)blockIdx.y : (int)blockIdx.x;
+  if (!CLU && epi.group_m > 0) {   // grouped order: a band of group_m M tiles sweeps the N tiles
     const int mt = (epi.M + TC_BM - 1) / TC_BM, nt = (epi.N + BN - 1) / BN;
     const int band = (int)blockIdx.x / (epi.group_m * nt);
     const int r = (int)blockIdx.x - band * epi.group_m * nt;
@@ -116,14 +111,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       mr = (b + 1) * epi.t_max;
     }
   }
-  if (!MC && (n0 >= n_valid || nkb <= 0 || dead)) {   // uniform over the CTA and over all splits of a tile
+  if (n0 >= n_valid || nkb <= 0 || dead) {   // uniform over the CTA and over all splits of a tile
     pdl_wait();
     return;
   }
-  // multicast clusters keep every CTA: the others wait on its share of A and its commits
-  const uint32_t mc_rank = MC ? cluster_ctarank() : 0;
-  const uint32_t mc_size = MC ? gridDim.y : 1;
-  const uint16_t mc_mask = (uint16_t)((1u << mc_size) - 1u);
 
   if (warp == 0) {
     __syncwarp();   // warp-aligned allocation
@@ -133,7 +124,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   if (threadIdx.x == 32) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], MC ? mc_size : 1);
+      mbar_init(&empty[s], 1);
     }
     mbar_init(done, 1);
     if constexpr (PUSH) {
@@ -146,7 +137,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if constexpr (MC) cluster_sync();   // every CTA's barriers exist before any multicast lands
   // push split: announce this CTA's receive barrier; the matching wait comes
   // just before the first remote store, long after every peer has arrived
   if constexpr (PUSH) cluster_arrive_relaxed();
@@ -162,12 +152,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     const int first = nkb < C::STAGES ? nkb : C::STAGES;
     for (int i = 0; i < first; ++i) {
       mbar_arrive_expect_tx(&full[i], TX);
-      if constexpr (MC) {
-        if ((uint32_t)((kb0 + i) % (int)mc_size) == mc_rank)
-          tma_load_2d_mc(sA + i * C::A_BYTES, &mapA, &full[i], (kb0 + i) * TC_BK, m0, mc_mask);
-      } else {
-        tma_load_2d(sA + i * C::A_BYTES, &mapA, &full[i], (kb0 + i) * TC_BK, m0);
-      }
+      tma_load_2d(sA + i * C::A_BYTES, &mapA, &full[i], (kb0 + i) * TC_BK, m0);
     }
     pdl_wait();
     tl_mark(epi.tl, TL_WORK);
@@ -179,12 +164,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       const uint32_t ph = (i / C::STAGES) & 1;
       if (!mbar_wait(&empty[s], ph ^ 1, status)) break;
       mbar_arrive_expect_tx(&full[s], TX);
-      if constexpr (MC) {
-        if ((uint32_t)((kb0 + i) % (int)mc_size) == mc_rank)
-          tma_load_2d_mc(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0, mc_mask);
-      } else {
-        tma_load_2d(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0);
-      }
+      tma_load_2d(sA + s * C::A_BYTES, &mapA, &full[s], (kb0 + i) * TC_BK, m0);
       tma_load_2d(sB + s * C::B_BYTES, &mapB, &full[s], (kb0 + i) * TC_BK, n0);
       issued = i + 1;
     }
@@ -205,8 +185,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       for (int kk = 0; kk < TC_BK / 16; ++kk)
         umma_bf16(tmem, umma_desc_sw128(a_addr + kk * 32), umma_desc_sw128(b_addr + kk * 32), idesc,
                   (i | kk) != 0);
-      if constexpr (MC) umma_commit_mc(&empty[s], mc_mask);
-      else umma_commit(&empty[s]);
+      umma_commit(&empty[s]);
     }
     umma_commit(done);
   }
@@ -625,9 +604,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   }
 
   if (tr && threadIdx.x == 0) tr[4] = global_ns();
-  // a multicast cluster stays until every CTA's commits (which arrive in all
-  // CTAs) have landed
-  if constexpr (MC) cluster_sync();
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
@@ -706,29 +682,17 @@ int tc_pick_bn_wide(int n) {
   return best;
 }
 
-template <int BN>
-constexpr bool mc_capable() {
-  return BN == 64 || BN == 128;
-}
-
 template <int BN, int MODE>
 static void launch_tc_t(const TcGemm& g, const Epi& epi, int* status, cudaStream_t st) {
   const int mt = (g.M + TC_BM - 1) / TC_BM, nt = (g.N + BN - 1) / BN;
   if (g.cluster && g.splits > 1) {
-    launch_ex(gemm_tc_kernel<BN, MODE, true, false>, dim3(mt * g.splits, nt, 1), dim3(128),
+    launch_ex(gemm_tc_kernel<BN, MODE, true>, dim3(mt * g.splits, nt, 1), dim3(128),
               TcCfg<BN, (BN <= 64)>::SMEM, st, g.pdl, g.splits, g.mapA, g.mapB, g.K, g.splits, g.ws, g.tickets, epi,
               status);
     return;
   }
-  if constexpr (mc_capable<BN>()) {
-    if (g.mc && g.splits == 1 && nt >= 2 && nt <= 8) {
-      launch_ex2(gemm_tc_kernel<BN, MODE, false, true>, dim3(mt, nt, 1), dim3(128), TcCfg<BN>::SMEM, st, g.pdl, 1,
-                 nt, g.mapA, g.mapB, g.K, 1, g.ws, g.tickets, epi, status);
-      return;
-    }
-  }
   const dim3 grid = epi.group_m > 0 ? dim3(nt * mt, 1, g.splits) : dim3(nt, mt, g.splits);
-  launch_ex(gemm_tc_kernel<BN, MODE, false, false>, grid, dim3(128), TcCfg<BN>::SMEM, st, g.pdl, 1, g.mapA, g.mapB,
+  launch_ex(gemm_tc_kernel<BN, MODE, false>, grid, dim3(128), TcCfg<BN>::SMEM, st, g.pdl, 1, g.mapA, g.mapB,
             g.K, g.splits, g.ws, g.tickets, epi, status);
 }
 
@@ -747,14 +711,11 @@ static void launch_tc_mode(const TcGemm& g, const Epi& epi, int* status, cudaStr
 
 template <int BN, int MODE>
 static void configure_one() {
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        TcCfg<BN>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        TcCfg<BN, (BN <= 64)>::SMEM);
-  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true, false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if constexpr (mc_capable<BN>())
-    cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         TcCfg<BN>::SMEM);
+  cudaFuncSetAttribute(gemm_tc_kernel<BN, MODE, true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
 
 template <int MODE>

@@ -22,7 +22,6 @@ struct TcGemm {
   int* tickets;  // workspace split: one zeroed int per output tile
   bool cluster = false;  // split K inside a thread-block cluster (splits in {2,4,8,16})
   bool pdl = false;      // programmatic dependent launch after the previous kernel
-  bool mc = false;       // many rows: cluster the N tiles of an M tile and multicast A (2..8 tiles)
 };
 
 bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);

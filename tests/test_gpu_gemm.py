@@ -10,12 +10,10 @@ SHAPES = [(128, 16, 64), (300, 9, 1280), (3840, 9, 1280), (1280, 40, 5120), (517
           (3840, 448, 1280)]
 
 
-@pytest.mark.parametrize("impl", [0, 2, 4, 5, 1])
+@pytest.mark.parametrize("impl", [0, 2, 4, 1])
 @pytest.mark.parametrize("M,N,K", SHAPES)
 def test_gemm_matches_torch(built_lib, cuda, impl, M, N, K):
     from paper_2608_12703_gb300 import asrspec as A
-    if impl == 5 and not (64 < N <= 512):
-        pytest.skip("multicast clusters need 2..8 row tiles of 64")
     g = torch.Generator(device="cpu").manual_seed(M * 7 + N * 3 + K)
     a = torch.randn(M, K, generator=g).to(torch.bfloat16).to(cuda)
     b = torch.randn(N, K, generator=g).to(torch.bfloat16).to(cuda)
