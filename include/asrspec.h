@@ -164,6 +164,21 @@ int asr_spec_verify_tree(asr_spec_handle h, const int32_t* tokens, const int32_t
                          int32_t n, int32_t* accepted, int32_t* bonus, int32_t* kv_len, int32_t* anchor,
                          int32_t* path);
 
+/* The restart flags of the last verify (Sec. 3: after a rejected draft the
+ * next round restarts drafting from the verified position, else it
+ * continues): restart[b] = 1 when accepted[b] < lens[b] (linear verify) or
+ * when the accepted path's last node has children (tree verify), 0 when every
+ * offered draft was accepted and for utterances that sat out.  [B] int32,
+ * stream-ordered after the verify call.  Errors: ASR_E_STATE (no prefill). */
+int asr_spec_restart(asr_spec_handle h, int32_t* restart);
+
+/* Test support: the head-mean attention profile behind the last verify's
+ * anchors (Sec. 5 "Verification-Attention Correction": the mean over heads of
+ * the per-head softmax attention of the anchor row at the anchor layer).
+ * out: [B][max_enc] fp32; entries at frames >= enc_len[b], and every entry of
+ * an utterance that sat out, are stale. */
+int asr_spec_debug_anchor_profile(asr_spec_handle h, float* out);
+
 /* Roll the committed cache back (App. "Decoding and Intervention Protocol":
  * the cached states of accepted tokens are what the next round reuses):
  * kv_len[b] <- new_len[b] (which must not exceed the current kv_len[b]) and

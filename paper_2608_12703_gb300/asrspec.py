@@ -28,7 +28,8 @@ EXPORTED = [
     "asr_spec_status", "asr_spec_last_error", "asr_spec_destroy", "asr_spec_synth_drafts",
     "asr_spec_test_gemm", "asr_spec_set_graphs", "asr_spec_profile", "asr_spec_profile_read",
     "asr_spec_gemm_noalloc", "asr_spec_timeline", "asr_spec_timeline_read",
-    "asr_spec_fused_trace", "asr_spec_fused_trace_read", "asr_spec_verify_tree",
+    "asr_spec_fused_trace", "asr_spec_fused_trace_read", "asr_spec_verify_tree", "asr_spec_restart",
+    "asr_spec_debug_anchor_profile",
 ]
 PROF_CLASSES = ["qkv", "resid", "query", "mlp_up", "self_attn", "cross_attn", "lm_head", "layernorm", "other",
                 "fused"]
@@ -81,6 +82,8 @@ def lib():
     L.asr_spec_verify.argtypes = [vp, p32, p32, i32, p32, p32, p32, p32]
     L.asr_spec_verify_tree.argtypes = [vp, p32, p32, p32, i32, p32, p32, p32, p32, p32]
     L.asr_spec_rollback.argtypes = [vp, p32, p32]
+    L.asr_spec_restart.argtypes = [vp, p32]
+    L.asr_spec_debug_anchor_profile.argtypes = [vp, vp]
     L.asr_spec_state.argtypes = [vp, p32, p32]
     L.asr_spec_debug_logits.argtypes = [vp, vp, i32]
     L.asr_spec_status.argtypes = [vp]
@@ -156,6 +159,14 @@ def asr_spec_verify(h, draft, lens, k, accepted, bonus, kv_len, anchor):
 def asr_spec_verify_tree(h, tokens, parent, lens, n, accepted, bonus, kv_len, anchor, path):
     return _check(h, lib().asr_spec_verify_tree(h, ptr(tokens), ptr(parent), ptr(lens), n, ptr(accepted), ptr(bonus),
                                                 ptr(kv_len), ptr(anchor), ptr(path)), "asr_spec_verify_tree")
+
+
+def asr_spec_restart(h, restart):
+    return _check(h, lib().asr_spec_restart(h, ptr(restart)), "asr_spec_restart")
+
+
+def asr_spec_debug_anchor_profile(h, out):
+    return _check(h, lib().asr_spec_debug_anchor_profile(h, ptr(out)), "asr_spec_debug_anchor_profile")
 
 
 def asr_spec_rollback(h, new_len, new_pending):

@@ -57,7 +57,9 @@ struct asr_spec {
   unsigned long long* row_key = nullptr;
   unsigned long long* frame_key = nullptr;  // [Bmax] keys + [Bmax] int tickets
   int* anchor_row = nullptr;
+  // out4: accepted, bonus, kv_len, anchor and restart of the last verify, [Bmax] each
   int *draft_buf = nullptr, *lens_buf = nullptr, *prompt_buf = nullptr, *out4 = nullptr, *misc = nullptr;
+  float* anchor_prof = nullptr;   // [Bmax][Tmax] head-mean profile of the last verify's anchor rows
   int* status = nullptr;
   float* ws = nullptr;
   size_t ws_floats = 0;
@@ -571,6 +573,8 @@ int enqueue_verify(asr_spec* h, int k) {
   A.bonus = h->out4 + h->Bmax;
   A.kv_len_out = h->out4 + 2 * h->Bmax;
   A.anchor_out = h->out4 + 3 * h->Bmax;
+  A.restart = h->out4 + 4 * h->Bmax;
+  A.profile = h->anchor_prof;
   A.q_anchor = h->q_anchor;
   A.ml = h->ml;
   const size_t cross_half = (size_t)h->Bmax * h->H * h->Tmax * 64 * h->es;
@@ -821,7 +825,8 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
     return finish(rc);
   if ((rc = dalloc(h, &h->draft_buf, (size_t)h->Bmax * std::max(h->kmax, 1) * 4)) ||
       (rc = dalloc(h, &h->lens_buf, h->Bmax * 4)) || (rc = dalloc(h, &h->prompt_buf, (size_t)h->Bmax * h->maxpos * 4)) ||
-      (rc = dalloc(h, &h->out4, 4 * h->Bmax * 4)) || (rc = dalloc(h, &h->misc, 64 * 4)) ||
+      (rc = dalloc(h, &h->out4, 5 * h->Bmax * 4)) || (rc = dalloc(h, &h->misc, 64 * 4)) ||
+      (rc = dalloc(h, &h->anchor_prof, (size_t)h->Bmax * h->Tmax * 4)) ||
       (rc = dalloc(h, &h->status, 4)))
     return finish(rc);
   CK(cudaMemset(h->status, 0, 4));
@@ -1039,6 +1044,24 @@ int asr_spec_verify_tree(asr_spec_handle h, const int32_t* tokens, const int32_t
   if (!lens || (n > 0 && (!tokens || !parent || !path)) || !accepted || !bonus || !kv_len || !anchor)
     return fail(h, ASR_E_INVAL, "null pointer");
   return verify_call(h, tokens, n > 0 ? parent : nullptr, lens, n, accepted, bonus, kv_len, anchor, path);
+}
+
+int asr_spec_restart(asr_spec_handle h, int32_t* restart) {
+  if (!h || !restart) return ASR_E_INVAL;
+  if (h->state < 2) return fail(h, ASR_E_STATE, "restart flags before prefill");
+  if (int rc = copy_out(h, restart, h->out4 + 4 * h->Bmax, h->B)) return rc;
+  if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
+}
+
+int asr_spec_debug_anchor_profile(asr_spec_handle h, float* out) {
+  if (!h || !out) return ASR_E_INVAL;
+  if (h->state < 2) return fail(h, ASR_E_STATE, "anchor profile before prefill");
+  const size_t bytes = (size_t)h->B * h->Tmax * 4;
+  CK(cudaMemcpyAsync(out, h->anchor_prof, bytes, h->host_io ? cudaMemcpyDeviceToHost : cudaMemcpyDeviceToDevice,
+                     h->st));
+  if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
 }
 
 int asr_spec_set_graphs(asr_spec_handle h, int enable) {

@@ -256,6 +256,7 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
       A.bonus[b] = -1;
       A.kv_len_out[b] = A.kv_len[b];
       A.anchor_out[b] = -1;
+      A.restart[b] = 0;
     }
     __syncthreads();
     if (rows > 0) mbar_wait(&bar, 0, A.status);       // no CTA leaves with copies in flight
@@ -282,10 +283,12 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
       ++n;
     }
     const int g = __shfl_sync(0xffffffffu, tok, c);
+    const unsigned kids = __ballot_sync(0xffffffffu, my_par == c);   // the last node's children
     if (lane == 0) {
       s_n = n;
       s_node = c;
       if (blockIdx.x == 0) {
+        A.restart[b] = kids != 0u;   // a child of the last node was rejected
         for (int j = n; j < A.k; ++j) A.path[(size_t)b * A.k + j] = -1;
         const int nl = A.kv_len[b] + 1 + n;
         A.accepted[b] = n;
@@ -314,6 +317,7 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
         A.kv_len[b] = nl;
         A.kv_len_out[b] = nl;
         A.pending[b] = g;
+        A.restart[b] = n < l;   // a draft was rejected: the next round restarts
       }
     }
   }
@@ -369,6 +373,7 @@ accept_anchor_kernel(AcceptAnchorArgs A) {
     const int fr = lane < FB ? lane : 0;
     for (int h = 0; h < H; ++h) pbar += ph[h][fr];
     pbar /= (float)H;
+    if (lane < rows) A.profile[(size_t)b * A.t_alloc + f0 + lane] = pbar;
     unsigned long long key = lane < rows ? argmax_key(pbar, (uint32_t)(f0 + lane)) : 0ull;
     key = warp_max_u64(key);
     if (lane == 0) {

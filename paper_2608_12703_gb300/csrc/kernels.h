@@ -126,6 +126,8 @@ struct AcceptAnchorArgs {
   int* kv_len;
   int* pending;
   int *accepted, *bonus, *kv_len_out, *anchor_out;
+  int* restart;                     // [B]: 1 when the next round restarts (a draft was rejected), else 0
+  float* profile;                   // [B][t_alloc]: the head-mean profile of the anchor row (test readback)
   const float* q_anchor;            // [R][d] cross-attention queries at the anchor layer
   const float* ml;                  // [R][H][2] their softmax (max, sum)
   const void* kc;                   // anchor layer's encoder keys [B_max][H][t_alloc][64]

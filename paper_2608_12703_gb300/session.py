@@ -30,6 +30,7 @@ class StepOut:
     bonus: np.ndarray
     kv_len: np.ndarray
     anchor: np.ndarray
+    restart: np.ndarray
 
 
 class Session:
@@ -44,7 +45,7 @@ class Session:
         self.max_batch, self.max_draft = max_batch, max_draft
         self.B = 0
         with torch.cuda.stream(self.stream):
-            self.out = torch.zeros((4, max_batch), dtype=torch.int32, device=self.dev)
+            self.out = torch.zeros((5, max_batch), dtype=torch.int32, device=self.dev)
         self.host_io = False
 
     @property
@@ -95,16 +96,18 @@ class Session:
         k = draft.shape[1] if k is None else k
         lens = np.asarray(lens, dtype=np.int32)
         if self.host_io:
-            acc, bon, kvl, anc = (np.zeros(self.B, np.int32) for _ in range(4))
+            acc, bon, kvl, anc, rst = (np.zeros(self.B, np.int32) for _ in range(5))
             A.asr_spec_verify(self.h, np.ascontiguousarray(draft[:, :k]), lens, k, acc, bon, kvl, anc)
-            return StepOut(acc, bon, kvl, anc)
+            A.asr_spec_restart(self.h, rst)
+            return StepOut(acc, bon, kvl, anc, rst)
         with torch.cuda.stream(self.stream):
             d = torch.from_numpy(np.ascontiguousarray(draft[:, :k])).to(self.dev)
             l = torch.from_numpy(lens).to(self.dev)
             o = self.out[:, :self.B]
             A.asr_spec_verify(self.h, d, l, k, o[0], o[1], o[2], o[3])
+            A.asr_spec_restart(self.h, o[4])
             oh = o.cpu().numpy()
-        return StepOut(oh[0].copy(), oh[1].copy(), oh[2].copy(), oh[3].copy())
+        return StepOut(*(oh[i].copy() for i in range(5)))
 
     def verify_tree(self, tokens, parent, lens):
         """Tree verify: tokens / parent [B][n] (node i + 1's token and parent),
@@ -114,10 +117,11 @@ class Session:
         n = tokens.shape[1]
         lens = np.asarray(lens, dtype=np.int32)
         if self.host_io:
-            acc, bon, kvl, anc = (np.zeros(self.B, np.int32) for _ in range(4))
+            acc, bon, kvl, anc, rst = (np.zeros(self.B, np.int32) for _ in range(5))
             path = np.full((self.B, max(n, 1)), -1, dtype=np.int32)
             A.asr_spec_verify_tree(self.h, tokens, parent, lens, n, acc, bon, kvl, anc, path)
-            return StepOut(acc, bon, kvl, anc), path[:, :n]
+            A.asr_spec_restart(self.h, rst)
+            return StepOut(acc, bon, kvl, anc, rst), path[:, :n]
         with torch.cuda.stream(self.stream):
             t = torch.from_numpy(tokens).to(self.dev)
             p = torch.from_numpy(parent).to(self.dev)
@@ -125,9 +129,10 @@ class Session:
             path = torch.full((self.B, max(n, 1)), -1, dtype=torch.int32, device=self.dev)
             o = self.out[:, :self.B]
             A.asr_spec_verify_tree(self.h, t, p, l, n, o[0], o[1], o[2], o[3], path)
+            A.asr_spec_restart(self.h, o[4])
             oh = o.cpu().numpy()
             ph = path.cpu().numpy()[:, :n]
-        return StepOut(oh[0].copy(), oh[1].copy(), oh[2].copy(), oh[3].copy()), ph
+        return StepOut(*(oh[i].copy() for i in range(5))), ph
 
     def host(self, t) -> np.ndarray:
         """Copy a device tensor written on this session's stream to the host."""
@@ -161,6 +166,14 @@ class Session:
             R = A.asr_spec_debug_logits(self.h, out, max_rows)
         self.stream.synchronize()
         return out[:R]
+
+    def anchor_profile(self) -> np.ndarray:
+        """The head-mean attention profiles behind the last verify's anchors, [B][max_enc]."""
+        with torch.cuda.stream(self.stream):
+            out = torch.empty((self.B, self.dims.max_enc), dtype=torch.float32, device=self.dev)
+            A.asr_spec_debug_anchor_profile(self.h, out)
+        self.stream.synchronize()
+        return out.cpu().numpy()
 
     def status(self) -> int:
         return A.asr_spec_status(self.h)

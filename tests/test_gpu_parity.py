@@ -1,16 +1,21 @@
 """The CUDA draft-verify step against the CPU oracle (teacher-forced, every round).
 
-Sizes: the tiny fp32 workload in full; the small bf16 decoder with a batch of
+Sizes: every workload at its full configuration -- the tiny fp32 decoder in
+full; the small decoder's batch-16 workload and all sixteen (k, error rate)
+points of the batch-32 acceptance/rollback sweep, with the oracle following
+sampled utterances through their whole transcripts; the large decoder's
+224-token batch-1 decode in full and its batch-64 workload with three sampled
+utterances followed to the end.  Also: the small decoder with a batch of
 ragged utterances (several GEMM tiles, a ragged encoder tail); edge cases
 (k = 0, sitting-out utterances, one encoder frame, a one-token prompt, k = 16,
-the context capacity); and the large decoder at full size on sampled rounds
-and sampled utterances of the batch-64 workload.
+the context capacity); long-form encoder memories.
 """
 import numpy as np
 import pytest
 
 import workload as W
-from tests.parity import ParityStats, compare_round, run_decode, scale_for
+from tests.parity import (ParityStats, assert_bounded, compare_round, run_decode, run_sampled_decode,
+                          sampled_truth, scale_for)
 
 pytestmark = pytest.mark.gpu
 
@@ -47,6 +52,7 @@ def test_tiny_fp32_full_workload(built_lib, cuda):
     _report(wl.name, st)
     assert st.emitted == sum(wl.n_out)
     assert st.near_ties == 0
+    assert st.anchor_near == 0
 
 
 @pytest.mark.parametrize("std,ln_kernel", [(0.02, False), (0.05, False), (0.02, True)])
@@ -67,6 +73,7 @@ def test_small_bf16_ragged_batch(built_lib, cuda, monkeypatch, std, ln_kernel):
                        _session(dims, blob, 5, 8), scale=scale_for(dims, std))
     _report(f"small std={std}{' ln-kernel' if ln_kernel else ''}", st)
     assert st.rows > 50
+    assert_bounded(st)
 
 
 def test_edge_cases_bf16(built_lib, cuda):
@@ -85,6 +92,7 @@ def test_edge_cases_bf16(built_lib, cuda):
     st, _ = run_decode(dims, blob, enc, enc_lens, prompt, total, 16, corr, _session(dims, blob, 3, 16),
                        k_schedule=sched, scale=scale_for(dims, 0.1))
     _report("edges", st)
+    assert_bounded(st)
 
 
 def test_edge_cases_fp32(built_lib, cuda):
@@ -102,23 +110,28 @@ def test_edge_cases_fp32(built_lib, cuda):
     assert st.near_ties == 0
 
 
-def test_large_bf16_batch1_sampled_rounds(built_lib, cuda):
-    """Full-size large decoder, batch 1, k = 8 with slipped drafts: the first rounds."""
+@pytest.mark.slow
+def test_large_bf16_batch1_full_decode(built_lib, cuda):
+    """Full-size large decoder, batch 1, k = 8 with a slip every round: the
+    whole 224-token decode, logits of every row checked."""
     wl = W.CONFIGS["large-bf16-b1-k8"]
     dims = wl.dims
     blob = _blob(dims)
     enc = W.make_encoder_states(dims, wl.enc_lens, wl.t_max)
     prompt = W.make_prompt(dims, 1)
-    total = [W.PROMPT_LEN + 24]
-    st, _ = run_decode(dims, blob, enc, list(wl.enc_lens), prompt, total, wl.k, W.make_corruption(wl),
-                       _session(dims, blob, 1, wl.k), max_rounds=6)
+    st, _ = run_decode(dims, blob, enc, list(wl.enc_lens), prompt, list(wl.total_lens), wl.k,
+                       W.make_corruption(wl), _session(dims, blob, 1, wl.k))
     _report(wl.name, st)
+    assert st.emitted == sum(wl.n_out)
+    assert_bounded(st)
 
 
-def test_large_bf16_batch64_sampled_utterances(built_lib, cuda):
-    """Full-size batch-64 verify (448 rows, ragged encoder lengths); the oracle
-    follows three of the utterances, the others take the workload's drafts."""
-    from oracle import Oracle, greedy_transcript
+@pytest.mark.slow
+def test_large_bf16_batch64_sampled_full_decode(built_lib, cuda):
+    """Full-size batch-64 verify (448 rows, ragged encoder lengths): the oracle
+    follows utterances 0, 7 and 63 through their whole transcripts (29, 54 and
+    65 tokens); their logits are compared every round while the other 61
+    utterances decode alongside."""
     from paper_2608_12703_gb300.session import Session
     wl = W.CONFIGS["large-bf16-b64-k6"]
     dims = wl.dims
@@ -126,35 +139,73 @@ def test_large_bf16_batch64_sampled_utterances(built_lib, cuda):
     sample = [0, 7, 63]
     enc = W.make_encoder_states(dims, wl.enc_lens, wl.t_max)
     prompt = W.make_prompt(dims, wl.batch)
-    total = np.array(wl.total_lens)
-    orc = Oracle(dims, blob)
-    orc.encode_cache(enc[sample], [wl.enc_lens[i] for i in sample])
-    orc.prefill(prompt[sample])
-    snap = orc.snapshot()
-    truth_s = greedy_transcript(orc, prompt[sample], np.minimum(total[sample], W.PROMPT_LEN + 16))
-    orc.restore(snap)
-    truth = np.zeros((wl.batch, dims.max_pos), dtype=np.int64)
-    truth[:, :W.PROMPT_LEN] = prompt
-    for j, b in enumerate(sample):
-        truth[b, :truth_s.shape[1]] = np.where(truth_s[j] >= 0, truth_s[j], 0)
-    corr = W.make_corruption(wl)
+    orc, snap, truth = sampled_truth(dims, blob, wl, sample, enc, prompt)
     sess = Session(dims, blob, max_batch=wl.batch, max_draft=wl.k)
-    sess.encode_cache(enc, list(wl.enc_lens))
-    sess.prefill(prompt)
-    st = ParityStats()
-    kv = np.full(wl.batch, W.PROMPT_LEN - 1)
-    lim = total.copy()
-    lim[sample] = np.minimum(total[sample], W.PROMPT_LEN + 16)
-    for _ in range(4):
-        kv[sample] = orc.kv_len
-        draft, lens = W.make_drafts(truth, lim, kv, wl.k, corr)
-        if np.all(lens[sample] < 0):
-            break
-        ro, rg = compare_round(orc, sess, draft, lens, st, sample=sample)
-        kv = rg.kv_len.copy()
-    _report(wl.name, st)
-    assert sess.status() == 0
+    st = run_sampled_decode(orc, snap, truth, sess, wl, sample, enc, prompt)
     sess.close()
+    _report(wl.name, st)
+    assert st.emitted == sum(wl.n_out[b] for b in sample)
+    assert_bounded(st)
+
+
+@pytest.mark.slow
+def test_small_bf16_batch16_sampled_full_decode(built_lib, cuda):
+    """The small decoder's batch-16 workload (1500 frames each, 128 tokens,
+    k = 8, error rate 0.25): the oracle follows four utterances through their
+    whole transcripts; 144 rows per round."""
+    from paper_2608_12703_gb300.session import Session
+    wl = W.CONFIGS["small-bf16-b16-k8"]
+    dims = wl.dims
+    blob = _blob(dims)
+    sample = [0, 5, 10, 15]
+    enc = W.make_encoder_states(dims, wl.enc_lens, wl.t_max)
+    prompt = W.make_prompt(dims, wl.batch)
+    orc, snap, truth = sampled_truth(dims, blob, wl, sample, enc, prompt)
+    sess = Session(dims, blob, max_batch=wl.batch, max_draft=wl.k)
+    st = run_sampled_decode(orc, snap, truth, sess, wl, sample, enc, prompt)
+    sess.close()
+    _report(wl.name, st)
+    assert st.emitted == sum(wl.n_out[b] for b in sample)
+    assert_bounded(st)
+
+
+_SWEEP = {}
+
+
+def _sweep_state():
+    """One GPU session (batch 32, k up to 16) and one oracle snapshot shared by
+    the sixteen sweep configurations: they differ only in k, the error rate
+    and the corruption stream."""
+    if "sess" not in _SWEEP:
+        from paper_2608_12703_gb300.session import Session
+        wl = W.CONFIGS["small-bf16-b32-k16-p0.05"]
+        dims = wl.dims
+        blob = _blob(dims)
+        sample = [0, 31]
+        enc = W.make_encoder_states(dims, wl.enc_lens, wl.t_max)
+        prompt = W.make_prompt(dims, wl.batch)
+        orc, snap, truth = sampled_truth(dims, blob, wl, sample, enc, prompt)
+        _SWEEP.update(sess=Session(dims, blob, max_batch=wl.batch, max_draft=16), orc=orc, snap=snap,
+                      truth=truth, sample=sample, enc=enc, prompt=prompt)
+    return _SWEEP
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("k", [2, 4, 8, 16])
+@pytest.mark.parametrize("p", [0.05, 0.2, 0.5, 0.8])
+def test_acceptance_rollback_sweep(built_lib, cuda, k, p):
+    """The acceptance/rollback sweep (small decoder, batch 32, 1500 frames,
+    128 tokens; half the rounds carry a one-token slip that forces a rejection
+    and a restart): for every (k, error rate) the oracle follows utterances 0
+    and 31 through their whole transcripts, logits checked every round, with
+    all 32 utterances scored (up to 544 rows at k = 16)."""
+    S = _sweep_state()
+    wl = W.CONFIGS[f"small-bf16-b32-k{k}-p{p:g}"]
+    st = run_sampled_decode(S["orc"], S["snap"], S["truth"], S["sess"], wl, S["sample"], S["enc"], S["prompt"])
+    _report(wl.name, st)
+    assert st.emitted == sum(wl.n_out[b] for b in S["sample"])
+    assert st.restarts > 0
+    assert_bounded(st)
 
 
 def test_long_form_encoder_memory(built_lib, cuda):
@@ -173,3 +224,4 @@ def test_long_form_encoder_memory(built_lib, cuda):
                        _session(dims, blob, 2, 8), max_rounds=6)
     _report("long-form 5200 + 2100 frames", st)
     assert st.rows > 20
+    assert_bounded(st)

@@ -51,7 +51,7 @@ def _compare_tree(orc, sess, tokens, parent, lens, st, scale=1.0):
     diverged = False
     for b in range(len(lens)):
         if lens[b] < 0:
-            assert rg.bonus[b] == -1 and rg.anchor[b] == -1 and rg.accepted[b] == 0
+            assert rg.bonus[b] == -1 and rg.anchor[b] == -1 and rg.accepted[b] == 0 and rg.restart[b] == 0
             assert rg.kv_len[b] == ro.kv_len[b]
             continue
         nrow = int(lens[b]) + 1
@@ -66,6 +66,9 @@ def _compare_tree(orc, sess, tokens, parent, lens, st, scale=1.0):
         else:
             assert rg.kv_len[b] == ro.kv_len[b]
             assert np.all(path[b, rg.accepted[b]:] == -1)
+            # the tree's restart flag: the path's last node has children (R16)
+            assert rg.restart[b] == ro.restart[b], (b, rg.restart[b], ro.restart[b])
+            st.restarts += int(rg.restart[b])
             st.anchors += 1
             prof = ro.anchor_profile[b]
             if rg.anchor[b] == ro.anchor[b]:
