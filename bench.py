@@ -391,20 +391,30 @@ NCU_TRAFFIC = {
 # Launch kinds of the timeline (ASR_TL_*; a LayerNorm-fused GEMM counts with its
 # GEMM) and the profile class (CUDA events) that times the same kernel.
 TL_KIND_CLASS = {17: "qkv", 18: "resid", 19: "query", 20: "mlp_up", 22: "lm_head", 4: "self_attn",
-                 5: "cross_attn", 3: "layernorm", 7: "fused"}
+                 5: "cross_attn", 3: "layernorm", 8: "qkv_self", 9: "query_cross"}
+
+# launches of a kernel class per verify call that runs it
+CLASS_PER_CALL = {"qkv": 1, "resid": 3, "query": 1, "mlp_up": 1, "lm_head": 0, "self_attn": 1, "cross_attn": 1,
+                  "layernorm": 3, "qkv_self": 1, "query_cross": 1}
 
 
 def kind_class(kind: int):
     return TL_KIND_CLASS.get(kind - 32 if kind >= 48 else kind)
 
 
-def algorithmic_work(dims, cls, traffic):
+def algorithmic_work(dims, cls, traffic, n_launches):
     """(bytes, flops, per-unit statement) of one decode's launches of a kernel class.
     Bytes are the unique operands a launch must read from HBM: weights for a
-    projection (its activations are L2-resident), the K/V rows for attention."""
+    projection (its activations are L2-resident), the K/V rows for attention.
+    A class's verify calls are its launches over its launches per call (the
+    few-row and the tensor-core layers each run in some of a decode's calls);
+    K/V bytes, counted over all calls, are shared in proportion."""
     es = 2 if dims.dtype == "bf16" else 4
     d, L, F, V = dims.d_model, dims.n_layers, dims.d_ffn, dims.vocab
     calls, self_b, cross_b, _, rows = (float(x) for x in traffic[:5])
+    per_call = CLASS_PER_CALL.get(cls, 1) * L or 1
+    c_calls = n_launches / per_call
+    share = c_calls / calls if calls else 0.0
     mk = {"qkv": (L * 3 * d * d, "3 d^2 weights per layer"),
           "resid": (L * (2 * d * d + F * d), "d^2 + d^2 + F d weights per layer (self out, cross out, MLP down)"),
           "query": (L * d * d, "d^2 weights per layer"),
@@ -412,19 +422,24 @@ def algorithmic_work(dims, cls, traffic):
           "lm_head": (V * d, "V d weights")}
     if cls in mk:
         params, what = mk[cls]
-        return (calls * params * es, 2.0 * rows * params,
+        return (c_calls * params * es, 2.0 * rows * share * params,
                 f"{what} x {es} bytes per verify call; 2 x scored rows x those parameters in flops")
     if cls == "self_attn":
-        return self_b, 0.0, "2 (K, V) x (P_b + n_b) keys x d x 2 bytes per active utterance per layer"
+        return self_b * share, 0.0, "2 (K, V) x (P_b + n_b) keys x d x 2 bytes per active utterance per layer"
     if cls == "cross_attn":
-        return cross_b, 0.0, "2 (K, V) x T_b frames x d x 2 bytes per active utterance per layer"
-    if cls == "fused":
-        params = L * (6 * d * d + 2 * F * d) + V * d
-        return (calls * params * es + self_b + cross_b, 2.0 * rows * params,
-                "all projection and LM-head weights x %d bytes per verify call + the self and cross K/V rows read "
-                "(2 x keys x d x %d bytes per active utterance per layer); 2 x scored rows x weights in flops" % (es, es))
+        return cross_b * share, 0.0, "2 (K, V) x T_b frames x d x 2 bytes per active utterance per layer"
+    if cls == "qkv_self":
+        params = L * 3 * d * d
+        return (c_calls * params * es + self_b * share, 2.0 * rows * share * params,
+                "3 d^2 weights per layer x %d bytes per verify call + the self K/V rows read (2 x (P_b + n_b) keys "
+                "x d x %d bytes per active utterance per layer); 2 x scored rows x weights in flops" % (es, es))
+    if cls == "query_cross":
+        params = L * d * d
+        return (c_calls * params * es + cross_b * share, 2.0 * rows * share * params,
+                "d^2 weights per layer x %d bytes per verify call + the encoder K/V read (2 x T_b frames x d x %d "
+                "bytes per active utterance per layer); 2 x scored rows x weights in flops" % (es, es))
     if cls == "layernorm":
-        return rows * (3 * L + 1) * d * (4 + es), 0.0, "rows x d x (4 read + 2 written) bytes per LayerNorm"
+        return rows * share * (3 * L + 1) * d * (4 + es), 0.0, "rows x d x (4 read + 2 written) bytes per LayerNorm"
     return 0.0, 0.0, ""
 
 
@@ -450,7 +465,7 @@ def roofline(wl_name, dims, tl, ms, launches, traffic, pk):
     ci = PROF_CLASSES.index(name)
     t = ms[ci] / 1e3
     n = int(launches[ci])
-    nbytes, flops, per_unit = algorithmic_work(dims, name, traffic)
+    nbytes, flops, per_unit = algorithmic_work(dims, name, traffic, n)
     balance = pk["bf16_sus"] * 1e12 / (pk["hbm"] * 1e9)
     if flops > 0 and flops / nbytes > balance:
         bound, unit, peak, work, scale = "tensor", "TFLOP/s", pk["bf16_sus"], flops, 1e12

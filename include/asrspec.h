@@ -226,8 +226,9 @@ void asr_spec_destroy(asr_spec_handle h);
 #define ASR_PROF_LMHEAD 6     /* LM head with fused argmax */
 #define ASR_PROF_LAYERNORM 7  /* stand-alone LayerNorm */
 #define ASR_PROF_OTHER 8      /* row plan, embedding, accept + anchor, encoder cache build, prefill steps */
-#define ASR_PROF_FUSED 9      /* fused verify of a step with few rows (all layers and the LM head, one kernel) */
-#define ASR_PROF_N 10
+#define ASR_PROF_QKV_SELF 9   /* few rows: LayerNorm + QKV projection + self-attention, one cluster per head */
+#define ASR_PROF_QUERY_CROSS 10  /* few rows: LayerNorm + cross query + cross-attention, one cluster per head */
+#define ASR_PROF_N 11
 int asr_spec_set_graphs(asr_spec_handle h, int enable);
 int asr_spec_profile(asr_spec_handle h, int enable);
 int asr_spec_profile_read(asr_spec_handle h, double* ms, int64_t* launches, uint64_t* traffic);
@@ -254,29 +255,27 @@ int asr_spec_profile_read(asr_spec_handle h, double* ms, int64_t* launches, uint
 #define ASR_TL_ATTN_SELF 4     /* self-attention */
 #define ASR_TL_ATTN_CROSS 5    /* cross-attention */
 #define ASR_TL_ACCEPT 6        /* acceptance, commit and anchor readout */
-#define ASR_TL_FUSED 7         /* fused verify of a step with few rows (layers + LM head; midpoint: LM head start) */
+#define ASR_TL_QKV_SELF 8      /* few rows: LayerNorm + QKV + self-attention, one cluster per head */
+#define ASR_TL_QUERY_CROSS 9   /* few rows: LayerNorm + cross query + cross-attention, one cluster per head */
 #define ASR_TL_GEMM 16         /* + epilogue: 0 plain, 1 QKV + cache append, 2 residual, 3 query, 4 GELU, 6 argmax */
 #define ASR_TL_LN_FUSED 32     /* added to a GEMM kind whose input LayerNorm is folded into it (no LayerNorm launch) */
 int asr_spec_timeline(asr_spec_handle h, int32_t enable);
 int asr_spec_timeline_read(asr_spec_handle h, uint64_t* ns, int32_t* kind, int32_t cap, int32_t* count);
 
-/* Diagnostics of the fused few-row verify (one persistent kernel for the
- * layers and the LM head of a step with batch x (k + 1) <= 9 rows, bf16 models
- * with d_model in {512, 768, 1024, 1280}; ASRSPEC_FUSED=1 in the environment
- * at create turns it on, it is off by default).
- *
- * asr_spec_fused_trace: when enabled, every fused verify records, per CTA,
- * the GPU global timer (ns) at 16 points per layer (layer start, then the end
- * of each stage and of the grid barrier after it: QKV, barrier, self-attention,
- * barrier, self out, barrier, cross query, barrier, cross-attention, barrier,
- * cross out, barrier, MLP up, barrier, MLP down) and at the LM head's start
- * and end; verify then launches directly (no graph).  ASR_E_INVAL when the
- * model has no fused path.
- * asr_spec_fused_trace_read: synchronise and copy the last traced call's
- * stamps, [n_cta][per_cta] words, up to `cap` words; per_cta = 16 L + 2;
- * n_cta = 0 before the first enable. */
-int asr_spec_fused_trace(asr_spec_handle h, int32_t enable);
-int asr_spec_fused_trace_read(asr_spec_handle h, uint64_t* out, int64_t cap, int32_t* per_cta, int32_t* n_cta);
+
+/* ---- Diagnostics of the few-row layers (not part of the paper's method) ---
+ * asr_spec_fewrow_trace: when enabled, every verify that runs the few-row
+ * layers (bf16 models, batch x (k + 1) <= 9 rows) records, per CTA of each of
+ * its 6 L layer launches, the GPU global timer (ns) at 12 phases: entry, past
+ * the wait on the previous launch, input rows ready, weights landed,
+ * projection reduced, exchange landed, attention done, exit, first K/V chunk
+ * landed, first chunk combined, merge inputs landed, (unused) (0 where a
+ * launch has no such phase); verify then launches directly (no graph).
+ * ASR_E_INVAL when the model has no few-row layers.
+ * asr_spec_fewrow_trace_read: synchronise and copy the last traced call's
+ * stamps, [n_launches][320 CTAs][12] words in launch order, up to `cap` words. */
+int asr_spec_fewrow_trace(asr_spec_handle h, int32_t enable);
+int asr_spec_fewrow_trace_read(asr_spec_handle h, uint64_t* out, int64_t cap, int32_t* n_launches);
 
 /* ---- Workload utility (not part of the paper's method) -------------------
  * Synthetic draft source used by benchmarks in place of a trained draft

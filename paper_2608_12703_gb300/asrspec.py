@@ -28,15 +28,15 @@ EXPORTED = [
     "asr_spec_status", "asr_spec_last_error", "asr_spec_destroy", "asr_spec_synth_drafts",
     "asr_spec_test_gemm", "asr_spec_set_graphs", "asr_spec_profile", "asr_spec_profile_read",
     "asr_spec_gemm_noalloc", "asr_spec_timeline", "asr_spec_timeline_read",
-    "asr_spec_fused_trace", "asr_spec_fused_trace_read", "asr_spec_verify_tree", "asr_spec_restart",
+    "asr_spec_verify_tree", "asr_spec_restart", "asr_spec_fewrow_trace", "asr_spec_fewrow_trace_read",
     "asr_spec_debug_anchor_profile",
 ]
 PROF_CLASSES = ["qkv", "resid", "query", "mlp_up", "self_attn", "cross_attn", "lm_head", "layernorm", "other",
-                "fused"]
+                "qkv_self", "query_cross"]
 TL_CAP = 65536
 TL_GEMM, TL_LN_FUSED = 16, 32
 TL_KINDS = {0: "other", 1: "plan", 2: "embed", 3: "layernorm", 4: "attn_self", 5: "attn_cross", 6: "accept_anchor",
-            7: "fused_verify"}
+            8: "qkv_self", 9: "query_cross"}
 TL_GEMM_EPILOGUES = {0: "plain", 1: "qkv", 2: "residual", 3: "query", 4: "gelu", 5: "cross_kv", 6: "argmax"}
 
 
@@ -83,6 +83,8 @@ def lib():
     L.asr_spec_verify_tree.argtypes = [vp, p32, p32, p32, i32, p32, p32, p32, p32, p32]
     L.asr_spec_rollback.argtypes = [vp, p32, p32]
     L.asr_spec_restart.argtypes = [vp, p32]
+    L.asr_spec_fewrow_trace.argtypes = [vp, i32]
+    L.asr_spec_fewrow_trace_read.argtypes = [vp, vp, ctypes.c_int64, vp]
     L.asr_spec_debug_anchor_profile.argtypes = [vp, vp]
     L.asr_spec_state.argtypes = [vp, p32, p32]
     L.asr_spec_debug_logits.argtypes = [vp, vp, i32]
@@ -99,8 +101,6 @@ def lib():
     L.asr_spec_gemm_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp]
     L.asr_spec_timeline.argtypes = [vp, i32]
     L.asr_spec_timeline_read.argtypes = [vp, vp, vp, i32, vp]
-    L.asr_spec_fused_trace.argtypes = [vp, i32]
-    L.asr_spec_fused_trace_read.argtypes = [vp, vp, ctypes.c_int64, vp, vp]
     for name in EXPORTED:
         if name not in ("asr_spec_last_error", "asr_spec_destroy"):
             getattr(L, name).restype = ctypes.c_int
@@ -237,18 +237,23 @@ def asr_spec_timeline_read(h):
     return ns[:n].copy(), kinds[:n].copy()
 
 
-def asr_spec_fused_trace(h, enable: bool):
-    return _check(h, lib().asr_spec_fused_trace(h, 1 if enable else 0), "asr_spec_fused_trace")
+FR_TRACE_CTAS, FR_TRACE_PHASES = 320, 12
 
 
-def asr_spec_fused_trace_read(h):
-    """Per-CTA stage timestamps (ns) of the last traced fused verify, [n_cta][16 L + 2]."""
-    per, n = ctypes.c_int32(0), ctypes.c_int32(0)
-    _check(h, lib().asr_spec_fused_trace_read(h, None, 0, ctypes.byref(per), ctypes.byref(n)),
-           "asr_spec_fused_trace_read")
-    out = np.zeros((n.value, per.value), dtype=np.uint64)
-    _check(h, lib().asr_spec_fused_trace_read(h, out.ctypes.data, out.size, ctypes.byref(per), ctypes.byref(n)),
-           "asr_spec_fused_trace_read")
+def asr_spec_fewrow_trace(h, enable: bool):
+    return _check(h, lib().asr_spec_fewrow_trace(h, 1 if enable else 0), "asr_spec_fewrow_trace")
+
+
+def asr_spec_fewrow_trace_read(h):
+    """Per-CTA phase stamps (ns) of the last traced call's few-row launches,
+    [n_launches][320][12] (entry, past wait, rows ready, weights landed,
+    reduced, exchange landed, attention done, exit, first K/V chunk landed,
+    first chunk combined, merge inputs landed; 0 = none)."""
+    n = ctypes.c_int32(0)
+    _check(h, lib().asr_spec_fewrow_trace_read(h, None, 0, ctypes.byref(n)), "asr_spec_fewrow_trace_read")
+    out = np.zeros((n.value, FR_TRACE_CTAS, FR_TRACE_PHASES), dtype=np.uint64)
+    _check(h, lib().asr_spec_fewrow_trace_read(h, out.ctypes.data, out.size, ctypes.byref(n)),
+           "asr_spec_fewrow_trace_read")
     return out
 
 

@@ -24,6 +24,8 @@ struct LayerW {
   // whose input is a LayerNorm output
   float *c1_qkv = nullptr, *c2_qkv = nullptr, *c1_cq = nullptr, *c2_cq = nullptr, *c1_fc1 = nullptr, *c2_fc1 = nullptr;
   CUtensorMap m_wqkv, m_wo, m_wcq, m_wco, m_w1, m_w2;
+  // the same weights packed for the few-row kernels (launch_fr_pack), or null
+  void *p_qkv = nullptr, *p_wo = nullptr, *p_wcq = nullptr, *p_wco = nullptr, *p_w1 = nullptr, *p_w2 = nullptr;
 };
 
 }  // namespace
@@ -88,24 +90,23 @@ struct asr_spec {
   bool ln_fold = false;
   float2* ln_part = nullptr;
   int ln_S = 0, ln_c = 0;
-  // fused verify for steps of at most VF_ROWS rows (ASRSPEC_FUSED=1 turns it
-  // on; off by default: 2.04 against 1.84 ms per batch-1 round of the large
-  // decoder, as measured): the grid (one CTA per SM, 0 = unavailable), the
-  // layer table, the grid barrier counter, the split-merge tickets and
-  // partials of its attention
-  bool use_fused = false;
-  int vf_G = 0, vf_bmax = 0;
-  VfLayer* vf_layers = nullptr;
-  unsigned* vf_bar = nullptr;
-  int* vf_tickets = nullptr;
-  float* vf_part = nullptr;
-  bool last_fused = false;    // the last verify ran the fused kernel (LM-head input in xf)
+  // few-row verify layers (csrc/fewrow.cu) for steps of at most VF_ROWS rows:
+  // the cluster size per head (0 = unavailable for this model or device);
+  // ASRSPEC_FEWROW=0 keeps the tensor-core chain for every step
+  bool use_fewrow = true;
+  int fr_C = 0;
+  int fr_sms = 0;   // SMs of the device: the GEMVs run one CTA (group) per SM
+  int fr_gd = 0;    // groups of the MLP down-projection (clusters resident at once)
+  bool last_fused = false;    // the last verify ran the few-row layers (LM-head input in xf)
+  // per-CTA phase stamps of the few-row launches of the last traced call
+  // (diagnostics): [6 L][FR_TRACE_CTAS][FR_TRACE_PHASES]
+  unsigned long long* fr_trace = nullptr;
+  bool fr_trace_on = false;
+  int fr_trace_n = 0;
   // tree verify: the nodes' parents and the accepted path ([B_max][max_draft]),
   // and whether the step being enqueued is one
   int *parent_buf = nullptr, *path_buf = nullptr;
   bool cur_tree = false;
-  unsigned long long* vf_trace = nullptr;   // per-stage timestamps of the fused kernel (diagnostics)
-  bool vf_trace_on = false;
   int wide_bn = 64;      // N tile for many rows (ASRSPEC_WIDE_BN: 64, 128, 192, 224, 256)
   int wide_target = 2 * 152;   // CTAs a many-row GEMM may fill by splitting K (ASRSPEC_WIDE_TARGET)
   int few_target = 2 * 152;    // the same for few rows (ASRSPEC_FEW_TARGET)
@@ -124,7 +125,7 @@ struct asr_spec {
     cudaGraphExec_t exec;
     long long launches[ASR_PROF_N];
     int ln_S, ln_c;   // the folded LayerNorm slices the captured body leaves (for debug_logits)
-    bool fused;       // the body is the fused verify kernel
+    bool fused;       // the body runs the few-row layers
   };
   std::map<std::pair<int, int>, Graph> graphs;
 };
@@ -475,6 +476,144 @@ int run_layers(asr_spec* h, int N) {
   return 0;
 }
 
+// The decoder layers of a step with at most VF_ROWS rows (csrc/fewrow.cu):
+// six launches per layer.
+int run_layers_few(asr_spec* h) {
+  const int d = h->d, F = h->F, H = h->H, C = h->fr_C, N = h->B * (h->kmax + 1);
+  const int nt_o = d / 8, nt_f = F / 8, KS = F / d;
+  const int g_o = std::min(nt_o, h->fr_sms), g_f = std::min(nt_f, h->fr_sms), g_d = h->fr_gd;
+  const size_t self_layer = (size_t)h->Bmax * H * h->maxpos * 64;
+  {
+    Prof p(h, ASR_PROF_OTHER, 1);
+    Tl t(h, ASR_TL_EMBED);
+    launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, std::min(N, VF_ROWS), d, h->x, h->st, h->use_pdl, h->tl_cur);
+  }
+  auto bf = [](void* p) { return static_cast<const __nv_bfloat16*>(p); };
+  h->fr_trace_n = 0;
+  auto trace_slot = [&]() -> unsigned long long* {
+    if (!h->fr_trace_on) return nullptr;
+    return h->fr_trace + (size_t)(h->fr_trace_n++) * FR_TRACE_CTAS * FR_TRACE_PHASES;
+  };
+  for (int l = 0; l < h->L; ++l) {
+    LayerW& w = h->lw[l];
+    FrHead hd{};
+    hd.x = h->x;
+    hd.d = d;
+    hd.H = H;
+    hd.C = C;
+    hd.B = h->B;
+    hd.max_pos = h->maxpos;
+    hd.plan = h->plan;
+    hd.kv_len = h->kv_len;
+    hd.enc_len = h->enc_len;
+    hd.att = static_cast<__nv_bfloat16*>(h->att);
+    hd.status = h->status;
+    // LayerNorm 1 -> QKV -> self-attention
+    FrHead hs = hd;
+    hs.W = bf(w.p_qkv);
+    hs.bias = w.bqkv;
+    hs.ln_g = w.ln1g;
+    hs.ln_b = w.ln1b;
+    hs.tiles_max = (24 + C - 1) / C;
+    hs.mrg_slots = (h->maxpos + 127) / 128;
+    hs.ks = static_cast<__nv_bfloat16*>(h->kself) + l * self_layer;
+    hs.vs = static_cast<__nv_bfloat16*>(h->vself) + l * self_layer;
+    hs.row0 = (long long)l * h->Bmax * H * h->maxpos;
+    hs.t_alloc = h->maxpos;
+    {
+      Prof p(h, ASR_PROF_QKV_SELF, 1);
+      Tl t(h, ASR_TL_QKV_SELF);
+      hs.tl = h->tl_cur;
+      hs.trace = trace_slot();
+      CK(launch_fr_self(&h->m_kself[0], &h->m_vself[0], hs, h->st, h->use_pdl));
+    }
+    FrGemv g{};
+    g.n_rows = h->plan.n_rows;
+    g.status = h->status;
+    g.x = h->x;
+    g.x_out = h->x;
+    // self-attention output projection + residual
+    FrGemv go = g;
+    go.W = bf(w.p_wo);
+    go.bias = w.bo;
+    go.N = d;
+    go.K = d;
+    go.tiles_max = (nt_o + g_o - 1) / g_o;
+    go.a = static_cast<const __nv_bfloat16*>(h->att);
+    {
+      Prof p(h, ASR_PROF_RESID, 1);
+      Tl t(h, ASR_TL_GEMM + EPI_RESID);
+      go.tl = h->tl_cur;
+      go.trace = trace_slot();
+      CK(launch_fr_gemv(go, FR_RESID, 1, g_o, d, h->st, h->use_pdl));
+    }
+    // LayerNorm 2 -> cross query -> cross-attention
+    FrHead hc = hd;
+    hc.W = bf(w.p_wcq);
+    hc.bias = w.bcq;
+    hc.ln_g = w.ln2g;
+    hc.ln_b = w.ln2b;
+    hc.tiles_max = (8 + C - 1) / C;
+    hc.mrg_slots = C;
+    hc.row0 = (long long)l * 2 * h->Bmax * H * h->Tmax;
+    hc.vofs = (long long)h->Bmax * H * h->Tmax;
+    hc.t_alloc = h->Tmax;
+    hc.q_anchor = l == h->anchor ? h->q_anchor : nullptr;
+    hc.ml = l == h->anchor ? h->ml : nullptr;
+    {
+      Prof p(h, ASR_PROF_QUERY_CROSS, 1);
+      Tl t(h, ASR_TL_QUERY_CROSS);
+      hc.tl = h->tl_cur;
+      hc.trace = trace_slot();
+      CK(launch_fr_cross(&h->m_xkv[0], hc, h->st, h->use_pdl));
+    }
+    // cross-attention output projection + residual
+    FrGemv gc = go;
+    gc.W = bf(w.p_wco);
+    gc.bias = w.bco;
+    {
+      Prof p(h, ASR_PROF_RESID, 1);
+      Tl t(h, ASR_TL_GEMM + EPI_RESID);
+      gc.tl = h->tl_cur;
+      gc.trace = trace_slot();
+      CK(launch_fr_gemv(gc, FR_RESID, 1, g_o, d, h->st, h->use_pdl));
+    }
+    // LayerNorm 3 -> MLP up + GELU
+    FrGemv gu = g;
+    gu.W = bf(w.p_w1);
+    gu.bias = w.b1;
+    gu.N = F;
+    gu.K = d;
+    gu.tiles_max = (nt_f + g_f - 1) / g_f;
+    gu.ln_g = w.ln3g;
+    gu.ln_b = w.ln3b;
+    gu.h_out = static_cast<__nv_bfloat16*>(h->hbuf);
+    {
+      Prof p(h, ASR_PROF_UP, 1);
+      Tl t(h, ASR_TL_GEMM + EPI_GELU);
+      gu.tl = h->tl_cur;
+      gu.trace = trace_slot();
+      CK(launch_fr_gemv(gu, FR_GELU, 1, g_f, d, h->st, h->use_pdl));
+    }
+    // MLP down + residual (K split over a cluster of F / d CTAs)
+    FrGemv gd = g;
+    gd.W = bf(w.p_w2);
+    gd.bias = w.b2;
+    gd.N = d;
+    gd.K = F;
+    gd.tiles_max = (nt_o + g_d - 1) / g_d;
+    gd.a = static_cast<const __nv_bfloat16*>(h->hbuf);
+    {
+      Prof p(h, ASR_PROF_RESID, 1);
+      Tl t(h, ASR_TL_GEMM + EPI_RESID);
+      gd.tl = h->tl_cur;
+      gd.trace = trace_slot();
+      CK(launch_fr_gemv(gd, FR_RESID, KS, g_d, d, h->st, h->use_pdl));
+    }
+  }
+  return 0;
+}
+
 bool dims_ok(const asr_model_dims& m) {
   return m.n_layers >= 1 && m.d_model >= 64 && m.d_model % 64 == 0 && m.d_model <= 2048 &&
          m.n_heads * 64 == m.d_model && m.d_ffn >= 64 && m.d_ffn % 64 == 0 && m.vocab >= 2 && m.max_pos >= 2 &&
@@ -504,48 +643,20 @@ int enqueue_verify(asr_spec* h, int k) {
                        h->row_key, h->status, tr, h->st, h->tl_cur, h->cur_tree ? h->parent_buf : nullptr);
   }
   const int N = B * (k + 1);
-  h->last_fused = h->vf_G > 0 && N <= VF_ROWS && B <= h->vf_bmax && !h->cur_tree;
-  if (h->last_fused) {   // few rows: one persistent kernel for the layers and the LM head
-    CK(cudaMemsetAsync(h->vf_bar, 0, 4, h->st));
-    VfArgs a{};
-    a.layers = h->vf_layers;
-    a.L = h->L;
-    a.d = h->d;
-    a.H = h->H;
-    a.F = h->F;
-    a.V = h->V;
-    a.max_pos = h->maxpos;
-    a.t_alloc = h->Tmax;
-    a.b_max = h->Bmax;
-    a.anchor = h->anchor;
-    a.B = B;
-    a.S = std::max(1, std::min(16, h->vf_G / (B * h->H)));
-    int total = 0;
-    vf_layout(h->d, h->F, h->L, &a.a_bytes, &a.slot_bytes, &total);
-    a.tok_emb = static_cast<const __nv_bfloat16*>(h->w_tok);
-    a.pos_emb = static_cast<const __nv_bfloat16*>(h->w_pos);
-    a.lnf_g = h->lnf_g;
-    a.lnf_b = h->lnf_b;
-    a.plan = h->plan;
-    a.kv_len = h->kv_len;
-    a.enc_len = h->enc_len;
-    a.x = h->x;
-    a.q = h->q;
-    a.q_anchor = h->q_anchor;
-    a.ml = h->ml;
-    a.part = h->vf_part;
-    a.att = static_cast<__nv_bfloat16*>(h->att);
-    a.hbuf = static_cast<__nv_bfloat16*>(h->hbuf);
-    a.xf = static_cast<__nv_bfloat16*>(h->xf);
-    a.row_key = h->row_key;
-    a.bar_ctr = h->vf_bar;
-    a.tickets = h->vf_tickets;
-    a.status = h->status;
-    a.trace = h->vf_trace_on ? h->vf_trace : nullptr;
-    Prof p(h, ASR_PROF_FUSED, 1);
-    Tl t(h, ASR_TL_FUSED);
-    a.tl = h->tl_cur;
-    CK(launch_verify_fused(&h->m_xkv[0], a, h->vf_G, h->st));
+  h->last_fused = h->fr_C > 0 && h->use_fewrow && N <= VF_ROWS && B <= VF_ROWS && !h->cur_tree;
+  if (h->last_fused) {   // few rows: six launches per layer, then LayerNorm + LM head
+    if (int rc = run_layers_few(h)) return rc;
+    {
+      Prof p(h, ASR_PROF_LAYERNORM, 1);
+      Tl t(h, ASR_TL_LAYERNORM);
+      launch_layernorm(h->x, h->lnf_g, h->lnf_b, h->xf, h->bf16, h->plan.n_rows, N, h->d, h->st, h->use_pdl,
+                       h->tl_cur);
+    }
+    Epi e{};
+    e.n_valid = h->plan.n_rows;
+    e.row_key = h->row_key;
+    e.d = h->d;
+    if (int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, h->d, h->xf, BUF_XF, N, EPI_ARGMAX, e)) return rc;
   } else {
     if (int rc = run_layers(h, N)) return rc;
     Epi e{};
@@ -849,31 +960,28 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   }
   if ((rc = dalloc(h, &h->counters, 8 * sizeof(unsigned long long)))) return finish(rc);
   CK(cudaMemset(h->counters, 0, 8 * sizeof(unsigned long long)));
-  if (const char* e = std::getenv("ASRSPEC_FUSED")) h->use_fused = std::atoi(e) != 0;
-  if (h->bf16 && h->use_fused && (h->vf_G = vf_grid(d, F, L)) > 0) {
-    std::vector<VfLayer> t(L);
-    for (int l = 0; l < L; ++l) {
-      const LayerW& w = h->lw[l];
-      VfLayer& v = t[l];
-      v.wqkv = static_cast<const __nv_bfloat16*>(w.wqkv);
-      v.wo = static_cast<const __nv_bfloat16*>(w.wo);
-      v.wcq = static_cast<const __nv_bfloat16*>(w.wcq);
-      v.wco = static_cast<const __nv_bfloat16*>(w.wco);
-      v.w1 = static_cast<const __nv_bfloat16*>(w.w1);
-      v.w2 = static_cast<const __nv_bfloat16*>(w.w2);
-      v.bqkv = w.bqkv; v.bo = w.bo; v.bcq = w.bcq; v.bco = w.bco; v.b1 = w.b1; v.b2 = w.b2;
-      v.ln1g = w.ln1g; v.ln1b = w.ln1b; v.ln2g = w.ln2g; v.ln2b = w.ln2b; v.ln3g = w.ln3g; v.ln3b = w.ln3b;
-      const size_t self_layer = (size_t)h->Bmax * h->H * h->maxpos * 64;
-      v.ks = static_cast<__nv_bfloat16*>(h->kself) + l * self_layer;
-      v.vs = static_cast<__nv_bfloat16*>(h->vself) + l * self_layer;
+  if (const char* e = std::getenv("ASRSPEC_FEWROW")) h->use_fewrow = std::atoi(e) != 0;
+  if (h->bf16) {
+    int C = 0;
+    int n_sm = 0, gd = 0;
+    if (fr_configure(d, F, h->H, h->maxpos, &C, &n_sm, &gd)) {
+      h->fr_C = C;
+      h->fr_sms = n_sm;
+      h->fr_gd = gd;
+      for (int l = 0; l < L; ++l) {   // packed copies of the layer weights
+        LayerW& w = h->lw[l];
+        struct {
+          void* src;
+          void** dst;
+          int N, K;
+        } mats[6] = {{w.wqkv, &w.p_qkv, 3 * d, d}, {w.wo, &w.p_wo, d, d},  {w.wcq, &w.p_wcq, d, d},
+                     {w.wco, &w.p_wco, d, d},     {w.w1, &w.p_w1, F, d},   {w.w2, &w.p_w2, d, F}};
+        for (auto& m : mats) {
+          if ((rc = dalloc(h, m.dst, (size_t)m.N * m.K * 2))) return finish(rc);
+          CK(launch_fr_pack(m.src, *m.dst, m.N, m.K, h->st));
+        }
+      }
     }
-    h->vf_bmax = std::min(h->Bmax, VF_ROWS);
-    const size_t part = (size_t)h->vf_bmax * h->H * 16 * VF_ROWS * 66;
-    if ((rc = dalloc(h, &h->vf_layers, L * sizeof(VfLayer))) || (rc = dalloc(h, &h->vf_bar, 4)) ||
-        (rc = dalloc(h, &h->vf_tickets, (size_t)h->vf_bmax * h->H * 4)) || (rc = dalloc(h, &h->vf_part, part * 4)))
-      return finish(rc);
-    CK(cudaMemcpy(h->vf_layers, t.data(), L * sizeof(VfLayer), cudaMemcpyHostToDevice));
-    CK(cudaMemset(h->vf_tickets, 0, (size_t)h->vf_bmax * h->H * 4));
   }
   configure_gemm_tc();
   configure_attention();
@@ -980,7 +1088,7 @@ int verify_call(asr_spec* h, const int32_t* draft, const int32_t* parent, const 
     ~TreeScope() { h->cur_tree = false; }
   } scope{h};
   h->cur_tree = tree;
-  if (h->use_graphs && !h->prof && !h->tl_on && !h->vf_trace_on) {
+  if (h->use_graphs && !h->prof && !h->tl_on && !h->fr_trace_on) {
     auto key = std::make_pair(B, tree ? 1000 + (int)k : (int)k);
     auto it = h->graphs.find(key);
     if (it == h->graphs.end()) {
@@ -1136,26 +1244,25 @@ int asr_spec_timeline_read(asr_spec_handle h, uint64_t* ns, int32_t* kind, int32
   return ASR_OK;
 }
 
-int asr_spec_fused_trace(asr_spec_handle h, int32_t enable) {
+int asr_spec_fewrow_trace(asr_spec_handle h, int32_t enable) {
   if (!h) return ASR_E_INVAL;
-  if (enable && h->vf_G == 0) return fail(h, ASR_E_INVAL, "the fused verify is not available for this model");
-  if (enable && !h->vf_trace) {
-    const size_t n = (size_t)h->vf_G * vf_trace_points(h->L);
-    int rc = dalloc(h, &h->vf_trace, n * sizeof(unsigned long long));
+  if (enable && h->fr_C == 0) return fail(h, ASR_E_INVAL, "the few-row layers are not available for this model");
+  if (enable && !h->fr_trace) {
+    const size_t n = (size_t)6 * h->L * FR_TRACE_CTAS * FR_TRACE_PHASES;
+    int rc = dalloc(h, &h->fr_trace, n * sizeof(unsigned long long));
     if (rc) return rc;
-    CK(cudaMemset(h->vf_trace, 0, n * sizeof(unsigned long long)));
+    CK(cudaMemset(h->fr_trace, 0, n * sizeof(unsigned long long)));
   }
-  h->vf_trace_on = enable != 0;
+  h->fr_trace_on = enable != 0;
   return ASR_OK;
 }
 
-int asr_spec_fused_trace_read(asr_spec_handle h, uint64_t* out, int64_t cap, int32_t* per_cta, int32_t* n_cta) {
-  if (!h || !per_cta || !n_cta || cap < 0 || (cap > 0 && !out)) return ASR_E_INVAL;
-  *per_cta = vf_trace_points(h->L);
-  *n_cta = h->vf_trace ? h->vf_G : 0;
-  const size_t n = std::min((size_t)cap, (size_t)(*n_cta) * (size_t)(*per_cta));
+int asr_spec_fewrow_trace_read(asr_spec_handle h, uint64_t* out, int64_t cap, int32_t* n_launches) {
+  if (!h || !n_launches || cap < 0 || (cap > 0 && !out)) return ASR_E_INVAL;
+  *n_launches = h->fr_trace ? h->fr_trace_n : 0;
+  const size_t n = std::min((size_t)cap, (size_t)(*n_launches) * FR_TRACE_CTAS * FR_TRACE_PHASES);
   CK(cudaStreamSynchronize(h->st));
-  if (n > 0) CK(cudaMemcpy(out, h->vf_trace, n * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
+  if (n > 0) CK(cudaMemcpy(out, h->fr_trace, n * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
   return ASR_OK;
 }
 

@@ -147,49 +147,72 @@ void launch_accept_anchor(const AcceptAnchorArgs& a, cudaStream_t st);
 void launch_tree_commit(const int* path, int k, const int* accepted, const int* kv_len, int B, int L, int H,
                         int max_pos, int b_max, void* kself, void* vself, int es, cudaStream_t st);
 
-// ---- Fused verify for few rows ----------------------------------------------------
-// One persistent cooperative kernel (one CTA per SM) runs the decoder layers and
-// the LM head of a verify step whose rows all fit one 16-row MMA tile
-// (VF_ROWS): the stages are separated by grid-wide barriers, and a producer
-// warp streams every projection's weight slice through a shared-memory ring
-// independently of them, so the next stage's weights load while the current
-// stage waits.  Writes what the multi-kernel chain writes (residual, caches,
-// q_anchor, ml, argmax keys); the accept + anchor kernel follows it.
+// ---- Few-row verify layers (csrc/fewrow.cu) ------------------------------------
+// A step of at most VF_ROWS rows runs each decoder layer as six launches:
+// LayerNorm + QKV + self-attention (one cluster per head), output projection,
+// LayerNorm + cross query + cross-attention (one cluster per head), output
+// projection, LayerNorm + MLP up, MLP down; the projections as GEMVs over
+// 8-feature tiles (no split-K exchange).
 constexpr int VF_ROWS = 9;
-struct VfLayer {
-  const __nv_bfloat16 *wqkv, *wo, *wcq, *wco, *w1, *w2;
-  const float *bqkv, *bo, *bcq, *bco, *b1, *b2;
-  const float *ln1g, *ln1b, *ln2g, *ln2b, *ln3g, *ln3b;
-  __nv_bfloat16 *ks, *vs;   // this layer's self K/V cache [B_max][H][max_pos][64]
+enum FrMode : int { FR_RESID = 0, FR_GELU = 1 };
+struct FrGemv {
+  const __nv_bfloat16* W;   // [N][K] weights
+  const float* bias;        // [N]
+  int N, K;                 // outputs, inputs
+  int tiles_max;            // 8-feature tiles per CTA, at most (<= 5): ceil(N / 8 / groups)
+  const float* x;           // FR_GELU: the residual stream [R][K] (LayerNorm input)
+  const float *ln_g, *ln_b;
+  const __nv_bfloat16* a;   // FR_RESID: bf16 input rows [R][K]
+  float* x_out;             // FR_RESID: x[r][m] += y + bias  ([R][N])
+  __nv_bfloat16* h_out;     // FR_GELU: bf16(gelu(y + bias))  ([R][N])
+  const int* n_rows;
+  int* status;
+  unsigned long long* tl;
+  unsigned long long* trace;   // per-CTA phase stamps [CTA][FR_TRACE_PHASES] (diagnostics), or null
 };
-struct VfArgs {
-  const VfLayer* layers;    // [L], device memory
-  int L, d, H, F, V, max_pos, t_alloc, b_max, anchor, B;
-  int S;                    // cross-attention splits per (utterance, head)
-  int a_bytes, slot_bytes;  // shared-memory layout (vf_layout)
-  const __nv_bfloat16 *tok_emb, *pos_emb;
-  const float *lnf_g, *lnf_b;
+struct FrHead {
+  const __nv_bfloat16* W;   // self: fused QKV weights [3d][d]; cross: query weights [d][d]
+  const float* bias;
+  const float *x, *ln_g, *ln_b;   // the residual stream and the LayerNorm in front of W
+  int d, H, C, B, max_pos;
+  int tiles_max;            // weight tiles per CTA, at most
+  int mrg_slots;            // partials a merging CTA can hold per row
   RowPlan plan;
   const int* kv_len;
   const int* enc_len;
-  float *x, *q, *q_anchor, *ml, *part;
-  __nv_bfloat16 *att, *hbuf, *xf;
-  unsigned long long* row_key;
-  unsigned* bar_ctr;        // grid barrier counter, zeroed before the launch
-  int* tickets;             // [B_max * H] split merge tickets, zero between uses
+  __nv_bfloat16 *ks, *vs;   // self: this layer's caches [B_max][H][max_pos][64] (new rows appended)
+  long long row0;           // tensor-map row of this layer's (utterance 0, head 0, key 0)
+  long long vofs;           // cross: rows from the K half to the V half of the encoder cache
+  int t_alloc;              // tensor-map rows per (utterance, head)
+  __nv_bfloat16* att;       // [R][d] attention output
+  float* q_anchor;          // cross at the anchor layer: fp32 queries [R][d], else null
+  float* ml;                // cross at the anchor layer: softmax (max, sum) [R][H][2], else null
   int* status;
   unsigned long long* tl;
-  unsigned long long* trace;   // per-stage timestamps [CTA][vf_trace_points(L)], or null
+  unsigned long long* trace;   // per-CTA phase stamps [CTA][FR_TRACE_PHASES] (diagnostics), or null
 };
-// Timestamps per CTA of a traced fused verify: 16 per layer (layer start, then
-// the end of each stage and of each grid barrier that follows it) + 2 (LM head
-// start and end).
-__host__ __device__ inline int vf_trace_points(int L) { return 16 * L + 2; }
-// Shared-memory layout for (d, F, L): activation/attention region, ring slot, total bytes.
-void vf_layout(int d, int F, int L, int* a_bytes, int* slot_bytes, int* total);
-// 0 when the kernel cannot run for these dimensions on this device.
-int vf_grid(int d, int F, int L);
-cudaError_t launch_verify_fused(const CUtensorMap* xmap, const VfArgs& a, int grid, cudaStream_t st);
+// Phase stamps of a traced few-row launch, GPU global timer (ns), thread 0 of
+// each CTA: 0 entry, 1 past the wait on the previous launch, 2 input rows
+// ready, 3 weights landed, 4 projection reduced, 5 exchange landed (head:
+// gathered q/k/v; K-split group: the other ranks' partials), 6 attention
+// done (head), 7 exit; head kernels also 8 first K/V chunk landed, 9 first
+// chunk's attention combined, 10 merge inputs landed.  Up to FR_TRACE_CTAS
+// CTAs per launch.
+constexpr int FR_TRACE_PHASES = 12;
+constexpr int FR_TRACE_CTAS = 320;
+// 1 and the cluster size per head when the kernels run for these dimensions on this device
+// (gd_out: the MLP down-projection's groups of F / d CTAs)
+int fr_configure(int d, int F, int H, int max_pos, int* C_out, int* sms_out, int* gd_out);
+size_t fr_gemv_smem(int d, int K, int tiles_max, int ks, int mode);
+size_t fr_head_smem(int d, int tiles_max, bool self_attn, int mrg_slots);
+// groups: CTA groups of ks (one cluster each); a.tiles_max = ceil(N / 8 / groups)
+// Pack a bf16 [N][K] weight matrix (N, K multiples of 8) into the few-row
+// kernels' tile layout: 8-row tiles, contiguous, 16-byte pieces piece-major.
+cudaError_t launch_fr_pack(const void* src, void* dst, int N, int K, cudaStream_t st);
+cudaError_t launch_fr_gemv(const FrGemv& a, int mode, int ks, int groups, int d, cudaStream_t st, bool pdl);
+cudaError_t launch_fr_self(const CUtensorMap* kmap, const CUtensorMap* vmap, const FrHead& a, cudaStream_t st,
+                           bool pdl);
+cudaError_t launch_fr_cross(const CUtensorMap* xmap, const FrHead& a, cudaStream_t st, bool pdl);
 
 // ---- Accept / commit ------------------------------------------------------------
 void launch_prefill_advance(int B, int c, const int* n_utt_rows, int* kv_len, cudaStream_t st);

@@ -8,12 +8,14 @@ CUDA events on the library's stream.
   python -m paper_2608_12703_gb300.profile_run --config large-bf16-b1-k8 --warmup 2 --rounds 3
 
 Options: --classes (CUDA-event time per kernel class), --timeline (the launch
-timeline per launch kind), --fused-trace (per-stage stamps of the opt-in fused
-verify), --tree-nodes N (tree verifies beside the linear one), --enc-len T
+timeline per launch kind), --fewrow-trace (per-CTA phase stamps of the
+few-row launches), --tree-nodes N (tree verifies beside the linear one), --enc-len T
 (encoder memories of T frames), --batch-sweep 1,4,16,64 (verification cost and
 anchor-readout share against batch size).
 
-Kernel launches per round (bf16 decoders, LayerNorm folded): 2 + 8 per layer + 2.
+Kernel launches per round (bf16 decoders): at most 9 rows (e.g. batch 1):
+2 + 6 per layer + 3 (few-row layers, final LayerNorm, LM head, accept);
+more rows: 2 + 8 per layer + 2 (tensor-core chain, LayerNorm folded).
 """
 from __future__ import annotations
 
@@ -62,34 +64,37 @@ def timeline_summary(ns, kinds, rounds):
     return "\n".join(lines)
 
 
-FUSED_INTERVALS = ["qkv", "barrier", "self_attn", "barrier", "self_out", "barrier", "cross_q", "barrier",
-                   "cross_attn", "barrier", "cross_out", "barrier", "mlp_up", "barrier", "mlp_down", "barrier"]
+FEWROW_KINDS = ["qkv_self", "self_out", "query_cross", "cross_out", "mlp_up", "mlp_down"]
+FEWROW_PHASES = ["entry", "past_wait", "rows", "weights", "reduced", "exchange", "attention", "exit", "kv_in",
+                 "combined", "merge_in"]
 
 
-def fused_trace_summary(tr):
-    """Per interval of a layer of the fused verify (trace [CTA][16 L + 2]):
-    the per-CTA duration (median and max over CTAs, mean over layers) and the
-    advance of the last CTA (max over CTAs of the end stamp minus that of the
-    start stamp, mean over layers), in us; then the LM head."""
+def fewrow_trace_summary(tr):
+    """Per few-row launch kind (averaged over layers): each phase's median and
+    maximum over CTAs, in us after the previous launch's last exit (negative:
+    the CTA was resident before it), and the launch's span from that exit to
+    its own last exit."""
     tr = tr.astype(np.int64)
-    n_cta, per = tr.shape
-    L = (per - 2) // 16
-    lines = [f"  fused verify trace: {n_cta} CTAs, {L} layers, span {(tr.max() - tr[:, 0].min()) / 1e3:.1f} us"]
-    lines.append(f"  {'interval':<12}{'cta med':>9}{'cta max':>9}{'last->last':>12}")
-    tot = 0.0
-    for j in range(16):
-        med, mx, ll = [], [], []
-        for l in range(L):
-            a, b = tr[:, 16 * l + j], tr[:, 16 * l + j + 1]
-            dur = (b - a) / 1e3
-            med.append(np.median(dur))
-            mx.append(dur.max())
-            ll.append((b.max() - a.max()) / 1e3)
-        tot += np.mean(ll)
-        lines.append(f"  {FUSED_INTERVALS[j]:<12}{np.mean(med):>9.2f}{np.mean(mx):>9.2f}{np.mean(ll):>12.2f}")
-    lm = (tr[:, 16 * L + 1] - tr[:, 16 * L]) / 1e3
-    lines.append(f"  per layer (sum of last->last) {tot:.2f} us; LM head per CTA med {np.median(lm):.2f} "
-                 f"max {lm.max():.2f} us")
+    n = tr.shape[0]
+    lines = [f"  few-row trace: {n} launches; us after the previous launch's last CTA exit, median / max over CTAs"]
+    lines.append("  " + f"{'kind':<12}" + "".join(f"{p:>16}" for p in FEWROW_PHASES) + f"{'span':>9}")
+    acc = {k: [] for k in FEWROW_KINDS}
+    for i in range(1, n):
+        prev_exit = tr[i - 1][:, 7].max()
+        cta = tr[i][:, 0] > 0
+        with np.errstate(all="ignore"):
+            rel = np.where(tr[i][cta] > 0, (tr[i][cta] - prev_exit) / 1e3, np.nan)
+        acc[FEWROW_KINDS[i % 6]].append(rel)
+    import warnings
+    warnings.simplefilter("ignore", RuntimeWarning)
+    for k in FEWROW_KINDS:
+        if not acc[k]:
+            continue
+        med = np.nanmean([np.nanmedian(r, axis=0) for r in acc[k]], axis=0)
+        mx = np.nanmean([np.nanmax(r, axis=0) for r in acc[k]], axis=0)
+        cells = "".join(f"{a:>8.2f}/{b:<7.2f}" if np.isfinite(a) else f"{'-':>16}"
+                        for a, b in zip(med[:11], mx[:11]))
+        lines.append(f"  {k:<12}{cells}{mx[7]:>9.2f}")
     return "\n".join(lines)
 
 
@@ -156,8 +161,8 @@ def main():
                     help="also time each kernel class with CUDA events (direct launches)")
     ap.add_argument("--timeline", action="store_true",
                     help="also record the launch timeline of the rounds (direct launches) and summarise it per kind")
-    ap.add_argument("--fused-trace", action="store_true",
-                    help="also record the per-stage timestamps of one fused verify and summarise them")
+    ap.add_argument("--fewrow-trace", action="store_true",
+                    help="also record the per-CTA phase stamps of one verify's few-row launches and summarise them")
     ap.add_argument("--batch-sweep", default="",
                     help="comma-separated batch sizes: verification cost and anchor-readout share of the large "
                          "decoder at each (replaces the single-workload run)")
@@ -228,6 +233,12 @@ def main():
         ns, kinds = A.asr_spec_timeline_read(sess.h)
         A.asr_spec_timeline(sess.h, False)
         print(timeline_summary(ns, kinds, args.rounds))
+    if args.fewrow_trace:
+        A.asr_spec_fewrow_trace(sess.h, True)
+        sess.verify_device(drafts[0], lens, wl.k)
+        tr = A.asr_spec_fewrow_trace_read(sess.h)
+        A.asr_spec_fewrow_trace(sess.h, False)
+        print(fewrow_trace_summary(tr))
     if args.tree_nodes:
         n = args.tree_nodes
         trng = np.random.default_rng(9)
@@ -257,12 +268,6 @@ def main():
         print(f"  tree verify, {n} nodes per utterance: us per round " + " ".join(f"{u:.1f}" for u in tus)
               + f"; status {tsess.status()}")
         tsess.close()
-    if args.fused_trace:
-        A.asr_spec_fused_trace(sess.h, True)
-        sess.verify_device(drafts[0], lens, wl.k)
-        tr = A.asr_spec_fused_trace_read(sess.h)
-        A.asr_spec_fused_trace(sess.h, False)
-        print(fused_trace_summary(tr))
     sess.close()
     if st:
         sys.exit(1)
