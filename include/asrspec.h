@@ -164,6 +164,60 @@ int asr_spec_verify_tree(asr_spec_handle h, const int32_t* tokens, const int32_t
                          int32_t n, int32_t* accepted, int32_t* bonus, int32_t* kv_len, int32_t* anchor,
                          int32_t* path);
 
+/* ---- The draft (App. "Draft architecture"; Sec. 3 "Speculative Loop") ----
+ *
+ * A one-block draft beside the target: its input at position p is
+ *   w_in [f_1; f_2; f_3; f_4] + b_in + tok_emb[token] + pos_emb[p],
+ * f_i the target's residual stream after layer max(0, i L / 4 - 1) at the row
+ * that scored the token (position p - 1; zeros at p = 0); then one pre-LN
+ * causal block (self-attention over the draft's own cache, cross-attention to
+ * the encoder states through its own K/V projections, feed-forward of width
+ * 2 d with erf GELU), its own final LayerNorm and the target's tied LM head.
+ * Continuation proposals have no target row: the draft's own block output at
+ * p - 1 stands in for all four representations. */
+
+/* Window kinds of the draft's audio cross-attention (App. "Attention
+ * conditions", "Window geometry"): frames [c - 20, c + 20] clipped to
+ * [0, T) around centre c = the last verification's anchor (deployed
+ * correction, Sec. 5), the anchor + 25 frames clipped to T - 1 (shifted
+ * control), a caller-given centre (random control), or every frame. */
+#define ASR_DRAFT_WIN_ANCHOR 0
+#define ASR_DRAFT_WIN_SHIFTED 1
+#define ASR_DRAFT_WIN_RANDOM 2
+#define ASR_DRAFT_WIN_NONE 3
+
+/* Attach a draft to a bf16 handle, before asr_spec_encode_cache.
+ *   draft: host fp32 blob of 16 d^2 + 18 d floats, in this order (row-major,
+ *   [out][in]): w_in [d][4 d], b_in [d], ln1_g, ln1_b [d], wq [d][d], bq,
+ *   wk [d][d], wv [d][d], bv, wo [d][d], bo, ln2_g, ln2_b, wcq [d][d], bcq,
+ *   wck [d][d], wcv [d][d], bcv, wco [d][d], bco, ln3_g, ln3_b, w1 [2 d][d],
+ *   b1 [2 d], w2 [d][2 d], b2, lnf_g, lnf_b.  Copied; the caller keeps it.
+ * encode_cache then also builds the draft's cross K/V, prefill its cache of
+ * the prompt rows.  Synchronous.  Errors: ASR_E_INVAL (fp32 model, blob size,
+ * max_batch > 256, max_pos or max_enc > 16384), ASR_E_STATE (a draft already
+ * attached, or encode_cache already ran), ASR_E_OOM, ASR_E_CUDA. */
+int asr_spec_draft_create(asr_spec_handle h, const asr_weights* draft);
+
+/* One drafting round, entirely on the device.  Per utterance b with
+ * committed length P = kv_len[b] and N = total_len[b]:
+ *   lens_out[b] = -1 when P + 1 >= N (it holds its transcript), else the
+ *   proposals made, min(k, N - P - 2);
+ * the draft first re-processes the positions the last (linear) verification
+ * committed, from that verification's rows (catch-up, every frame), then
+ * scores the pending token at P (restart) and its own proposals at P + 1, ...
+ * (continuations), each with the round's audio window; proposal j is the
+ * argmax of the pass that scored position P + j - 1.
+ *   window: ASR_DRAFT_WIN_*; centers [B] int32 (ASR_DRAFT_WIN_RANDOM only,
+ *           frames in [0, enc_len[b])); before the first verification the
+ *           anchor is frame 0.
+ *   total_len [B] int32; draft_out [B][k] int32 (entries past lens_out[b]
+ *   are unspecified); lens_out [B] int32 -- both fit asr_spec_verify (tokens,
+ *   lens, k) as they are.
+ * Errors: ASR_E_INVAL (k outside [0, max_draft], window kind, null pointer),
+ * ASR_E_STATE (no draft, or no prefill). */
+int asr_spec_draft_propose(asr_spec_handle h, int32_t k, int32_t window, const int32_t* centers,
+                           const int32_t* total_len, int32_t* draft_out, int32_t* lens_out);
+
 /* The restart flags of the last verify (Sec. 3: after a rejected draft the
  * next round restarts drafting from the verified position, else it
  * continues): restart[b] = 1 when accepted[b] < lens[b] (linear verify) or

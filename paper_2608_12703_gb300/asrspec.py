@@ -29,8 +29,9 @@ EXPORTED = [
     "asr_spec_test_gemm", "asr_spec_set_graphs", "asr_spec_profile", "asr_spec_profile_read",
     "asr_spec_gemm_noalloc", "asr_spec_timeline", "asr_spec_timeline_read",
     "asr_spec_verify_tree", "asr_spec_restart", "asr_spec_fewrow_trace", "asr_spec_fewrow_trace_read",
-    "asr_spec_debug_anchor_profile",
+    "asr_spec_debug_anchor_profile", "asr_spec_draft_create", "asr_spec_draft_propose",
 ]
+DRAFT_WIN = {"anchor": 0, "shifted": 1, "random": 2, None: 3}
 PROF_CLASSES = ["qkv", "resid", "query", "mlp_up", "self_attn", "cross_attn", "lm_head", "layernorm", "other",
                 "qkv_self", "query_cross"]
 TL_CAP = 65536
@@ -83,6 +84,8 @@ def lib():
     L.asr_spec_verify_tree.argtypes = [vp, p32, p32, p32, i32, p32, p32, p32, p32, p32]
     L.asr_spec_rollback.argtypes = [vp, p32, p32]
     L.asr_spec_restart.argtypes = [vp, p32]
+    L.asr_spec_draft_create.argtypes = [vp, ctypes.POINTER(AsrWeights)]
+    L.asr_spec_draft_propose.argtypes = [vp, i32, i32, p32, p32, p32, p32]
     L.asr_spec_fewrow_trace.argtypes = [vp, i32]
     L.asr_spec_fewrow_trace_read.argtypes = [vp, vp, ctypes.c_int64, vp]
     L.asr_spec_debug_anchor_profile.argtypes = [vp, vp]
@@ -163,6 +166,17 @@ def asr_spec_verify_tree(h, tokens, parent, lens, n, accepted, bonus, kv_len, an
 
 def asr_spec_restart(h, restart):
     return _check(h, lib().asr_spec_restart(h, ptr(restart)), "asr_spec_restart")
+
+
+def asr_spec_draft_create(h, blob: np.ndarray):
+    blob = np.ascontiguousarray(blob, dtype=np.float32)
+    w = AsrWeights(blob.ctypes.data_as(ctypes.POINTER(ctypes.c_float)), blob.size)
+    return _check(h, lib().asr_spec_draft_create(h, ctypes.byref(w)), "asr_spec_draft_create")
+
+
+def asr_spec_draft_propose(h, k, window, centers, total_len, draft_out, lens_out):
+    return _check(h, lib().asr_spec_draft_propose(h, k, window, ptr(centers), ptr(total_len), ptr(draft_out),
+                                                  ptr(lens_out)), "asr_spec_draft_propose")
 
 
 def asr_spec_debug_anchor_profile(h, out):

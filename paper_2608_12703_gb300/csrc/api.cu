@@ -30,6 +30,18 @@ struct LayerW {
 
 }  // namespace
 
+// The one-block draft (asr_spec_draft_create): weights as the target layer's,
+// feed-forward width 2 d, its own cross K/V projections and final LayerNorm.
+struct DraftW {
+  void *w_in = nullptr, *wqkv = nullptr, *wo = nullptr, *wcq = nullptr, *wco = nullptr, *w1 = nullptr, *w2 = nullptr,
+       *w_cross = nullptr;
+  float *b_in = nullptr, *bqkv = nullptr, *bo = nullptr, *bcq = nullptr, *bco = nullptr, *b1 = nullptr, *b2 = nullptr,
+        *b_cross = nullptr;
+  float *ln1g = nullptr, *ln1b = nullptr, *ln2g = nullptr, *ln2b = nullptr, *ln3g = nullptr, *ln3b = nullptr,
+        *lnfg = nullptr, *lnfb = nullptr;
+  CUtensorMap m_in, m_qkv, m_wo, m_wcq, m_wco, m_w1, m_w2;
+};
+
 struct asr_spec {
   asr_model_dims dims{};
   int L = 0, d = 0, H = 0, F = 0, V = 0, maxpos = 0, Bmax = 0, kmax = 0, Tmax = 0, anchor = 0;
@@ -128,6 +140,20 @@ struct asr_spec {
     bool fused;       // the body runs the few-row layers
   };
   std::map<std::pair<int, int>, Graph> graphs;
+  // the draft: weights, caches, the tapped target rows and its pass buffers
+  bool has_draft = false;
+  DraftW dw;
+  int taps[4] = {0, 0, 0, 0};   // target layers whose outputs the draft reads
+  void *d_ks = nullptr, *d_vs = nullptr, *d_xkv = nullptr;
+  float *d_taps = nullptr, *d_last_tap = nullptr, *d_x = nullptr, *d_q = nullptr;
+  void *d_xin = nullptr, *d_xn = nullptr, *d_att = nullptr, *d_h = nullptr, *d_xf = nullptr;
+  RowPlan d_plan{};
+  int *d_row_src = nullptr, *d_row_lo = nullptr, *d_row_hi = nullptr, *d_win_lo = nullptr, *d_win_hi = nullptr;
+  int *d_lens = nullptr, *d_nprop = nullptr, *d_last_row = nullptr, *d_prev_pos = nullptr, *d_out = nullptr;
+  int *d_total = nullptr, *d_centers = nullptr, *d_lens_out = nullptr;
+  unsigned long long* d_row_key = nullptr;
+  bool d_after_verify = false;
+  int last_k = 0;   // k of the last linear verification (stride of its drafts)
 };
 
 namespace {
@@ -290,7 +316,8 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   return 0;
 }
 
-enum BufId { BUF_XN = 1, BUF_ATT = 2, BUF_H = 3, BUF_XF = 4 };
+enum BufId { BUF_XN = 1, BUF_ATT = 2, BUF_H = 3, BUF_XF = 4, BUF_DIN = 5, BUF_DXN = 6, BUF_DATT = 7, BUF_DH = 8,
+             BUF_DXF = 9 };
 
 // Folded LayerNorm of a consumer GEMM: B = xn (bf16(g * x), written by the
 // producer of x) and the producer's slice statistics.
@@ -354,6 +381,17 @@ void attention(asr_spec* h, AttnArgs& a, bool self_attn, int layer) {
   a.tl = h->tl_cur;
   launch_attention_tc(a, h->status, h->st);
   a.tl = nullptr;
+}
+
+// With a draft: the residual stream after a tapped layer into its column of
+// the tap rows [R][4][d] (the draft's inputs, App. "Draft architecture").
+int tap_copy(asr_spec* h, int l, int rows) {
+  if (!h->has_draft) return 0;
+  for (int i = 0; i < 4; ++i)
+    if (h->taps[i] == l)
+      CK(cudaMemcpy2DAsync(h->d_taps + (size_t)i * h->d, 4 * (size_t)h->d * 4, h->x, (size_t)h->d * 4,
+                           (size_t)h->d * 4, rows, cudaMemcpyDeviceToDevice, h->st));
+  return 0;
 }
 
 int run_layers(asr_spec* h, int N) {
@@ -472,6 +510,7 @@ int run_layers(asr_spec* h, int N) {
     e.x = h->x;
     producer(e, l + 1 < h->L ? h->lw[l + 1].ln1g : h->lnf_g);
     if (int rc = gemm_rows(h, w.w2, &w.m_w2, d, h->F, h->hbuf, BUF_H, N, EPI_RESID, e)) return rc;
+    if (int rc = tap_copy(h, l, N)) return rc;
   }
   return 0;
 }
@@ -610,8 +649,99 @@ int run_layers_few(asr_spec* h) {
       gd.trace = trace_slot();
       CK(launch_fr_gemv(gd, FR_RESID, KS, g_d, d, h->st, h->use_pdl));
     }
+    if (int rc = tap_copy(h, l, VF_ROWS)) return rc;
   }
   return 0;
+}
+
+// One pass of the draft's block over the rows of `plan` (at most `rows`):
+// input combination w_in [f_1..f_4] + b_in + embeddings, LayerNorm ->
+// self-attention over the draft's cache (K/V of the rows appended) -> out
+// projection; LayerNorm -> cross-attention over the draft's encoder K/V
+// (window per row) -> out projection; LayerNorm -> MLP (2 d, GELU); final
+// LayerNorm -> the target's tied LM head with argmax (when `lm`).
+int draft_block(asr_spec* h, const RowPlan& plan, int rows, bool lm) {
+  const int d = h->d, F2 = 2 * h->d;
+  DraftW& w = h->dw;
+  Epi base{};
+  base.n_valid = plan.n_rows;
+  base.d = d;
+  base.row_b = plan.row_b;
+  base.row_pos = plan.row_pos;
+  base.kv_bf16 = 1;
+  base.act_bf16 = 1;
+  base.max_pos = h->maxpos;
+  base.n_heads = h->H;
+  DraftArgs A{};
+  A.d = d;
+  A.plan = plan;
+  Epi e = base;
+  e.bias = w.b_in;
+  e.out_f32 = h->d_x;
+  if (int rc = gemm_rows(h, w.w_in, &w.m_in, d, 4 * d, h->d_xin, BUF_DIN, rows, EPI_Q, e)) return rc;
+  launch_draft_embed(A, rows, h->w_tok, h->w_pos, h->d_x, h->st);
+  auto ln = [&](const float* g, const float* b, void* y) {
+    launch_layernorm(h->d_x, g, b, y, 1, plan.n_rows, rows, d, h->st, false, nullptr);
+  };
+  DraftAttn at{};
+  at.q = h->d_q;
+  at.B = h->B;
+  at.H = h->H;
+  at.d = d;
+  at.plan = plan;
+  at.row_lo = h->d_row_lo;
+  at.row_hi = h->d_row_hi;
+  at.out = static_cast<__nv_bfloat16*>(h->d_att);
+  // self-attention block
+  ln(w.ln1g, w.ln1b, h->d_xn);
+  e = base;
+  e.bias = w.bqkv;
+  e.out_f32 = h->d_q;
+  e.kcache = h->d_ks;
+  e.vcache = h->d_vs;
+  if (int rc = gemm_rows(h, w.wqkv, &w.m_qkv, 3 * d, d, h->d_xn, BUF_DXN, rows, EPI_QKV, e)) return rc;
+  at.kc = static_cast<const __nv_bfloat16*>(h->d_ks);
+  at.vc = static_cast<const __nv_bfloat16*>(h->d_vs);
+  at.t_alloc = h->maxpos;
+  at.causal = 1;
+  launch_draft_attn(at, h->st);
+  e = base;
+  e.bias = w.bo;
+  e.x = h->d_x;
+  if (int rc = gemm_rows(h, w.wo, &w.m_wo, d, d, h->d_att, BUF_DATT, rows, EPI_RESID, e)) return rc;
+  // cross-attention block
+  ln(w.ln2g, w.ln2b, h->d_xn);
+  e = base;
+  e.bias = w.bcq;
+  e.out_f32 = h->d_q;
+  if (int rc = gemm_rows(h, w.wcq, &w.m_wcq, d, d, h->d_xn, BUF_DXN, rows, EPI_Q, e)) return rc;
+  const size_t half = (size_t)h->Bmax * h->H * h->Tmax * 64;
+  at.kc = static_cast<const __nv_bfloat16*>(h->d_xkv);
+  at.vc = static_cast<const __nv_bfloat16*>(h->d_xkv) + half;
+  at.t_alloc = h->Tmax;
+  at.causal = 0;
+  launch_draft_attn(at, h->st);
+  e = base;
+  e.bias = w.bco;
+  e.x = h->d_x;
+  if (int rc = gemm_rows(h, w.wco, &w.m_wco, d, d, h->d_att, BUF_DATT, rows, EPI_RESID, e)) return rc;
+  // MLP block
+  ln(w.ln3g, w.ln3b, h->d_xn);
+  e = base;
+  e.bias = w.b1;
+  e.act = h->d_h;
+  if (int rc = gemm_rows(h, w.w1, &w.m_w1, F2, d, h->d_xn, BUF_DXN, rows, EPI_GELU, e)) return rc;
+  e = base;
+  e.bias = w.b2;
+  e.x = h->d_x;
+  if (int rc = gemm_rows(h, w.w2, &w.m_w2, d, F2, h->d_h, BUF_DH, rows, EPI_RESID, e)) return rc;
+  if (!lm) return 0;
+  ln(w.lnfg, w.lnfb, h->d_xf);
+  e = Epi{};
+  e.n_valid = plan.n_rows;
+  e.row_key = h->d_row_key;
+  e.d = d;
+  return gemm_rows(h, h->w_tok, &h->m_tok, h->V, d, h->d_xf, BUF_DXF, rows, EPI_ARGMAX, e);
 }
 
 bool dims_ok(const asr_model_dims& m) {
@@ -1035,6 +1165,24 @@ int asr_spec_encode_cache(asr_spec_handle h, int32_t B, const void* enc_states, 
     Prof pg(h, ASR_PROF_OTHER, 1);
     launch_gemm_simt(enc_states, 0, h->w_cross, 0, M, N, d, EPI_CROSSKV, e, h->st);
   }
+  if (h->has_draft && h->bf16) {   // the draft's own cross K/V of the same encoder states
+    Epi de = e;
+    de.bias = h->dw.b_cross;
+    de.kcache = h->d_xkv;
+    de.N = 2 * d;
+    TcGemm g{};
+    g.bn = h->enc_bn;
+    if (!make_tmap_bf16(&g.mapA, enc_states, M, d, 128) || !make_tmap_bf16(&g.mapB, h->dw.w_cross, 2 * d, d, g.bn))
+      return fail(h, ASR_E_INVAL, "encoder states must be 16-byte aligned");
+    g.M = M;
+    g.N = 2 * d;
+    g.K = d;
+    g.splits = 1;
+    g.ws = h->ws;
+    g.tickets = h->tickets;
+    Prof pg(h, ASR_PROF_OTHER, 1);
+    launch_gemm_tc(g, EPI_CROSSKV, de, h->status, h->st);
+  }
   CK(cudaGetLastError());
   h->B = B;
   h->t_max = t_max;
@@ -1049,6 +1197,10 @@ int asr_spec_prefill(asr_spec_handle h, const int32_t* prompt, int32_t P0) {
   if (!prompt || P0 < 1) return fail(h, ASR_E_INVAL, "bad arguments");
   if (P0 > h->maxpos) return fail(h, ASR_E_CAPACITY, "prompt longer than max_pos");
   if (int rc = copy_in(h, h->prompt_buf, prompt, (size_t)h->B * P0)) return rc;
+  if (h->has_draft) {
+    CK(cudaMemsetAsync(h->d_last_tap, 0, (size_t)h->Bmax * 4 * h->d * 4, h->st));
+    h->d_after_verify = false;
+  }
   const int c_max = h->kmax + 1;
   for (int p0 = 0; p0 < P0 - 1; p0 += c_max) {
     const int c = std::min(c_max, P0 - 1 - p0);
@@ -1057,6 +1209,20 @@ int asr_spec_prefill(asr_spec_handle h, const int32_t* prompt, int32_t P0) {
       launch_plan_prefill_chunk(h->prompt_buf, P0, p0, c, h->B, h->V, h->ready, h->plan, h->status, h->st);
     }
     if (int rc = run_layers(h, h->B * c)) return rc;
+    if (h->has_draft) {   // the draft's cache of the same prompt rows (their taps as its inputs)
+      DraftArgs A{};
+      A.B = h->B;
+      A.d = h->d;
+      A.enc_len = h->enc_len;
+      A.taps = h->d_taps;
+      A.last_tap = h->d_last_tap;
+      A.plan = h->plan;
+      A.row_lo = h->d_row_lo;
+      A.row_hi = h->d_row_hi;
+      A.x_in = static_cast<__nv_bfloat16*>(h->d_xin);
+      launch_draft_prefill_gather(A, h->B * c, h->st);
+      if (int rc = draft_block(h, h->plan, h->B * c, false)) return rc;
+    }
     Prof p(h, ASR_PROF_OTHER, 1);
     launch_prefill_advance(h->B, c, h->plan.n_utt_rows, h->kv_len, h->st);
   }
@@ -1126,6 +1292,8 @@ int verify_call(asr_spec* h, const int32_t* draft, const int32_t* parent, const 
   if (int rc = copy_out(h, anchor, o + 3 * h->Bmax, B)) return rc;
   if (tree && path && k > 0)
     if (int rc = copy_out(h, path, h->path_buf, (size_t)B * k)) return rc;
+  h->d_after_verify = h->has_draft && !tree;
+  if (!tree) h->last_k = k;
   if (h->host_io) CK(cudaStreamSynchronize(h->st));
   return ASR_OK;
 }
@@ -1152,6 +1320,211 @@ int asr_spec_verify_tree(asr_spec_handle h, const int32_t* tokens, const int32_t
   if (!lens || (n > 0 && (!tokens || !parent || !path)) || !accepted || !bonus || !kv_len || !anchor)
     return fail(h, ASR_E_INVAL, "null pointer");
   return verify_call(h, tokens, n > 0 ? parent : nullptr, lens, n, accepted, bonus, kv_len, anchor, path);
+}
+
+int asr_spec_draft_create(asr_spec_handle h, const asr_weights* dw) {
+  if (!h || !dw || !dw->blob) return ASR_E_INVAL;
+  if (!h->bf16) return fail(h, ASR_E_INVAL, "the draft needs a bf16 model");
+  if (h->has_draft) return fail(h, ASR_E_STATE, "the handle already has a draft");
+  if (h->state != 0) return fail(h, ASR_E_STATE, "create the draft before encode_cache");
+  if (h->Bmax > 256) return fail(h, ASR_E_INVAL, "the draft serves at most 256 utterances");
+  if (h->maxpos > 16384 || h->Tmax > 16384) return fail(h, ASR_E_INVAL, "the draft attends to at most 16384 keys");
+  const int d = h->d, F2 = 2 * d, L = h->L;
+  const size_t expect = 16 * (size_t)d * d + 18 * (size_t)d;
+  if (dw->n_floats != expect) return fail(h, ASR_E_INVAL, "draft blob size");
+  const float* src = dw->blob;
+  size_t off = 0;
+  auto take = [&](size_t n) {
+    const float* p = src + off;
+    off += n;
+    return p;
+  };
+  DraftW& w = h->dw;
+  int rc = 0;
+  auto vec = [&](float** dst, size_t n, const float* v) {
+    int r = dalloc(h, dst, n * 4);
+    if (!r) r = upload_f32(h, *dst, v, n);
+    return r;
+  };
+  auto mat = [&](void** dst, size_t n, const float* v) {
+    int r = dalloc(h, dst, n * 2);
+    if (!r) r = upload(h, *dst, v, n);
+    return r;
+  };
+  const float* w_in = take((size_t)4 * d * d);
+  const float* b_in = take(d);
+  const float* ln1g = take(d);
+  const float* ln1b = take(d);
+  const float* wq = take((size_t)d * d);
+  const float* bq = take(d);
+  const float* wk = take((size_t)d * d);
+  const float* wv = take((size_t)d * d);
+  const float* bv = take(d);
+  const float* wo = take((size_t)d * d);
+  const float* bo = take(d);
+  const float* ln2g = take(d);
+  const float* ln2b = take(d);
+  const float* wcq = take((size_t)d * d);
+  const float* bcq = take(d);
+  const float* wck = take((size_t)d * d);
+  const float* wcv = take((size_t)d * d);
+  const float* bcv = take(d);
+  const float* wco = take((size_t)d * d);
+  const float* bco = take(d);
+  const float* ln3g = take(d);
+  const float* ln3b = take(d);
+  const float* w1 = take((size_t)F2 * d);
+  const float* b1 = take(F2);
+  const float* w2 = take((size_t)d * F2);
+  const float* b2 = take(d);
+  const float* lnfg = take(d);
+  const float* lnfb = take(d);
+  std::vector<float> tmp((size_t)3 * d * d);
+  std::memcpy(tmp.data(), wq, (size_t)d * d * 4);
+  std::memcpy(tmp.data() + (size_t)d * d, wk, (size_t)d * d * 4);
+  std::memcpy(tmp.data() + (size_t)2 * d * d, wv, (size_t)d * d * 4);
+  std::vector<float> bqkv(3 * d, 0.f), bx(2 * d, 0.f), wx((size_t)2 * d * d);
+  std::memcpy(bqkv.data(), bq, d * 4);
+  std::memcpy(bqkv.data() + 2 * d, bv, d * 4);
+  std::memcpy(wx.data(), wck, (size_t)d * d * 4);
+  std::memcpy(wx.data() + (size_t)d * d, wcv, (size_t)d * d * 4);
+  std::memcpy(bx.data() + d, bcv, d * 4);
+  if ((rc = mat(&w.w_in, (size_t)4 * d * d, w_in)) || (rc = vec(&w.b_in, d, b_in)) ||
+      (rc = mat(&w.wqkv, (size_t)3 * d * d, tmp.data())) || (rc = vec(&w.bqkv, 3 * d, bqkv.data())) ||
+      (rc = mat(&w.wo, (size_t)d * d, wo)) || (rc = vec(&w.bo, d, bo)) || (rc = mat(&w.wcq, (size_t)d * d, wcq)) ||
+      (rc = vec(&w.bcq, d, bcq)) || (rc = mat(&w.w_cross, (size_t)2 * d * d, wx.data())) ||
+      (rc = vec(&w.b_cross, 2 * d, bx.data())) || (rc = mat(&w.wco, (size_t)d * d, wco)) || (rc = vec(&w.bco, d, bco)) ||
+      (rc = mat(&w.w1, (size_t)F2 * d, w1)) || (rc = vec(&w.b1, F2, b1)) || (rc = mat(&w.w2, (size_t)d * F2, w2)) ||
+      (rc = vec(&w.b2, d, b2)) || (rc = vec(&w.ln1g, d, ln1g)) || (rc = vec(&w.ln1b, d, ln1b)) ||
+      (rc = vec(&w.ln2g, d, ln2g)) || (rc = vec(&w.ln2b, d, ln2b)) || (rc = vec(&w.ln3g, d, ln3g)) ||
+      (rc = vec(&w.ln3b, d, ln3b)) || (rc = vec(&w.lnfg, d, lnfg)) || (rc = vec(&w.lnfb, d, lnfb)))
+    return rc;
+  if (!make_tmap_bf16(&w.m_in, w.w_in, d, 4 * d, 128) || !make_tmap_bf16(&w.m_qkv, w.wqkv, 3 * d, d, 128) ||
+      !make_tmap_bf16(&w.m_wo, w.wo, d, d, 128) || !make_tmap_bf16(&w.m_wcq, w.wcq, d, d, 128) ||
+      !make_tmap_bf16(&w.m_wco, w.wco, d, d, 128) || !make_tmap_bf16(&w.m_w1, w.w1, F2, d, 128) ||
+      !make_tmap_bf16(&w.m_w2, w.w2, d, F2, 128))
+    return fail(h, ASR_E_CUDA, "tensor map encode failed");
+  for (int i = 0; i < 4; ++i) h->taps[i] = std::max(0, (i + 1) * L / 4 - 1);
+  const size_t Bm = h->Bmax, R = h->R_pad;
+  const size_t self_b = Bm * h->H * h->maxpos * 64 * 2, cross_b = 2 * Bm * h->H * h->Tmax * 64 * 2;
+  if ((rc = dalloc(h, &h->d_ks, self_b)) || (rc = dalloc(h, &h->d_vs, self_b)) || (rc = dalloc(h, &h->d_xkv, cross_b)) ||
+      (rc = dalloc(h, &h->d_taps, R * 4 * d * 4)) || (rc = dalloc(h, &h->d_last_tap, Bm * 4 * d * 4)) ||
+      (rc = dalloc(h, &h->d_x, R * d * 4)) || (rc = dalloc(h, &h->d_q, R * 3 * d * 4)) ||
+      (rc = dalloc(h, &h->d_xin, R * 4 * d * 2)) || (rc = dalloc(h, &h->d_xn, R * d * 2)) ||
+      (rc = dalloc(h, &h->d_att, R * d * 2)) || (rc = dalloc(h, &h->d_h, R * F2 * 2)) ||
+      (rc = dalloc(h, &h->d_xf, R * d * 2)) || (rc = dalloc(h, &h->d_row_key, R * 8)))
+    return rc;
+  RowPlan& p = h->d_plan;
+  int* ints = nullptr;
+  const size_t n_int = 7 * R + (Bm + 1) + 1 + Bm + 3 * R + 9 * Bm + Bm * std::max(h->kmax, 1);
+  if ((rc = dalloc(h, &ints, n_int * 4))) return rc;
+  CK(cudaMemset(ints, 0, n_int * 4));
+  int* q = ints;
+  auto cut = [&](size_t n) {
+    int* r = q;
+    q += n;
+    return r;
+  };
+  p.row_b = cut(R);
+  p.row_i = cut(R);
+  p.row_pos = cut(R);
+  p.row_epos = cut(R);
+  p.row_mask = reinterpret_cast<unsigned*>(cut(R));
+  p.row_tok = cut(R);
+  (void)cut(R);
+  p.row_start = cut(Bm + 1);
+  p.n_rows = cut(1);
+  p.n_utt_rows = cut(Bm);
+  h->d_row_src = cut(R);
+  h->d_row_lo = cut(R);
+  h->d_row_hi = cut(R);
+  h->d_win_lo = cut(Bm);
+  h->d_win_hi = cut(Bm);
+  h->d_lens = cut(Bm);
+  h->d_nprop = cut(Bm);
+  h->d_last_row = cut(Bm);
+  h->d_prev_pos = cut(Bm);
+  h->d_total = cut(Bm);
+  h->d_centers = cut(Bm);
+  h->d_lens_out = cut(Bm);
+  h->d_out = cut(Bm * std::max(h->kmax, 1));
+  CK(cudaMemset(h->d_ks, 0, self_b));
+  CK(cudaMemset(h->d_vs, 0, self_b));
+  CK(cudaMemset(h->d_xkv, 0, cross_b));
+  CK(cudaDeviceSynchronize());
+  h->has_draft = true;
+  return ASR_OK;
+}
+
+int asr_spec_draft_propose(asr_spec_handle h, int32_t k, int32_t window, const int32_t* centers,
+                           const int32_t* total_len, int32_t* draft_out, int32_t* lens_out) {
+  if (!h) return ASR_E_INVAL;
+  if (!h->has_draft) return fail(h, ASR_E_STATE, "no draft (asr_spec_draft_create)");
+  if (h->state < 2) return fail(h, ASR_E_STATE, "propose before prefill");
+  if (k < 0 || k > h->kmax) return fail(h, ASR_E_INVAL, "k outside [0, max_draft]");
+  if (window < DRAFT_WIN_ANCHOR || window > DRAFT_WIN_NONE) return fail(h, ASR_E_INVAL, "window kind");
+  if (!total_len || !lens_out || (k > 0 && !draft_out) || (window == DRAFT_WIN_RANDOM && !centers))
+    return fail(h, ASR_E_INVAL, "null pointer");
+  const int B = h->B;
+  if (int rc = copy_in(h, h->d_total, total_len, B)) return rc;
+  if (window == DRAFT_WIN_RANDOM)
+    if (int rc = copy_in(h, h->d_centers, centers, B)) return rc;
+  DraftArgs A{};
+  A.B = B;
+  A.d = h->d;
+  A.k = k;
+  A.k_verify = h->last_k;
+  A.win_kind = window;
+  A.vocab = h->V;
+  A.max_pos = h->maxpos;
+  A.status = h->status;
+  A.after_verify = h->d_after_verify ? 1 : 0;
+  A.kv_len = h->kv_len;
+  A.pending = h->pending;
+  A.enc_len = h->enc_len;
+  A.total_len = h->d_total;
+  A.v_row_start = h->plan.row_start;
+  A.v_n_utt_rows = h->plan.n_utt_rows;
+  A.accepted = h->out4;
+  A.anchor = h->out4 + 3 * h->Bmax;
+  A.v_draft = h->draft_buf;
+  A.centers = h->d_centers;
+  A.taps = h->d_taps;
+  A.last_tap = h->d_last_tap;
+  A.x_prev = h->d_x;
+  A.plan = h->d_plan;
+  A.row_src = h->d_row_src;
+  A.row_lo = h->d_row_lo;
+  A.row_hi = h->d_row_hi;
+  A.win_lo = h->d_win_lo;
+  A.win_hi = h->d_win_hi;
+  A.lens = h->d_lens;
+  A.n_prop = h->d_nprop;
+  A.last_row = h->d_last_row;
+  A.prev_pos = h->d_prev_pos;
+  A.draft_out = h->d_out;
+  A.row_key = h->d_row_key;
+  A.x_in = static_cast<__nv_bfloat16*>(h->d_xin);
+  // pass 0: catch-up of the last verification's accepted drafts + the restart
+  const int rows0 = std::min(h->R_pad, B * (h->kmax + 1));
+  launch_draft_round_plan(A, h->st);
+  launch_draft_gather(A, rows0, h->st);
+  if (int rc = draft_block(h, h->d_plan, rows0, true)) return rc;
+  launch_draft_take(A, h->st);
+  for (int i = 1; i < k; ++i) {   // continuation proposals, one row per utterance still proposing
+    launch_draft_next_plan(A, i, h->st);
+    launch_draft_gather(A, B, h->st);
+    if (int rc = draft_block(h, h->d_plan, B, true)) return rc;
+    launch_draft_take(A, h->st);
+  }
+  launch_draft_finish(A, h->d_lens_out, h->st);
+  CK(cudaGetLastError());
+  h->d_after_verify = false;
+  if (k > 0)
+    if (int rc = copy_out(h, draft_out, h->d_out, (size_t)B * k)) return rc;
+  if (int rc = copy_out(h, lens_out, h->d_lens_out, B)) return rc;
+  if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
 }
 
 int asr_spec_restart(asr_spec_handle h, int32_t* restart) {
@@ -1275,6 +1648,7 @@ int asr_spec_rollback(asr_spec_handle h, const int32_t* new_len, const int32_t* 
   Prof p(h, ASR_PROF_OTHER, 1);
   launch_rollback(h->misc, h->lens_buf, h->B, h->V, h->kv_len, h->pending, h->status, h->st);
   CK(cudaGetLastError());
+  h->d_after_verify = false;   // the draft has no verification rows of the rewound state
   if (h->host_io) CK(cudaStreamSynchronize(h->st));
   return ASR_OK;
 }

@@ -214,6 +214,50 @@ cudaError_t launch_fr_self(const CUtensorMap* kmap, const CUtensorMap* vmap, con
                            bool pdl);
 cudaError_t launch_fr_cross(const CUtensorMap* xmap, const FrHead& a, cudaStream_t st, bool pdl);
 
+// ---- Draft side (csrc/draft.cu) ---------------------------------------------------
+// Window centre of the draft's audio cross-attention for proposals
+// (App. "Window geometry"): the verification anchor (deployed), 500 ms later
+// (shifted control), a given frame (random control), or no window.
+enum DraftWin : int { DRAFT_WIN_ANCHOR = 0, DRAFT_WIN_SHIFTED = 1, DRAFT_WIN_RANDOM = 2, DRAFT_WIN_NONE = 3 };
+struct DraftArgs {
+  int B, d, k, k_verify, win_kind;
+  int vocab, max_pos;
+  int* status;               // device status word (ASR_ST_* bits)
+  int after_verify;          // 1: a verification ran since the last round (catch-up rows)
+  const int *kv_len, *pending, *enc_len, *total_len;
+  const int *v_row_start, *v_n_utt_rows;   // the last verification's row plan
+  const int *accepted, *anchor;             // its outputs
+  const int* v_draft;        // [B][k_verify] its drafts
+  const int* centers;        // [B] window centres of the random control, or null
+  const float* taps;         // [R][4][d] tapped target rows (verification or prefill chunk)
+  float* last_tap;           // [B_max][4][d] the tap of the last prompt row per utterance
+  const float* x_prev;       // [R][d] the previous pass's block output (continuation rows)
+  RowPlan plan;              // the draft pass's rows
+  int *row_src, *row_lo, *row_hi;   // [R_max] feature source; audio window [lo, hi) per row
+  int *win_lo, *win_hi;      // [B_max] the round's window
+  int *lens, *n_prop, *last_row, *prev_pos;   // [B_max]
+  int* draft_out;            // [B][k] proposals
+  unsigned long long* row_key;   // [R_max] LM-head argmax keys of the pass
+  __nv_bfloat16* x_in;       // [R_max][4 d] the pass's input representations
+};
+struct DraftAttn {
+  const float* q;            // [R][d] fp32
+  const __nv_bfloat16 *kc, *vc;   // [B_max][H][t_alloc][64]
+  int t_alloc, B, H, d, causal;
+  RowPlan plan;
+  const int *row_lo, *row_hi;
+  __nv_bfloat16* out;        // [R][d]
+};
+void launch_draft_round_plan(const DraftArgs& a, cudaStream_t st);
+void launch_draft_next_plan(const DraftArgs& a, int i, cudaStream_t st);
+void launch_draft_gather(const DraftArgs& a, int rows_max, cudaStream_t st);
+void launch_draft_prefill_gather(const DraftArgs& a, int rows_max, cudaStream_t st);
+void launch_draft_embed(const DraftArgs& a, int rows_max, const void* tok_emb, const void* pos_emb, float* x,
+                        cudaStream_t st);
+void launch_draft_take(const DraftArgs& a, cudaStream_t st);
+void launch_draft_finish(const DraftArgs& a, int* lens_out, cudaStream_t st);
+void launch_draft_attn(const DraftAttn& a, cudaStream_t st);
+
 // ---- Accept / commit ------------------------------------------------------------
 void launch_prefill_advance(int B, int c, const int* n_utt_rows, int* kv_len, cudaStream_t st);
 void launch_prefill_finish(const int* prompt, int P0, int B, int* pending, const int* ready, cudaStream_t st);

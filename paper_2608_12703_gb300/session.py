@@ -2,9 +2,9 @@
 
 PyTorch supplies device memory and the CUDA stream; every computation runs in
 the library's kernels.  ``Session`` mirrors the C ABI one call per method;
-``decode_device`` runs a whole speculative decode on the device with the
-library's synthetic draft source, and ``decode_host`` runs it through host
-buffers (one call per round, as a user without device memory would).
+``DeviceDrafts`` is the library's synthetic draft source (a reference
+transcript plus corruptions) and ``DraftModel`` its one-block draft model;
+both hand each round's drafts to ``verify_device`` without leaving the GPU.
 """
 from __future__ import annotations
 
@@ -209,3 +209,38 @@ class DeviceDrafts:
         A.asr_spec_synth_drafts(self.sess.h, self.truth, self.total, self.repl, self.k_repl, self.shift, self.k,
                                 self.draft, self.lens)
         return self.draft, self.lens
+
+
+class DraftModel:
+    """The one-block draft on the device (App. "Draft architecture"): attach it
+    to a session before ``encode_cache``; ``propose`` runs one drafting round
+    (catch-up of the last verification, restart, continuations) and leaves
+    drafts and lens on the device, ready for ``Session.verify_device``."""
+
+    def __init__(self, sess: Session, blob: np.ndarray, total_lens, k: int, window="anchor"):
+        if sess.B:
+            raise A.AsrSpecError("attach the draft before encode_cache")
+        A.asr_spec_draft_create(sess.h, blob)
+        self.sess, self.k, self.window = sess, k, A.DRAFT_WIN[window]
+        dev = sess.dev
+        with torch.cuda.stream(sess.stream):
+            self.total = torch.tensor(np.asarray(total_lens, dtype=np.int32), device=dev)
+            n = self.total.numel()
+            self.centers = torch.zeros(n, dtype=torch.int32, device=dev)
+            self.draft = torch.zeros((n, max(k, 1)), dtype=torch.int32, device=dev)
+            self.lens = torch.zeros(n, dtype=torch.int32, device=dev)
+        sess.stream.synchronize()
+
+    def set_centers(self, centers):
+        """Window centres of the random control for the next round (host ints)."""
+        with torch.cuda.stream(self.sess.stream):
+            self.centers.copy_(torch.from_numpy(np.asarray(centers, dtype=np.int32)))
+
+    def propose(self, k: Optional[int] = None):
+        """One round of at most k (default: the k given at creation) proposals."""
+        k = self.k if k is None else k
+        if k > self.k:
+            raise A.AsrSpecError("k above the draft buffer's width")
+        A.asr_spec_draft_propose(self.sess.h, k, self.window, self.centers, self.total, self.draft, self.lens)
+        n = self.lens.numel()
+        return self.draft.view(-1)[:n * k].view(n, k), self.lens   # [B][k], row stride k
