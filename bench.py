@@ -38,6 +38,9 @@ import workload as W  # noqa: E402
 
 MAIN_CONFIG = "large-bf16-b64-k6"
 BATCH1_CONFIG = "large-bf16-b1-k8"
+# the other workloads, reported as extra keys: the tiny fp32 decoder, the
+# small decoder at batch 16 and one point of the batch-32 acceptance/rollback sweep
+EXTRA_CONFIGS = ("small-bf16-b16-k8", "small-bf16-b32-k16-p0.2", "tiny-fp32-b1-k4")
 METRIC = "accepted tokens/s"
 
 
@@ -378,15 +381,103 @@ class DecodeRun:
                     h2d_bytes_per_step=int(h2d // steps), d2h_bytes_per_step=int(d2h // steps), seconds=dt)
 
 
-# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one
-# ncu capture of the kernel on the workload, as summarised in profiles/; averaged
-# over the kernel's launches in one layer.  Only valid for the kernel code the
-# capture ran on: drop an entry when that kernel changes.
-NCU_TRAFFIC = {
-    ("large-bf16-b1-k8", "resid"): (6.76e6, "profiles/gemm_tc_kernel_resid_large-bf16-b1-k8.md"),
-    ("large-bf16-b64-k6", "resid"): (11.21e6, "profiles/gemm_tc_kernel_large-bf16-b64-k6_tensor.md"),
-    ("large-bf16-b64-k6", "cross_attn"): (337.7e6, "profiles/attn_tc_kernel_large-bf16-b64-k6_dram.md"),
-}
+class DraftLoop:
+    """The real cached loop on the device (Sec. 3 "Speculative Loop"): each
+    round the library's one-block draft proposes (catch-up of the last
+    verification, restart, k - 1 continuations, audio window around the last
+    anchor), the target verifies, nothing is read back in between.  The draft
+    is random-init (no trained weights): its acceptance is not the paper's,
+    its cost is.  rho = one draft step / one verification (Eq. breakeven),
+    one draft step = a round's drafting time / k."""
+
+    def __init__(self, wl: W.Workload, window="anchor"):
+        import torch
+        from paper_2608_12703_gb300.session import DraftModel, Session
+        self.torch, self.wl = torch, wl
+        dims = wl.dims
+        self.sess = Session(dims, weights(dims), max_batch=wl.batch, max_draft=wl.k)
+        self.dm = DraftModel(self.sess, W.make_draft_weights(dims), wl.total_lens, wl.k, window)
+        enc = W.make_encoder_states(dims, wl.enc_lens, wl.t_max)
+        self.prompt = W.make_prompt(dims, wl.batch)
+        with torch.cuda.stream(self.sess.stream):
+            self.enc = torch.from_numpy(enc).to("cuda").to(self.sess.storage_dtype)
+            self.enc_lens_d = torch.from_numpy(np.array(wl.enc_lens, dtype=np.int32)).cuda()
+            self.prompt_d = torch.from_numpy(self.prompt).cuda()
+        self.sess.stream.synchronize()
+        self.rounds, self.emitted, self.acc_sum, self.offered = self._count_rounds()
+
+    def _begin(self):
+        from paper_2608_12703_gb300 import asrspec as A
+        s = self.sess
+        A.asr_spec_encode_cache(s.h, self.wl.batch, self.enc, self.wl.t_max, self.enc_lens_d)
+        s.B = self.wl.batch
+        A.asr_spec_prefill(s.h, self.prompt_d, self.prompt.shape[1])
+
+    def _count_rounds(self):
+        self._begin()
+        n = emitted = acc = offered = 0
+        while True:
+            d, l = self.dm.propose()
+            lh = self.sess.host(l)
+            if (lh < 0).all():
+                break
+            o = self.sess.host(self.sess.verify_device(d, l, self.wl.k))
+            live = lh >= 0
+            emitted += int(o[0][live].sum() + live.sum())
+            acc += int(o[0][live].sum())
+            offered += int(lh[live].sum())
+            n += 1
+        kv, _ = self.sess.state()
+        assert np.array_equal(kv + 1, self.wl.total_lens), (kv, self.wl.total_lens)
+        assert self.sess.status() == 0
+        return n, emitted, acc, offered
+
+    def decode(self, ev=None):
+        self._begin()
+        torch, k = self.torch, self.wl.k
+        for _ in range(self.rounds):
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(3)] if ev is not None else None
+            if e:
+                e[0].record(self.sess.stream)
+            d, l = self.dm.propose()
+            if e:
+                e[1].record(self.sess.stream)
+            self.sess.verify_device(d, l, k)
+            if e:
+                e[2].record(self.sess.stream)
+                ev.append(e)
+
+    def timed(self, steps, warmup):
+        torch = self.torch
+        for _ in range(warmup):
+            self.decode()
+        torch.cuda.synchronize()
+        ev = []
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(self.sess.stream)
+        for _ in range(steps):
+            self.decode(ev)
+        end.record(self.sess.stream)
+        torch.cuda.synchronize()
+        assert self.sess.status() == 0
+        ms = start.elapsed_time(end)
+        draft_us = np.array([a.elapsed_time(b) for a, b, _ in ev]) * 1e3
+        verify_us = np.array([b.elapsed_time(c) for _, b, c in ev]) * 1e3
+        k = self.wl.k
+        step_us = float(np.median(draft_us)) / k
+        return {"workload": self.wl.name, "window": "anchor", "draft": "one-block, random-init (seeded)",
+                "value": steps * self.emitted / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms / steps,
+                "rounds_per_step": self.rounds, "emitted_per_step": self.emitted,
+                "mean_accepted_per_round": self.acc_sum / max(self.rounds, 1),
+                "acceptance_of_offered": self.acc_sum / max(self.offered, 1),
+                "draft_round_us": {"median": float(np.median(draft_us)), "p10": float(np.percentile(draft_us, 10)),
+                                   "p90": float(np.percentile(draft_us, 90))},
+                "verify_us": {"median": float(np.median(verify_us)), "p10": float(np.percentile(verify_us, 10)),
+                              "p90": float(np.percentile(verify_us, 90))},
+                "draft_step_us": step_us, "rho": step_us / float(np.median(verify_us)),
+                "draft_share_of_loop": float(draft_us.sum() / (draft_us.sum() + verify_us.sum())),
+                "steps": steps, "warmup": warmup}
+
 
 # Launch kinds of the timeline (ASR_TL_*; a LayerNorm-fused GEMM counts with its
 # GEMM) and the profile class (CUDA events) that times the same kernel.
@@ -473,7 +564,8 @@ def roofline(wl_name, dims, tl, ms, launches, traffic, pk):
         bound, unit, peak, work, scale = "hbm", "GB/s", pk["hbm"], nbytes, 1e9
     achieved = work / t / scale
     chain = work / busy[name] / scale
-    ncu = NCU_TRAFFIC.get((wl_name, name))
+    from paper_2608_12703_gb300.ncu_traffic import lookup
+    ncu = lookup(wl_name, name)   # None unless captured on the kernel's current sources
     return {"kernel": name, "bound": bound, "achieved": round(achieved, 2), "peak": peak, "unit": unit,
             "frac": round(achieved / peak, 4), "traffic": ncu[0] if ncu else None,
             "traffic_source": ncu[1] if ncu else None,
@@ -497,6 +589,30 @@ def step_bytes(dims, traffic, calls_override=None):
     w = L * (6 * d * d + 2 * F * d) * es + V * d * es
     kv = float(traffic[1]) + float(traffic[2]) + float(traffic[3])
     return (calls * w + kv) / max(calls, 1)
+
+
+def extra_config(wl: W.Workload, pk, gpu_index: int, cpu_seconds: float, steps: int = 2, warmup: int = 3):
+    """One more workload: whole-decode tokens/s, per-call verify latency, the
+    verify step's HBM fraction, and the oracle on a bounded sample of it (the
+    whole decode where it fits the time)."""
+    run = DecodeRun(wl)
+    res = run.timed(steps, warmup, None, gpu_index=gpu_index)
+    _, _, traffic = run.profile()
+    bpc = step_bytes(wl.dims, traffic)
+    med = res["verify_us"]["median"]
+    tokens, dt, rounds, desc = oracle_sample(wl, run.truth, cpu_seconds)
+    out = {"value": steps * run.tokens_per_decode / (res["ms"] / 1e3), "unit": "tokens/s",
+           "ms_per_step": res["ms"] / steps, "steps": steps, "warmup": warmup,
+           "dtype": "bf16" if wl.dims.dtype == "bf16" else "f32", "batch": wl.batch, "k": wl.k,
+           "verify_us": res["verify_us"], "verify_rounds_per_step": run.rounds,
+           "verify_hbm": {"bytes_per_call": bpc, "frac": bpc / (med * 1e-6) / (pk["hbm"] * 1e9),
+                          "frac_nominal_8tbs": bpc / (med * 1e-6) / 8e12},
+           "clocks": res["clocks"], "gpu_launches": res["launches"],
+           "cpu_baseline": {"value": tokens / dt, "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
+                            "seconds_per_verify_round": dt / max(rounds, 1), "sample": desc}}
+    run.sess.close()
+    del run
+    return out
 
 
 # ----------------------------------------------------------------------------
@@ -613,6 +729,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-batch1", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-extra", action="store_true", help="skip the draft loops and the other workloads")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     args = ap.parse_args()
     if args.warmup < 3:
@@ -692,6 +809,19 @@ def main():
                                "frac": bpc / (b1["verify_us"]["median"] * 1e-6) / (pk["hbm"] * 1e9),
                                "frac_nominal_8tbs": bpc / (b1["verify_us"]["median"] * 1e-6) / 8e12},
                 "clocks": b1["clocks"], "roofline": roofline(wl1.name, wl1.dims, tl1, pm, pl, pt, pk)}
+            del r1
+        if not args.no_extra:
+            line["draft_loop"] = {}
+            for name in (BATCH1_CONFIG, args.config):
+                torch.cuda.empty_cache()
+                dl = DraftLoop(W.CONFIGS[name])
+                line["draft_loop"][name] = dl.timed(2, 3)
+                dl.sess.close()
+                del dl
+            line["configs"] = {}
+            for name in EXTRA_CONFIGS:
+                torch.cuda.empty_cache()
+                line["configs"][name] = extra_config(W.CONFIGS[name], pk, local, args.cpu_seconds)
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()

@@ -63,6 +63,9 @@ extern "C" {
 #define ASR_ST_WAIT_TIMEOUT 8   /* a bounded pipeline wait gave up; results of that call are invalid */
 #define ASR_ST_NOT_READY 16     /* an utterance slot without an encoder cache or prefill */
 #define ASR_ST_BAD_TREE 32      /* tree verify: a node's parent outside [0, node) */
+#define ASR_ST_BOUNDS 64        /* bounds-check mode (environment ASRSPEC_CHECK=1 at create): a kernel
+                                   found an index derived from device data out of range and skipped
+                                   that access; results of that call are invalid */
 
 typedef struct asr_spec* asr_spec_handle;
 
@@ -324,8 +327,15 @@ int asr_spec_timeline_read(asr_spec_handle h, uint64_t* ns, int32_t* kind, int32
  * the wait on the previous launch, input rows ready, weights landed,
  * projection reduced, exchange landed, attention done, exit, first K/V chunk
  * landed, first chunk combined, merge inputs landed, (unused) (0 where a
- * launch has no such phase); verify then launches directly (no graph).
- * ASR_E_INVAL when the model has no few-row layers.
+ * launch has no such phase); verify then launches directly (no graph).  A
+ * verify of more rows records its 6 L tensor-core projections instead (in
+ * layer order: QKV, self out, cross query, cross out, MLP up, MLP down), for
+ * their first 320 CTAs: 0 entry, 1 set-up done, 2 first k-block landed,
+ * 3 MMAs done, 4 exit, 5 K-split partial staged (one CTA per tile: tile
+ * staged in shared memory), 6 partials landed (staging barrier passed),
+ * 7 reduction done (rows written), 8 past the wait on the previous launch,
+ * 9 last k-block issued, 10 epilogue operands loaded, 11 first rows written
+ * (many-row kernel).  ASR_E_INVAL for an fp32 model.
  * asr_spec_fewrow_trace_read: synchronise and copy the last traced call's
  * stamps, [n_launches][320 CTAs][12] words in launch order, up to `cap` words. */
 int asr_spec_fewrow_trace(asr_spec_handle h, int32_t enable);
@@ -349,8 +359,12 @@ int asr_spec_synth_drafts(asr_spec_handle h, const int32_t* truth, const int32_t
  * with K split inside a thread-block cluster and wide N tiles (impl 4), or
  * the SIMT GEMM (impl 1);
  * impl 3 runs the LM-head epilogue instead and writes C[n] = the index m of
- * the largest value of column n (lowest m on ties).  A, B bf16 row-major
- * device arrays, C fp32.  K % 64 == 0.  Synchronous. */
+ * the largest value of column n (lowest m on ties).  Impls 5 - 7 run the
+ * many-row kernel (one tile per SM; K split over a cluster pair from 48
+ * k-blocks in 7) with zero bias and write C transposed, [n][m]: 5 the query
+ * epilogue, 6 GELU (bf16 result widened to fp32), 7 the residual epilogue
+ * onto x = 0; M % 128 == 0.  A, B bf16 row-major device arrays, C fp32.
+ * K % 64 == 0.  Synchronous. */
 int asr_spec_test_gemm(int32_t impl, const void* A, const void* B, float* C, int32_t M, int32_t N,
                        int32_t K, void* stream);
 

@@ -20,7 +20,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libasrspec.so")
 ASR_OK = 0
 ERRORS = {-1: "ASR_E_INVAL", -2: "ASR_E_STATE", -3: "ASR_E_CAPACITY", -4: "ASR_E_OOM",
           -5: "ASR_E_CUDA", -6: "ASR_E_DEVICE"}
-ST_BAD_TOKEN, ST_BAD_LENS, ST_CAPACITY, ST_WAIT_TIMEOUT, ST_NOT_READY, ST_BAD_TREE = 1, 2, 4, 8, 16, 32
+ST_BAD_TOKEN, ST_BAD_LENS, ST_CAPACITY, ST_WAIT_TIMEOUT, ST_NOT_READY, ST_BAD_TREE, ST_BOUNDS = 1, 2, 4, 8, 16, 32, 64
 
 EXPORTED = [
     "asr_spec_create", "asr_spec_set_host_io", "asr_spec_encode_cache", "asr_spec_prefill",

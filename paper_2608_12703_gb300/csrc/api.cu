@@ -82,6 +82,10 @@ struct asr_spec {
   int* attn_tickets = nullptr;                       // [B_max * H], tensor-core attention merge
   CUtensorMap m_kself[2], m_vself[2], m_xkv[2];      // boxes of 128 and 256 rows
   std::map<std::pair<int, int>, CUtensorMap> bmaps;  // (buffer id, BN) -> map
+  std::map<int, CUtensorMap> xmaps;                   // BN -> map of the residual stream (fp32, box 128 x BN)
+  int n_sms = 0;
+  bool use_wide = true;   // many-row projections on the one-tile-per-SM kernel (ASRSPEC_WIDE=0: the split-K chain)
+  int wide_stages = 0;    // its stages per pipeline (ASRSPEC_WIDE_STAGES; 0 = as deep as shared memory allows)
 
   // profiling: CUDA events around each kernel class (direct launches only)
   bool prof = false;
@@ -262,12 +266,29 @@ const CUtensorMap* bmap(asr_spec* h, int id, const void* buf, int rows, int cols
   return &(h->bmaps[key] = m);
 }
 
+const CUtensorMap* xmap(asr_spec* h, int bn) {
+  auto it = h->xmaps.find(bn);
+  if (it != h->xmaps.end()) return &it->second;
+  CUtensorMap m;
+  if (!make_tmap_f32(&m, h->x, h->R_pad, h->d, 128, bn)) return nullptr;
+  return &(h->xmaps[bn] = m);
+}
+
+// The next launch's slot of the per-CTA phase trace, or null (tracing off or the buffer full).
+unsigned long long* trace_slot(asr_spec* h) {
+  if (!h->fr_trace_on || h->fr_trace_n >= 6 * h->L) return nullptr;
+  return h->fr_trace + (size_t)(h->fr_trace_n++) * FR_TRACE_CTAS * FR_TRACE_PHASES;
+}
+
 // One projection over the verify rows: out-features m (weights = A), rows n (activations = B).
 int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, const void* X, int x_id, int N,
               int mode, const Epi& epi_in) {
   Epi epi = epi_in;
   epi.M = M;
   epi.N = N;
+  epi.status = h->status;
+  if (mode == EPI_QKV) epi.b_max = h->Bmax;
+  if (mode != EPI_ARGMAX && !epi.trace) epi.trace = trace_slot(h);
   const int cls = mode == EPI_QKV     ? ASR_PROF_QKV
                   : mode == EPI_RESID ? ASR_PROF_RESID
                   : mode == EPI_Q     ? ASR_PROF_QUERY
@@ -276,6 +297,29 @@ int gemm_rows(asr_spec* h, const void* W, const CUtensorMap* mW, int M, int K, c
   Prof p(h, cls, 1);
   if (!h->bf16) {
     launch_gemm_simt(W, 0, X, 0, M, N, K, mode, epi, h->st);
+    return 0;
+  }
+  WideGemm w{};
+  if (N > 64 && h->use_wide && wide_pick(M, N, K, mode, h->n_sms, &w.bn, &w.split) &&
+      (mode != EPI_RESID || epi.x == h->x)) {
+    const CUtensorMap* mb = bmap(h, x_id, X, h->R_pad, K, w.bn);
+    const CUtensorMap* mx = mode == EPI_RESID ? xmap(h, w.bn) : mW;
+    if (!mb || !mx) return fail(h, ASR_E_CUDA, "tensor map encode failed");
+    w.mapA = *mW;
+    w.mapB = *mb;
+    w.mapX = *mx;
+    w.M = M;
+    w.N = N;
+    w.K = K;
+    w.pdl = h->use_pdl;
+    w.stages = h->wide_stages;
+    Tl t(h, ASR_TL_GEMM + mode + (epi.ln_part ? ASR_TL_LN_FUSED : 0));
+    epi.tl = h->tl_cur;
+    launch_gemm_wide(w, mode, epi, h->status, h->st);
+    if (epi.xg) {   // every tile wrote the statistics of its 128-feature slice
+      h->ln_c = 128;
+      h->ln_S = M / 128;
+    }
     return 0;
   }
   TcGemm g{};
@@ -413,11 +457,12 @@ int run_layers(asr_spec* h, int N) {
     Tl t(h, ASR_TL_EMBED);
     if (h->ln_fold) {   // the first LayerNorm's operand and statistics (one slice of d features)
       launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st, h->use_pdl, h->tl_cur,
-                   static_cast<__nv_bfloat16*>(h->xn), h->lw[0].ln1g, h->ln_part);
+                   static_cast<__nv_bfloat16*>(h->xn), h->lw[0].ln1g, h->ln_part, h->V, h->maxpos, h->status);
       h->ln_S = 1;
       h->ln_c = d;
     } else {
-      launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st, h->use_pdl, h->tl_cur);
+      launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, N, d, h->x, h->st, h->use_pdl, h->tl_cur, nullptr, nullptr,
+                   nullptr, h->V, h->maxpos, h->status);
     }
   }
   // a residual projection that also produces the next LayerNorm's folded operand
@@ -444,6 +489,7 @@ int run_layers(asr_spec* h, int N) {
                               EPI_QKV, e))
       return rc;
     AttnArgs a{};
+    a.status = h->status;
     a.q = h->q;
     a.kc = ks;
     a.vc = vs;
@@ -525,14 +571,10 @@ int run_layers_few(asr_spec* h) {
   {
     Prof p(h, ASR_PROF_OTHER, 1);
     Tl t(h, ASR_TL_EMBED);
-    launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, std::min(N, VF_ROWS), d, h->x, h->st, h->use_pdl, h->tl_cur);
+    launch_embed(h->w_tok, h->w_pos, h->bf16, h->plan, std::min(N, VF_ROWS), d, h->x, h->st, h->use_pdl, h->tl_cur,
+                 nullptr, nullptr, nullptr, h->V, h->maxpos, h->status);
   }
   auto bf = [](void* p) { return static_cast<const __nv_bfloat16*>(p); };
-  h->fr_trace_n = 0;
-  auto trace_slot = [&]() -> unsigned long long* {
-    if (!h->fr_trace_on) return nullptr;
-    return h->fr_trace + (size_t)(h->fr_trace_n++) * FR_TRACE_CTAS * FR_TRACE_PHASES;
-  };
   for (int l = 0; l < h->L; ++l) {
     LayerW& w = h->lw[l];
     FrHead hd{};
@@ -563,7 +605,7 @@ int run_layers_few(asr_spec* h) {
       Prof p(h, ASR_PROF_QKV_SELF, 1);
       Tl t(h, ASR_TL_QKV_SELF);
       hs.tl = h->tl_cur;
-      hs.trace = trace_slot();
+      hs.trace = trace_slot(h);
       CK(launch_fr_self(&h->m_kself[0], &h->m_vself[0], hs, h->st, h->use_pdl));
     }
     FrGemv g{};
@@ -583,7 +625,7 @@ int run_layers_few(asr_spec* h) {
       Prof p(h, ASR_PROF_RESID, 1);
       Tl t(h, ASR_TL_GEMM + EPI_RESID);
       go.tl = h->tl_cur;
-      go.trace = trace_slot();
+      go.trace = trace_slot(h);
       CK(launch_fr_gemv(go, FR_RESID, 1, g_o, d, h->st, h->use_pdl));
     }
     // LayerNorm 2 -> cross query -> cross-attention
@@ -603,7 +645,7 @@ int run_layers_few(asr_spec* h) {
       Prof p(h, ASR_PROF_QUERY_CROSS, 1);
       Tl t(h, ASR_TL_QUERY_CROSS);
       hc.tl = h->tl_cur;
-      hc.trace = trace_slot();
+      hc.trace = trace_slot(h);
       CK(launch_fr_cross(&h->m_xkv[0], hc, h->st, h->use_pdl));
     }
     // cross-attention output projection + residual
@@ -614,7 +656,7 @@ int run_layers_few(asr_spec* h) {
       Prof p(h, ASR_PROF_RESID, 1);
       Tl t(h, ASR_TL_GEMM + EPI_RESID);
       gc.tl = h->tl_cur;
-      gc.trace = trace_slot();
+      gc.trace = trace_slot(h);
       CK(launch_fr_gemv(gc, FR_RESID, 1, g_o, d, h->st, h->use_pdl));
     }
     // LayerNorm 3 -> MLP up + GELU
@@ -631,7 +673,7 @@ int run_layers_few(asr_spec* h) {
       Prof p(h, ASR_PROF_UP, 1);
       Tl t(h, ASR_TL_GEMM + EPI_GELU);
       gu.tl = h->tl_cur;
-      gu.trace = trace_slot();
+      gu.trace = trace_slot(h);
       CK(launch_fr_gemv(gu, FR_GELU, 1, g_f, d, h->st, h->use_pdl));
     }
     // MLP down + residual (K split over a cluster of F / d CTAs)
@@ -646,7 +688,7 @@ int run_layers_few(asr_spec* h) {
       Prof p(h, ASR_PROF_RESID, 1);
       Tl t(h, ASR_TL_GEMM + EPI_RESID);
       gd.tl = h->tl_cur;
-      gd.trace = trace_slot();
+      gd.trace = trace_slot(h);
       CK(launch_fr_gemv(gd, FR_RESID, KS, g_d, d, h->st, h->use_pdl));
     }
     if (int rc = tap_copy(h, l, VF_ROWS)) return rc;
@@ -673,7 +715,12 @@ int draft_block(asr_spec* h, const RowPlan& plan, int rows, bool lm) {
   base.max_pos = h->maxpos;
   base.n_heads = h->H;
   DraftArgs A{};
+  A.B = h->B;
   A.d = d;
+  A.vocab = h->V;
+  A.max_pos = h->maxpos;
+  A.r_max = h->R_pad;
+  A.status = h->status;
   A.plan = plan;
   Epi e = base;
   e.bias = w.b_in;
@@ -692,6 +739,7 @@ int draft_block(asr_spec* h, const RowPlan& plan, int rows, bool lm) {
   at.row_lo = h->d_row_lo;
   at.row_hi = h->d_row_hi;
   at.out = static_cast<__nv_bfloat16*>(h->d_att);
+  at.status = h->status;
   // self-attention block
   ln(w.ln1g, w.ln1b, h->d_xn);
   e = base;
@@ -765,6 +813,7 @@ int copy_out(asr_spec* h, int32_t* dst, const int* src, size_t n) {
 // draft/lens buffers and writes the internal output block.
 int enqueue_verify(asr_spec* h, int k) {
   const int B = h->B;
+  h->fr_trace_n = 0;   // the phase trace (when on) holds this call's launches
   {
     Prof p(h, ASR_PROF_OTHER, 1);
     Tl t(h, ASR_TL_PLAN);
@@ -837,7 +886,7 @@ int enqueue_verify(asr_spec* h, int k) {
   if (h->cur_tree) {   // the accepted path's K/V to consecutive positions
     Prof p2(h, ASR_PROF_OTHER, 1);
     launch_tree_commit(h->path_buf, k, h->out4, h->kv_len, B, h->L, h->H, h->maxpos, h->Bmax, h->kself, h->vself,
-                       (int)h->es, h->st);
+                       (int)h->es, h->status, h->st);
   }
   return 0;
 }
@@ -863,6 +912,24 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
   h->Tmax = dims->max_enc;
   h->anchor = dims->anchor_layer >= 0 ? dims->anchor_layer : (3 * h->L) / 4;
   h->bf16 = dims->dtype == 1;
+  {
+    int dev = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&h->n_sms, cudaDevAttrMultiProcessorCount, dev);
+  }
+  if (const char* e = std::getenv("ASRSPEC_WIDE")) h->use_wide = std::atoi(e) != 0;
+  if (const char* e = std::getenv("ASRSPEC_WIDE_STAGES")) h->wide_stages = std::max(0, std::atoi(e));
+  {   // bounds-check mode: process-wide (each kernel module's constant), set by every create
+    const char* e = std::getenv("ASRSPEC_CHECK");
+    const int on = e && std::atoi(e) != 0;
+    set_check_gemm_tc(on);
+    set_check_gemm_simt(on);
+    set_check_gemm_wide(on);
+    set_check_rows(on);
+    set_check_attention(on);
+    set_check_attention_tc(on);
+    set_check_fewrow(on);
+    set_check_draft(on);
+  }
   if (const char* e = std::getenv("ASRSPEC_PDL")) h->use_pdl = std::atoi(e) != 0;
   if (const char* e = std::getenv("ASRSPEC_WIDE_BN")) {
     const int v = std::atoi(e);
@@ -1144,6 +1211,7 @@ int asr_spec_encode_cache(asr_spec_handle h, int32_t B, const void* enc_states, 
   e.t_max = t_max;
   e.max_enc = h->Tmax;
   e.b_max = h->Bmax;
+  e.status = h->status;
   const int M = B * t_max, N = h->L * 2 * d;
   e.M = M;
   e.N = N;
@@ -1213,6 +1281,10 @@ int asr_spec_prefill(asr_spec_handle h, const int32_t* prompt, int32_t P0) {
       DraftArgs A{};
       A.B = h->B;
       A.d = h->d;
+      A.vocab = h->V;
+      A.max_pos = h->maxpos;
+      A.r_max = h->R_pad;
+      A.status = h->status;
       A.enc_len = h->enc_len;
       A.taps = h->d_taps;
       A.last_tap = h->d_last_tap;
@@ -1477,6 +1549,7 @@ int asr_spec_draft_propose(asr_spec_handle h, int32_t k, int32_t window, const i
   A.win_kind = window;
   A.vocab = h->V;
   A.max_pos = h->maxpos;
+  A.r_max = h->R_pad;
   A.status = h->status;
   A.after_verify = h->d_after_verify ? 1 : 0;
   A.kv_len = h->kv_len;
@@ -1619,7 +1692,7 @@ int asr_spec_timeline_read(asr_spec_handle h, uint64_t* ns, int32_t* kind, int32
 
 int asr_spec_fewrow_trace(asr_spec_handle h, int32_t enable) {
   if (!h) return ASR_E_INVAL;
-  if (enable && h->fr_C == 0) return fail(h, ASR_E_INVAL, "the few-row layers are not available for this model");
+  if (enable && !h->bf16) return fail(h, ASR_E_INVAL, "the phase trace needs a bf16 model");
   if (enable && !h->fr_trace) {
     const size_t n = (size_t)6 * h->L * FR_TRACE_CTAS * FR_TRACE_PHASES;
     int rc = dalloc(h, &h->fr_trace, n * sizeof(unsigned long long));
@@ -1763,6 +1836,57 @@ int asr_spec_test_gemm(int32_t impl, const void* A, const void* B, float* C, int
     CK(cudaMemcpy(C, idx.data(), (size_t)N * 4, cudaMemcpyHostToDevice));
     cudaFree(keys);
     cudaFree(status);
+  } else if (impl >= 5 && impl <= 7) {
+    // the many-row kernel: 5 = query epilogue, 6 = GELU (bf16 out), 7 = residual (onto x = 0);
+    // zero bias, outputs [N][M]
+    const int mode = impl == 5 ? EPI_Q : impl == 6 ? EPI_GELU : EPI_RESID;
+    int sms = 0, dev = 0;
+    CK(cudaGetDevice(&dev));
+    CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    WideGemm w{};
+    if (!wide_pick(M, N, K, mode, sms, &w.bn, &w.split)) return ASR_E_INVAL;
+    if (!make_tmap_bf16(&w.mapA, A, M, K, 128) || !make_tmap_bf16(&w.mapB, B, N, K, w.bn)) return ASR_E_INVAL;
+    w.mapX = w.mapA;
+    if (mode == EPI_RESID && !make_tmap_f32(&w.mapX, C, N, M, 128, w.bn)) return ASR_E_INVAL;
+    w.M = M;
+    w.N = N;
+    w.K = K;
+    float* bias = nullptr;
+    int* status = nullptr;
+    __nv_bfloat16* act = nullptr;
+    CK(cudaMalloc(&bias, (size_t)M * 4));
+    CK(cudaMalloc(&status, 4));
+    CK(cudaMemsetAsync(bias, 0, (size_t)M * 4, st));
+    CK(cudaMemsetAsync(status, 0, 4, st));
+    e.d = M;
+    e.bias = bias;
+    if (mode == EPI_GELU) {
+      CK(cudaMalloc(&act, (size_t)M * N * 2));
+      e.act = act;
+      e.act_bf16 = 1;
+    } else if (mode == EPI_RESID) {
+      CK(cudaMemsetAsync(C, 0, (size_t)M * N * 4, st));
+      e.x = C;
+    }
+    launch_gemm_wide(w, mode, e, status, st);
+    CK(cudaGetLastError());
+    CK(cudaStreamSynchronize(st));
+    if (mode == EPI_GELU) {   // bf16 -> fp32 through the host
+      std::vector<uint16_t> hb((size_t)M * N);
+      std::vector<float> hf((size_t)M * N);
+      CK(cudaMemcpy(hb.data(), act, hb.size() * 2, cudaMemcpyDeviceToHost));
+      for (size_t i = 0; i < hb.size(); ++i) {
+        const uint32_t u = (uint32_t)hb[i] << 16;
+        std::memcpy(&hf[i], &u, 4);
+      }
+      CK(cudaMemcpy(C, hf.data(), hf.size() * 4, cudaMemcpyHostToDevice));
+      cudaFree(act);
+    }
+    int hs = 0;
+    CK(cudaMemcpy(&hs, status, 4, cudaMemcpyDeviceToHost));
+    cudaFree(bias);
+    cudaFree(status);
+    if (hs) return ASR_E_DEVICE;
   } else {
     TcGemm g{};
     g.bn = impl == 4 && N > 64 ? tc_pick_bn_wide(N) : tc_pick_bn(N);

@@ -21,6 +21,8 @@
 
 namespace asrspec {
 
+ASRSPEC_CHECK_SETTER(set_check_attention)
+
 constexpr float ATTN_SCALE = 0.125f;  // 1 / sqrt(64)
 
 // q . k over 64 dims, visiting the 32 element pairs starting at pair (j mod 32):
@@ -55,6 +57,7 @@ __global__ void __launch_bounds__(ATTN_THREADS) attn_chunk_kernel(AttnArgs a) {
   if (nr == 0) return;
   const int row0 = a.plan.row_start[b];
   const int n_keys = a.causal ? a.kv_len[b] + nr : a.enc_len[b];
+  if (bounds_bad(a.status, n_keys > a.t_alloc || n_keys > a.n_chunks * a.chunk)) return;
   const int key0 = chunk * CHUNK;
   if (key0 >= n_keys) return;
   const int nk = min(CHUNK, n_keys - key0);
@@ -129,6 +132,7 @@ __global__ void attn_merge_kernel(AttnArgs a, int chunk_len) {
   if (i >= nr) return;
   const int r = a.plan.row_start[b] + i;
   const int n_keys = a.causal ? a.kv_len[b] + nr : a.enc_len[b];
+  if (bounds_bad(a.status, n_keys > a.t_alloc || n_keys > a.n_chunks * chunk_len)) return;
   const int nc = (n_keys + chunk_len - 1) / chunk_len;
   const float* part = a.part + ((size_t)b * a.H + h) * a.n_chunks * a.k1 * 66 + (size_t)i * 66;
   const size_t cstride = (size_t)a.k1 * 66;
@@ -420,7 +424,7 @@ void launch_accept_anchor(const AcceptAnchorArgs& A, cudaStream_t st) {
 __global__ void __launch_bounds__(256)
 tree_commit_kernel(const int* __restrict__ path, int k, const int* __restrict__ accepted,
                    const int* __restrict__ kv_len, int B, int L, int H, int max_pos, int b_max, uint32_t* kself,
-                   uint32_t* vself) {
+                   uint32_t* vself, int* status) {
   const int w = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
   if (w >= B * L * H) return;
   const int b = w / (L * H), rem = w - b * L * H, l = rem / H, h = rem - l * H;
@@ -432,6 +436,7 @@ tree_commit_kernel(const int* __restrict__ path, int k, const int* __restrict__ 
   uint32_t* V = vself + head * 32;
   for (int j = 0; j < n; ++j) {
     const int src = path[(size_t)b * k + j];
+    if (bounds_bad(status, P < 0 || src < 1 || P + max(src, j + 1) >= max_pos)) return;
     if (src == j + 1) continue;
     K[(size_t)(P + j + 1) * 32 + lane] = K[(size_t)(P + src) * 32 + lane];
     V[(size_t)(P + j + 1) * 32 + lane] = V[(size_t)(P + src) * 32 + lane];
@@ -439,11 +444,12 @@ tree_commit_kernel(const int* __restrict__ path, int k, const int* __restrict__ 
 }
 
 void launch_tree_commit(const int* path, int k, const int* accepted, const int* kv_len, int B, int L, int H,
-                        int max_pos, int b_max, void* kself, void* vself, int es, cudaStream_t st) {
+                        int max_pos, int b_max, void* kself, void* vself, int es, int* status, cudaStream_t st) {
   if (es != 2) return;   // tree verify runs on bf16 caches only (the ABI refuses others)
   const long long threads = 32ll * B * L * H;
   tree_commit_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, st>>>(
-      path, k, accepted, kv_len, B, L, H, max_pos, b_max, static_cast<uint32_t*>(kself), static_cast<uint32_t*>(vself));
+      path, k, accepted, kv_len, B, L, H, max_pos, b_max, static_cast<uint32_t*>(kself), static_cast<uint32_t*>(vself),
+      status);
 }
 
 }  // namespace asrspec

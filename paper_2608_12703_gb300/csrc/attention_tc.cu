@@ -29,6 +29,8 @@
 
 namespace asrspec {
 
+ASRSPEC_CHECK_SETTER(set_check_attention_tc)
+
 constexpr int TCA_THREADS = 128;
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -103,6 +105,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__
   }
   const int row0 = a.plan.row_start[b];
   const int n_keys = a.causal ? a.kv_len[b] + nr : a.enc_len[b];
+  if (bounds_bad(status, n_keys > a.t_alloc || nr > a.rows_max)) {   // uniform over the cluster
+    pdl_wait();
+    return;
+  }
   const int nc = (n_keys + TCA_CH - 1) / TCA_CH;
   const int n_iter = split < nc ? (nc - split + S - 1) / S : 0;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;

@@ -25,9 +25,28 @@ enum StatusBits : int {
   ST_WAIT_TIMEOUT = 1 << 3,  // a bounded wait gave up (mbarrier / pipeline)
   ST_NOT_READY = 1 << 4,     // verify on an utterance without encoder cache
   ST_BAD_TREE = 1 << 5,      // tree verify: a parent outside [0, node)
+  ST_BOUNDS = 1 << 6,        // bounds-check mode: an index derived from device data was out of range
 };
 
 __device__ __forceinline__ void set_status(int* status, int bits) { atomicOr(status, bits); }
+
+// Bounds-check mode (ASRSPEC_CHECK=1 when a handle is created): kernels
+// re-check, at the point of access, the indexes they derive from device data
+// (cache slots from row plans, token and position ids, key ranges, row
+// sources); a failed check sets ST_BOUNDS and the access is skipped instead of
+// reading or writing out of range.  Off, each check is one uniform branch on a
+// constant.  The flag lives in each translation unit's constant bank and is
+// set through that unit's set_check_* function.
+static __constant__ int c_check_mode;
+__device__ __forceinline__ bool bounds_bad(int* status, bool bad) {
+  if (c_check_mode && bad) {
+    if (status) atomicOr(status, ST_BOUNDS);
+    return true;
+  }
+  return false;
+}
+#define ASRSPEC_CHECK_SETTER(name) \
+  void name(int on) { cudaMemcpyToSymbol(c_check_mode, &on, sizeof(int)); }
 
 // ---------------------------------------------------------------------------
 // Numeric helpers

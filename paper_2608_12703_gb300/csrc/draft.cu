@@ -20,6 +20,8 @@
 
 namespace asrspec {
 
+ASRSPEC_CHECK_SETTER(set_check_draft)
+
 namespace {
 
 constexpr int DP_T = 256;                  // threads of the one-CTA plan kernels (B <= 256 per pass)
@@ -177,6 +179,9 @@ __global__ void draft_gather_kernel(DraftArgs A) {
   for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < R * per; e += gridDim.x * blockDim.x) {
     const int r = e / per, c = 2 * (e - r * per);   // column c, c + 1 of [4 d]
     const int src = A.row_src[r];
+    if (bounds_bad(A.status, src >= A.r_max || (src <= -3 && -3 - src >= A.r_max) || r >= A.r_max ||
+                                 (src == -1 && (A.plan.row_b[r] < 0 || A.plan.row_b[r] >= A.B))))
+      continue;
     float2 v;
     if (src >= 0) v = *reinterpret_cast<const float2*>(A.taps + (size_t)src * 4 * d + c);
     else if (src == -1) v = *reinterpret_cast<const float2*>(A.last_tap + (size_t)A.plan.row_b[r] * 4 * d + c);
@@ -198,6 +203,7 @@ __global__ void draft_prefill_gather_kernel(DraftArgs A) {
   for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < R * per; e += gridDim.x * blockDim.x) {
     const int r = e / per, c = 2 * (e - r * per);
     const int b = A.plan.row_b[r], p = A.plan.row_pos[r];
+    if (bounds_bad(A.status, r >= A.r_max || b < 0 || b >= A.B)) continue;
     float2 v = make_float2(0.f, 0.f);
     if (p > 0) v = A.plan.row_i[r] > 0 ? *reinterpret_cast<const float2*>(A.taps + (size_t)(r - 1) * 4 * d + c)
                                       : *reinterpret_cast<const float2*>(A.last_tap + (size_t)b * 4 * d + c);
@@ -226,6 +232,8 @@ __global__ void draft_embed_kernel(DraftArgs A, const __nv_bfloat16* tok_emb, co
   const int R = *A.plan.n_rows, d = A.d;
   for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < R * d; e += gridDim.x * blockDim.x) {
     const int r = e / d, c = e - r * d;
+    const int tok = A.plan.row_tok[r], pos = A.plan.row_epos[r];
+    if (bounds_bad(A.status, tok < 0 || tok >= A.vocab || pos < 0 || pos >= A.max_pos || r >= A.r_max)) continue;
     x[e] += __bfloat162float(tok_emb[(size_t)A.plan.row_tok[r] * d + c]) +
             __bfloat162float(pos_emb[(size_t)A.plan.row_epos[r] * d + c]);
   }
@@ -271,6 +279,7 @@ __global__ void __launch_bounds__(128) draft_attn_kernel(DraftAttn a) {
     const int r = r0 + i;
     const int lo = a.causal ? 0 : a.row_lo[r];
     const int hi = a.causal ? a.plan.row_pos[r] + 1 : a.row_hi[r];
+    if (bounds_bad(a.status, lo < 0 || hi > a.t_alloc || hi <= lo)) continue;   // uniform over the CTA
     if (tid < 64) s_q[tid] = a.q[(size_t)r * a.d + hh * 64 + tid] * 0.125f;
     __syncthreads();
     float m = -INFINITY;

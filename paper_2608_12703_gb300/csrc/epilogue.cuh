@@ -48,6 +48,8 @@ struct Epi {
   int b_max = 0;
   // LM head argmax
   unsigned long long* row_key = nullptr;
+  // device status word, for the bounds-check mode (ST_BOUNDS), or null
+  int* status = nullptr;
   // LayerNorm folded into the GEMM (consumer).  The B operand is bf16(g * x)
   // and y = rstd_n (acc - mu_n c1_m) + c2_m (+ bias), with c1 = W g, c2 = W b
   // and the row statistics combined from ln_S slices of ln_c features each:
@@ -67,11 +69,17 @@ struct Epi {
   // > 0: one-dimensional grid walked in bands of group_m M tiles, each band
   // sweeping every N tile (L2 reuse when both operands exceed the L2)
   int group_m = 0;
-  // optional phase timestamps (ns, %globaltimer) per CTA: [CTA][8]
-  // (entry, set-up done, first stage full, MMAs done, end; cluster split:
-  // partials staged, first cluster barrier passed, reduction done)
+  // optional phase timestamps (ns, %globaltimer) per CTA: [CTA][FR_TRACE_PHASES]
+  // for the first FR_TRACE_CTAS CTAs (0 entry, 1 set-up done, 2 first stage
+  // full, 3 MMAs done, 4 end; cluster split: 5 partials staged, 6 exchange
+  // landed, 7 reduction done)
   unsigned long long* trace = nullptr;
 };
+
+// Bounds-check mode: a self-cache slot (utterance rb, position rp) outside the cache.
+__device__ __forceinline__ bool qkv_slot_bad(const Epi& e, int rb, int rp) {
+  return bounds_bad(e.status, rp < 0 || rp >= e.max_pos || rb < 0 || (e.b_max > 0 && rb >= e.b_max));
+}
 
 template <typename T>
 __device__ __forceinline__ void store_as(void* base, size_t idx, float v) {
@@ -103,6 +111,7 @@ __device__ __forceinline__ void epi_apply(const Epi& e, int m, int n, float acc)
       int which = (m - e.d) / e.d;            // 0 = k, 1 = v
       int f = (m - e.d) - which * e.d;
       int h = f >> 6, c = f & 63;
+      if (qkv_slot_bad(e, e.row_b[n], e.row_pos[n])) return;
       size_t idx = (((size_t)e.row_b[n] * e.n_heads + h) * e.max_pos + e.row_pos[n]) * 64 + c;
       void* base = which == 0 ? e.kcache : e.vcache;
       if (e.kv_bf16) store_as<__nv_bfloat16>(base, idx, v);
@@ -110,6 +119,7 @@ __device__ __forceinline__ void epi_apply(const Epi& e, int m, int n, float acc)
     }
   } else if constexpr (MODE == EPI_CROSSKV) {
     int b = m / e.t_max, t = m - b * e.t_max;
+    if (bounds_bad(e.status, b >= e.b_max || t >= e.max_enc)) return;
     if (t >= e.enc_len[b]) return;
     int two_d = 2 * e.d;
     int l = n / two_d;
@@ -134,6 +144,7 @@ struct EpiPre {
   float bias[U];
   float old[U];   // EPI_RESID: x before the update
   int rb[U], rp[U];   // EPI_QKV: utterance and position of the row
+  bool bad[U];        // EPI_QKV: the slot failed the bounds-check mode
   float c1[U], c2[U];   // folded LayerNorm (consumer)
   float gain[U];        // next LayerNorm's gain (EPI_RESID producer)
 };
@@ -149,6 +160,7 @@ __device__ __forceinline__ void epi_load(const Epi& e, const int* m, const int* 
     if constexpr (MODE == EPI_QKV) {
       p.rb[u] = ok[u] && m[u] >= e.d ? e.row_b[n[u]] : 0;
       p.rp[u] = ok[u] && m[u] >= e.d ? e.row_pos[n[u]] : 0;
+      p.bad[u] = ok[u] && m[u] >= e.d && qkv_slot_bad(e, p.rb[u], p.rp[u]);
     }
     if constexpr (MODE != EPI_RESID && MODE != EPI_CROSSKV) {
       p.c1[u] = ok[u] && e.ln_part ? __ldg(e.ln_c1 + m[u]) : 0.f;
@@ -170,7 +182,7 @@ __device__ __forceinline__ void epi_store(const Epi& e, const int* m, const int*
       const float val = v[u] + p.bias[u];
       if (m[u] < e.d) {
         e.out_f32[(size_t)n[u] * e.d + m[u]] = val;
-      } else {
+      } else if (!p.bad[u]) {
         const int which = (m[u] - e.d) / e.d;
         const int f = (m[u] - e.d) - which * e.d;
         const size_t idx = (((size_t)p.rb[u] * e.n_heads + (f >> 6)) * e.max_pos + p.rp[u]) * 64 + (f & 63);
@@ -256,6 +268,7 @@ __device__ __forceinline__ void epi_rows(const Epi& e, const float* stg, int lds
       if constexpr (MODE == EPI_QKV) {
         rb[r] = ok[r] && kind ? e.row_b[n] : 0;
         rp[r] = ok[r] && kind ? e.row_pos[n] : 0;
+        if (ok[r] && kind && qkv_slot_bad(e, rb[r], rp[r])) ok[r] = false;
       }
     }
 #pragma unroll

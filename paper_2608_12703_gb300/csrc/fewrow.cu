@@ -35,6 +35,8 @@
 
 namespace asrspec {
 
+ASRSPEC_CHECK_SETTER(set_check_fewrow)
+
 namespace {
 
 constexpr int FR_T = 256;               // threads (8 warps)
@@ -475,7 +477,9 @@ __global__ void __launch_bounds__(FR_T) fr_self_kernel(const __grid_constant__ C
     const int lt = lt0 + pr.i, which = lt >> 3, m = 8 * gtile(lt) + 2 * pr.n2;
     const float y0 = pr.v0 + __ldg(A.bias + m), y1 = pr.v1 + __ldg(A.bias + m + 1);
     const uint32_t v = which == 0 ? bf2_bits(y0 * 0.125f, y1 * 0.125f) : bf2_bits(y0, y1);
-    if (which > 0 && pr.r < R) {
+    if (which > 0 && pr.r < R &&
+        !bounds_bad(A.status, A.plan.row_b[pr.r] < 0 || A.plan.row_b[pr.r] >= A.B || s_pos[pr.r] < 0 ||
+                                  s_pos[pr.r] >= A.max_pos)) {
       const int f = m - which * d;
       const size_t slot = (((size_t)A.plan.row_b[pr.r] * H + hh) * A.max_pos + s_pos[pr.r]) * 64 + (f & 63);
       *reinterpret_cast<uint32_t*>((which == 1 ? A.ks : A.vs) + slot) = v;

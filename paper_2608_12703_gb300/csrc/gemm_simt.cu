@@ -8,6 +8,8 @@
 
 namespace asrspec {
 
+ASRSPEC_CHECK_SETTER(set_check_gemm_simt)
+
 constexpr int SG_BM = 64, SG_BN = 64, SG_BK = 16;
 
 template <typename TA, typename TB, int MODE>

@@ -28,6 +28,8 @@
 
 namespace asrspec {
 
+ASRSPEC_CHECK_SETTER(set_check_gemm_tc)
+
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;
 
@@ -90,8 +92,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
   }
   const int m0 = tile_m * TC_BM, n0 = tile_n * BN;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  unsigned long long* tr = epi.trace ? epi.trace + 8ull * (blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z))
-                                     : nullptr;
+  const unsigned cta_id = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z);
+  unsigned long long* tr =
+      epi.trace && cta_id < FR_TRACE_CTAS ? epi.trace + (unsigned long long)FR_TRACE_PHASES * cta_id : nullptr;
   if (tr && threadIdx.x == 0) tr[0] = global_ns();
   tl_mark(epi.tl, TL_ENTRY);
   const int n_valid = epi.n_valid ? *epi.n_valid : epi.N;
@@ -156,6 +159,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
     }
     pdl_wait();
     tl_mark(epi.tl, TL_WORK);
+    if (tr) tr[8] = global_ns();
     for (int i = 0; i < first; ++i) tma_load_2d(sB + i * C::B_BYTES, &mapB, &full[i], (kb0 + i) * TC_BK, n0);
     pdl_launch();
     int issued = first;
@@ -168,6 +172,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
       tma_load_2d(sB + s * C::B_BYTES, &mapB, &full[s], (kb0 + i) * TC_BK, n0);
       issued = i + 1;
     }
+    if (tr) tr[9] = global_ns();
     // Drain: every issued copy has landed before this CTA can exit.
     for (int i = issued - C::STAGES > 0 ? issued - C::STAGES : 0; i < issued; ++i)
       mbar_wait(&full[i % C::STAGES], (i / C::STAGES) & 1, status);
@@ -285,9 +290,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__
 #pragma unroll
       for (int i = 0; i < 16; ++i) stg[(c0 + i) * LDS + ml] = v[i];
     }
+    if (tr && threadIdx.x == 0) tr[5] = global_ns();
     __syncthreads();
+    if (tr && threadIdx.x == 0) tr[6] = global_ns();
     const int rows = n_valid - n0 < BN ? n_valid - n0 : BN;
     epi_rows<MODE>(epi, stg, LDS, m0 + 4 * lane, 4 * lane, n0, warp, rows, ln_mu, ln_rs);
+    if (tr && threadIdx.x == 0) tr[7] = global_ns();
   } else if (splits == 1) {
     // encoder-cache build: this thread's frame (utterance fb, frame ft) and whether it is real
     const int fb = MODE == EPI_CROSSKV ? m / epi.t_max : 0, ft = MODE == EPI_CROSSKV ? m - fb * epi.t_max : 0;
@@ -643,6 +651,21 @@ bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool make_tmap_f32(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
+                   uint32_t box_rows) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) || (cols * 4) % 16 || (box_cols * 4) % 16) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 4};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }

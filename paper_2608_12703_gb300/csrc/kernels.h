@@ -29,6 +29,23 @@ int tc_pick_bn(int n_max);
 int tc_pick_bn_wide(int n);
 void launch_gemm_tc(const TcGemm& g, int mode, const Epi& epi, int* status, cudaStream_t st);
 size_t tc_smem_bytes(int bn);
+// 2-D fp32 tensor map over [rows][cols], no swizzle, box {box_cols, box_rows}.
+bool make_tmap_f32(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
+                   uint32_t box_rows);
+
+// Many-row projections (csrc/gemm_wide.cuh): one 128 x bn tile per CTA, about
+// one CTA per SM; modes QKV, Q, GELU, RESID (M % 128 == 0, K % 64 == 0).
+struct WideGemm {
+  CUtensorMap mapA;   // weights [M][K], box 64 x 128
+  CUtensorMap mapB;   // rows [R][K], box 64 x bn
+  CUtensorMap mapX;   // RESID: the residual stream [R][d] fp32, box 128 x bn (others: unused)
+  int M, N, K;
+  int bn, split;      // N tile (32 .. 256, RESID <= 128); 1, or 2 = K split over a cluster pair
+  int stages = 0;     // stages per pipeline, at least 2 (0: as deep as shared memory allows)
+  bool pdl = false;
+};
+bool wide_pick(int M, int N, int K, int mode, int sms, int* bn, int* split);
+void launch_gemm_wide(const WideGemm& g, int mode, const Epi& epi, int* status, cudaStream_t st);
 void configure_gemm_tc();
 void configure_attention();
 
@@ -72,8 +89,8 @@ void launch_plan_prefill_chunk(const int* prompt, int P0, int p0, int c, int B, 
 // xg / gain / st_part: the folded first LayerNorm's operand bf16(gain * x) [R][d]
 // and the rows' statistics (one slice of d features), or null.
 void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
-                  cudaStream_t st, bool pdl = false, unsigned long long* tl = nullptr, __nv_bfloat16* xg = nullptr,
-                  const float* gain = nullptr, float2* st_part = nullptr);
+                  cudaStream_t st, bool pdl, unsigned long long* tl, __nv_bfloat16* xg, const float* gain,
+                  float2* st_part, int vocab, int max_pos, int* status);
 // c1[m] = sum_k W[m][k] g[k], c2[m] = sum_k W[m][k] b[k] for a bf16 W [M][K].
 void launch_ln_fold(const void* W, const float* g, const float* b, int M, int K, float* c1, float* c2,
                     cudaStream_t st);
@@ -111,6 +128,7 @@ struct AttnArgs {
   bool pdl = false;        // programmatic dependent launch
   bool tree = false;       // self-attention of a tree verify: slots past kv_len visible by plan.row_mask
   unsigned long long* tl = nullptr;   // launch timeline slot (tl_mark), or null
+  int* status = nullptr;   // device status word (bounds-check mode)
 };
 void launch_attention(const AttnArgs& a, cudaStream_t st);
 void launch_attention_tc(const AttnArgs& a, int* status, cudaStream_t st);
@@ -145,7 +163,7 @@ void launch_accept_anchor(const AcceptAnchorArgs& a, cudaStream_t st);
 // the nodes' slots kv_len_old + path[j] to the positions kv_len_old + j + 1.
 // Reads the new kv_len and the accepted count (kv_len_old = kv_len - 1 - n).
 void launch_tree_commit(const int* path, int k, const int* accepted, const int* kv_len, int B, int L, int H,
-                        int max_pos, int b_max, void* kself, void* vself, int es, cudaStream_t st);
+                        int max_pos, int b_max, void* kself, void* vself, int es, int* status, cudaStream_t st);
 
 // ---- Few-row verify layers (csrc/fewrow.cu) ------------------------------------
 // A step of at most VF_ROWS rows runs each decoder layer as six launches:
@@ -221,7 +239,7 @@ cudaError_t launch_fr_cross(const CUtensorMap* xmap, const FrHead& a, cudaStream
 enum DraftWin : int { DRAFT_WIN_ANCHOR = 0, DRAFT_WIN_SHIFTED = 1, DRAFT_WIN_RANDOM = 2, DRAFT_WIN_NONE = 3 };
 struct DraftArgs {
   int B, d, k, k_verify, win_kind;
-  int vocab, max_pos;
+  int vocab, max_pos, r_max;   // token ids, positions, rows of the pass buffers
   int* status;               // device status word (ASR_ST_* bits)
   int after_verify;          // 1: a verification ran since the last round (catch-up rows)
   const int *kv_len, *pending, *enc_len, *total_len;
@@ -247,6 +265,7 @@ struct DraftAttn {
   RowPlan plan;
   const int *row_lo, *row_hi;
   __nv_bfloat16* out;        // [R][d]
+  int* status;               // device status word (bounds-check mode)
 };
 void launch_draft_round_plan(const DraftArgs& a, cudaStream_t st);
 void launch_draft_next_plan(const DraftArgs& a, int i, cudaStream_t st);
@@ -268,5 +287,15 @@ void launch_synth_drafts(const int* truth, const int* total_len, const int* repl
 void launch_mark_ready(const int* enc_len, int B, int t_max, int* ready, int* kv_len, int* pending, int* status,
                        cudaStream_t st);
 int attn_chunk_len(int kv_bf16);
+
+// Bounds-check mode switches, one per translation unit (see bounds_bad).
+void set_check_gemm_tc(int on);
+void set_check_gemm_simt(int on);
+void set_check_gemm_wide(int on);
+void set_check_rows(int on);
+void set_check_attention(int on);
+void set_check_attention_tc(int on);
+void set_check_fewrow(int on);
+void set_check_draft(int on);
 
 }  // namespace asrspec

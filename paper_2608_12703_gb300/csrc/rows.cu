@@ -5,6 +5,8 @@
 
 namespace asrspec {
 
+ASRSPEC_CHECK_SETTER(set_check_rows)
+
 constexpr int PLAN_THREADS = 1024;
 
 // Exclusive block scan of one int per thread (PLAN_THREADS threads).
@@ -186,7 +188,7 @@ template <typename T>
 __global__ void __launch_bounds__(128)
 embed_kernel(const T* __restrict__ tok_emb, const T* __restrict__ pos_emb, RowPlan plan, int d,
              float* __restrict__ x, __nv_bfloat16* __restrict__ xg, const float* __restrict__ gain,
-             float2* __restrict__ st_part, unsigned long long* tl) {
+             float2* __restrict__ st_part, unsigned long long* tl, int vocab, int max_pos, int* status) {
   __shared__ float red[4];
   tl_mark(tl, TL_ENTRY);
   pdl_wait();
@@ -195,6 +197,7 @@ embed_kernel(const T* __restrict__ tok_emb, const T* __restrict__ pos_emb, RowPl
   const int r = blockIdx.x;
   if (r >= *plan.n_rows) return;   // uniform over the CTA
   const int t = plan.row_tok[r], p = plan.row_epos[r];
+  if (bounds_bad(status, t < 0 || t >= vocab || p < 0 || p >= max_pos)) return;   // uniform over the CTA
   float v[16];
   float s = 0.f;
 #pragma unroll
@@ -258,14 +261,14 @@ void launch_ln_fold(const void* W, const float* g, const float* b, int M, int K,
 
 void launch_embed(const void* tok_emb, const void* pos_emb, int w_bf16, RowPlan plan, int R_max, int d, float* x,
                   cudaStream_t st, bool pdl, unsigned long long* tl, __nv_bfloat16* xg, const float* gain,
-                  float2* st_part) {
+                  float2* st_part, int vocab, int max_pos, int* status) {
   if (w_bf16)
     launch_ex(embed_kernel<__nv_bfloat16>, dim3(R_max), dim3(128), 0, st, pdl, 1,
               static_cast<const __nv_bfloat16*>(tok_emb), static_cast<const __nv_bfloat16*>(pos_emb), plan, d, x, xg,
-              gain, st_part, tl);
+              gain, st_part, tl, vocab, max_pos, status);
   else
     launch_ex(embed_kernel<float>, dim3(R_max), dim3(128), 0, st, pdl, 1, static_cast<const float*>(tok_emb),
-              static_cast<const float*>(pos_emb), plan, d, x, xg, gain, st_part, tl);
+              static_cast<const float*>(pos_emb), plan, d, x, xg, gain, st_part, tl, vocab, max_pos, status);
 }
 
 // LayerNorm for any d % 4 == 0: a sum pass, a centred sum-of-squares pass over the

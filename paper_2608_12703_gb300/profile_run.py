@@ -11,7 +11,8 @@ Options: --classes (CUDA-event time per kernel class), --timeline (the launch
 timeline per launch kind), --fewrow-trace (per-CTA phase stamps of the
 few-row launches), --tree-nodes N (tree verifies beside the linear one), --enc-len T
 (encoder memories of T frames), --batch-sweep 1,4,16,64 (verification cost and
-anchor-readout share against batch size).
+anchor-readout share against batch size), --gemm IMPL,M,N,K (one GEMM shape
+through the kernel test entry, for captures of a single kernel).
 
 Kernel launches per round (bf16 decoders): at most 9 rows (e.g. batch 1):
 2 + 6 per layer + 3 (few-row layers, final LayerNorm, LM head, accept);
@@ -98,6 +99,65 @@ def fewrow_trace_summary(tr):
     return "\n".join(lines)
 
 
+GEMM_KINDS = ["qkv", "self_out", "cross_query", "cross_out", "mlp_up", "mlp_down"]
+GEMM_PHASES = ["setup", "past_wait", "first_full", "loads_out", "mma_done", "staged", "landed", "epi_ready",
+               "first_rows", "reduced", "end"]
+
+
+def gemm_trace_summary(tr):
+    """Per many-row projection (averaged over layers): each phase's median and
+    maximum over CTAs, in us after the launch's first CTA entry (phases 1, 8,
+    2, 9, 3, 5, 6, 10, 11, 7, 4 of the GEMM's stamps)."""
+    tr = tr.astype(np.int64)
+    lines = [f"  GEMM trace: {tr.shape[0]} launches; us after the launch's first CTA entry, median / max over CTAs"]
+    lines.append("  " + f"{'kind':<12}{'CTAs':>6}" + "".join(f"{p:>16}" for p in GEMM_PHASES))
+    acc = {k: [] for k in GEMM_KINDS}
+    for i in range(tr.shape[0]):
+        cta = tr[i][:, 0] > 0
+        if not cta.any():
+            continue
+        t0 = tr[i][cta, 0].min()
+        with np.errstate(all="ignore"):
+            rel = np.where(tr[i][cta] > 0, (tr[i][cta] - t0) / 1e3, np.nan)
+        acc[GEMM_KINDS[i % 6]].append(rel)
+    import warnings
+    warnings.simplefilter("ignore", RuntimeWarning)
+    for k in GEMM_KINDS:
+        if not acc[k]:
+            continue
+        cols = [1, 8, 2, 9, 3, 5, 6, 10, 11, 7, 4]
+        med = np.nanmean([np.nanmedian(r, axis=0) for r in acc[k]], axis=0)
+        mx = np.nanmean([np.nanmax(r, axis=0) for r in acc[k]], axis=0)
+        cells = "".join(f"{med[c]:>8.2f}/{mx[c]:<7.2f}" if np.isfinite(med[c]) else f"{'-':>16}" for c in cols)
+        lines.append(f"  {k:<12}{acc[k][0].shape[0]:>6}{cells}")
+    return "\n".join(lines)
+
+
+def gemm_only(args):
+    """One GEMM shape through the kernel test entry, timed with CUDA events."""
+    import torch
+    from paper_2608_12703_gb300 import asrspec as A
+    from paper_2608_12703_gb300 import build as B
+    B.build()
+    impl, M, N, K = (int(x) for x in args.gemm.split(","))
+    g = torch.Generator(device="cpu").manual_seed(0)
+    a = (0.25 * torch.randn(M, K, generator=g)).to(torch.bfloat16).cuda()
+    b = torch.randn(N, K, generator=g).to(torch.bfloat16).cuda()
+    c = torch.empty((max(M, N), max(M, N)), device="cuda")
+    st = torch.cuda.current_stream()
+    us = []
+    for i in range(args.warmup + args.rounds):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        A.asr_spec_test_gemm(impl, a, b, c, M, N, K, st.cuda_stream)
+        e1.record(st)
+        torch.cuda.synchronize()
+        if i >= args.warmup:
+            us.append(e0.elapsed_time(e1) * 1e3)
+    print(f"gemm impl {impl} M {M} N {N} K {K}: us per call (with the entry's set-up) "
+          + " ".join(f"{u:.1f}" for u in us))
+
+
 def batch_sweep(batches, k, rounds, warmup):
     """Verification cost against batch size on the large decoder: the first B
     utterances of the 64-utterance workload (ragged encoder lengths), k drafts
@@ -162,7 +222,8 @@ def main():
     ap.add_argument("--timeline", action="store_true",
                     help="also record the launch timeline of the rounds (direct launches) and summarise it per kind")
     ap.add_argument("--fewrow-trace", action="store_true",
-                    help="also record the per-CTA phase stamps of one verify's few-row launches and summarise them")
+                    help="also record the per-CTA phase stamps of one verify's few-row launches (more rows: its "
+                         "tensor-core projections) and summarise them")
     ap.add_argument("--batch-sweep", default="",
                     help="comma-separated batch sizes: verification cost and anchor-readout share of the large "
                          "decoder at each (replaces the single-workload run)")
@@ -172,7 +233,12 @@ def main():
     ap.add_argument("--tree-nodes", type=int, default=0,
                     help="also time tree verifies of this many nodes per utterance (random trees whose first k "
                          "nodes form one branch) beside the linear verify")
+    ap.add_argument("--gemm", default="",
+                    help="IMPL,M,N,K: run only the GEMM test entry (asr_spec_test_gemm) with random bf16 operands, "
+                         "--warmup + --rounds times, and print the per-call time")
     args = ap.parse_args()
+    if args.gemm:
+        return gemm_only(args)
     if args.batch_sweep:
         from paper_2608_12703_gb300 import build as B
         B.build()
@@ -238,7 +304,10 @@ def main():
         sess.verify_device(drafts[0], lens, wl.k)
         tr = A.asr_spec_fewrow_trace_read(sess.h)
         A.asr_spec_fewrow_trace(sess.h, False)
-        print(fewrow_trace_summary(tr))
+        if dims.dtype == "bf16" and wl.batch * (wl.k + 1) > 9:
+            print(gemm_trace_summary(tr))
+        else:
+            print(fewrow_trace_summary(tr))
     if args.tree_nodes:
         n = args.tree_nodes
         trng = np.random.default_rng(9)

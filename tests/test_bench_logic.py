@@ -62,7 +62,14 @@ def test_tensor_bound_when_rows_exceed_the_balance():
     assert r["peak"] == PK["bf16_sus"]
 
 
-def test_attention_work_is_the_counted_kv_bytes():
+def test_attention_work_is_the_counted_kv_bytes(tmp_path, monkeypatch):
+    import paper_2608_12703_gb300.ncu_traffic as NT
+    monkeypatch.setattr(NT, "TRAFFIC_FILE", str(tmp_path / "traffic.json"))
+    csv_path = tmp_path / "raw.csv"
+    csv_path.write_text('"ID","Kernel Name","dram__bytes_read.sum","dram__bytes_write.sum"\n'
+                        '"","","Mbyte","Kbyte"\n'
+                        '"0","attn_tc_kernel<1>","330.5","7200"\n')
+    NT.record(str(csv_path), "attn_tc", "large-bf16-b64-k6", "cross_attn", "attn_tc", "profiles/x.md")
     dims = W.LARGE
     traffic = np.array([4, 3e8, 9e9, 1e8, 36, 0, 0, 0])
     tl = _timeline([(5, 0, 0, 50000)])
@@ -70,7 +77,7 @@ def test_attention_work_is_the_counted_kv_bytes():
     r = bench.roofline("large-bf16-b64-k6", dims, tl, ms, launches, traffic, PK)
     assert r["kernel"] == "cross_attn" and r["bound"] == "hbm"
     assert r["achieved"] == pytest.approx(9e9 / 2e-3 / 1e9, rel=1e-3)
-    assert r["traffic"] == bench.NCU_TRAFFIC[("large-bf16-b64-k6", "cross_attn")][0]
+    assert r["traffic"] == pytest.approx(337.7e6) and r["traffic_source"] == "profiles/x.md"
 
 
 def test_few_row_classes_carry_their_attention_bytes():

@@ -1,5 +1,6 @@
-"""Kernel test of the GEMMs: tcgen05 (one pass and split-K) and SIMT against a
-plain PyTorch fp32 matmul of the same bf16 operands."""
+"""Kernel test of the GEMMs: tcgen05 (one pass and split-K), the many-row
+kernel (query, GELU and residual epilogues; K split over a cluster pair) and
+SIMT against a plain PyTorch fp32 matmul of the same bf16 operands."""
 import pytest
 import torch
 
@@ -40,3 +41,29 @@ def test_fused_argmax_matches_torch(built_lib, cuda, M, N, K):
     picked = ref[got, torch.arange(N, device=cuda)]
     assert torch.all(best - picked <= 1e-3 * K ** 0.5), (best - picked).max()
     assert (got == ref.argmax(dim=0)).float().mean() > 0.99
+
+
+WIDE_SHAPES = [(1280, 448, 1280), (3840, 448, 1280), (5120, 448, 1280), (1280, 448, 5120), (768, 144, 3072),
+               (2304, 544, 768), (256, 65, 64), (128, 300, 128)]
+
+
+@pytest.mark.parametrize("impl", [5, 6, 7])
+@pytest.mark.parametrize("M,N,K", WIDE_SHAPES)
+def test_wide_gemm_matches_torch(built_lib, cuda, impl, M, N, K):
+    """The many-row kernel's tile choices (N tiles of 32 .. 256, ragged last
+    tile, K split in two from 48 k-blocks); GELU against torch's erf GELU
+    within the bf16 rounding of the stored result."""
+    from paper_2608_12703_gb300 import asrspec as A
+    g = torch.Generator(device="cpu").manual_seed(M * 5 + N + K * 3)
+    a = (0.25 * torch.randn(M, K, generator=g)).to(torch.bfloat16).to(cuda)
+    b = torch.randn(N, K, generator=g).to(torch.bfloat16).to(cuda)
+    c = torch.full((N, M), float("nan"), device=cuda)
+    A.asr_spec_test_gemm(impl, a, b, c, M, N, K, torch.cuda.current_stream().cuda_stream)
+    ref = (a.float() @ b.float().T).T
+    if impl == 6:
+        ref = torch.nn.functional.gelu(ref)
+        err = ((c - ref).abs() - 8e-3 * ref.abs()).max().item()
+        assert err <= 1e-4 * K ** 0.5, err
+    else:
+        err = (c - ref).abs().max().item()
+        assert err <= 1e-4 * K ** 0.5, err
