@@ -221,6 +221,17 @@ int asr_spec_draft_create(asr_spec_handle h, const asr_weights* draft);
 int asr_spec_draft_propose(asr_spec_handle h, int32_t k, int32_t window, const int32_t* centers,
                            const int32_t* total_len, int32_t* draft_out, int32_t* lens_out);
 
+/* Confidence threshold of the draft's proposals (App. "Draft length and
+ * confidence threshold": the block length varies per utterance): with
+ * threshold > 0 a round stops proposing for an utterance at the first
+ * position whose argmax probability under the draft (softmax of its
+ * logits) is below the threshold; that position is scored but not proposed.
+ * 0 (the default) turns it off.  Applies to later asr_spec_draft_propose
+ * calls; with it on, the LM head writes the pass's logits and a second
+ * kernel takes the argmax and its probability.
+ * Errors: ASR_E_INVAL (threshold outside [0, 1]), ASR_E_STATE (no draft), ASR_E_OOM. */
+int asr_spec_draft_set_threshold(asr_spec_handle h, float threshold);
+
 /* The restart flags of the last verify (Sec. 3: after a rejected draft the
  * next round restarts drafting from the verified position, else it
  * continues): restart[b] = 1 when accepted[b] < lens[b] (linear verify) or

@@ -30,6 +30,7 @@ EXPORTED = [
     "asr_spec_gemm_noalloc", "asr_spec_timeline", "asr_spec_timeline_read",
     "asr_spec_verify_tree", "asr_spec_restart", "asr_spec_fewrow_trace", "asr_spec_fewrow_trace_read",
     "asr_spec_debug_anchor_profile", "asr_spec_draft_create", "asr_spec_draft_propose",
+    "asr_spec_draft_set_threshold",
 ]
 DRAFT_WIN = {"anchor": 0, "shifted": 1, "random": 2, None: 3}
 PROF_CLASSES = ["qkv", "resid", "query", "mlp_up", "self_attn", "cross_attn", "lm_head", "layernorm", "other",
@@ -86,6 +87,7 @@ def lib():
     L.asr_spec_restart.argtypes = [vp, p32]
     L.asr_spec_draft_create.argtypes = [vp, ctypes.POINTER(AsrWeights)]
     L.asr_spec_draft_propose.argtypes = [vp, i32, i32, p32, p32, p32, p32]
+    L.asr_spec_draft_set_threshold.argtypes = [vp, ctypes.c_float]
     L.asr_spec_fewrow_trace.argtypes = [vp, i32]
     L.asr_spec_fewrow_trace_read.argtypes = [vp, vp, ctypes.c_int64, vp]
     L.asr_spec_debug_anchor_profile.argtypes = [vp, vp]
@@ -177,6 +179,10 @@ def asr_spec_draft_create(h, blob: np.ndarray):
 def asr_spec_draft_propose(h, k, window, centers, total_len, draft_out, lens_out):
     return _check(h, lib().asr_spec_draft_propose(h, k, window, ptr(centers), ptr(total_len), ptr(draft_out),
                                                   ptr(lens_out)), "asr_spec_draft_propose")
+
+
+def asr_spec_draft_set_threshold(h, threshold: float):
+    return _check(h, lib().asr_spec_draft_set_threshold(h, float(threshold)), "asr_spec_draft_set_threshold")
 
 
 def asr_spec_debug_anchor_profile(h, out):

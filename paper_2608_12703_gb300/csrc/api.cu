@@ -157,6 +157,9 @@ struct asr_spec {
   int *d_total = nullptr, *d_centers = nullptr, *d_lens_out = nullptr;
   unsigned long long* d_row_key = nullptr;
   bool d_after_verify = false;
+  float d_threshold = 0.f;            // confidence threshold of the proposals (0 = off)
+  float* d_logits = nullptr;          // threshold on: the pass's logits [R_pad][V]
+  float* d_row_p = nullptr;           // threshold on: [R_pad] probability of each row's argmax
   int last_k = 0;   // k of the last linear verification (stride of its drafts)
 };
 
@@ -789,7 +792,14 @@ int draft_block(asr_spec* h, const RowPlan& plan, int rows, bool lm) {
   e.n_valid = plan.n_rows;
   e.row_key = h->d_row_key;
   e.d = d;
-  return gemm_rows(h, h->w_tok, &h->m_tok, h->V, d, h->d_xf, BUF_DXF, rows, EPI_ARGMAX, e);
+  if (h->d_threshold <= 0.f)
+    return gemm_rows(h, h->w_tok, &h->m_tok, h->V, d, h->d_xf, BUF_DXF, rows, EPI_ARGMAX, e);
+  // confidence threshold: the logits, then per row the argmax and its probability
+  e.out_f32 = h->d_logits;
+  e.ld = h->V;
+  if (int rc = gemm_rows(h, h->w_tok, &h->m_tok, h->V, d, h->d_xf, BUF_DXF, rows, EPI_F32, e)) return rc;
+  launch_draft_softmax(h->d_logits, h->V, plan.n_rows, rows, h->d_row_key, h->d_row_p, h->st);
+  return 0;
 }
 
 bool dims_ok(const asr_model_dims& m) {
@@ -1578,6 +1588,8 @@ int asr_spec_draft_propose(asr_spec_handle h, int32_t k, int32_t window, const i
   A.draft_out = h->d_out;
   A.row_key = h->d_row_key;
   A.x_in = static_cast<__nv_bfloat16*>(h->d_xin);
+  A.threshold = h->d_threshold;
+  A.row_p = h->d_row_p;
   // pass 0: catch-up of the last verification's accepted drafts + the restart
   const int rows0 = std::min(h->R_pad, B * (h->kmax + 1));
   launch_draft_round_plan(A, h->st);
@@ -1597,6 +1609,18 @@ int asr_spec_draft_propose(asr_spec_handle h, int32_t k, int32_t window, const i
     if (int rc = copy_out(h, draft_out, h->d_out, (size_t)B * k)) return rc;
   if (int rc = copy_out(h, lens_out, h->d_lens_out, B)) return rc;
   if (h->host_io) CK(cudaStreamSynchronize(h->st));
+  return ASR_OK;
+}
+
+int asr_spec_draft_set_threshold(asr_spec_handle h, float threshold) {
+  if (!h) return ASR_E_INVAL;
+  if (!h->has_draft) return fail(h, ASR_E_STATE, "no draft (asr_spec_draft_create)");
+  if (!(threshold >= 0.f && threshold <= 1.f)) return fail(h, ASR_E_INVAL, "threshold outside [0, 1]");
+  if (threshold > 0.f && !h->d_logits) {
+    if (int rc = dalloc(h, &h->d_logits, (size_t)h->R_pad * h->V * 4)) return rc;
+    if (int rc = dalloc(h, &h->d_row_p, (size_t)h->R_pad * 4)) return rc;
+  }
+  h->d_threshold = threshold;
   return ASR_OK;
 }
 

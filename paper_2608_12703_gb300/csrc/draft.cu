@@ -240,8 +240,10 @@ __global__ void draft_embed_kernel(DraftArgs A, const __nv_bfloat16* tok_emb, co
 }
 
 // After a pass's LM head: each utterance with a row in the pass takes its
-// argmax as the next proposal (until it holds lens[b] of them) and keeps the
-// row's position for the next continuation row.
+// argmax as the next proposal (until it holds lens[b] of them, or, with the
+// confidence threshold on, until the argmax's probability falls below it:
+// the block then ends unproposed) and keeps the row's position for the next
+// continuation row.
 __global__ void draft_take_kernel(DraftArgs A) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= A.B) return;
@@ -250,9 +252,68 @@ __global__ void draft_take_kernel(DraftArgs A) {
   const int n = A.n_prop[b];
   A.prev_pos[b] = A.plan.row_pos[r];
   if (n < A.lens[b]) {
+    if (A.threshold > 0.f && A.row_p[r] < A.threshold) {   // not confident: the block ends here
+      A.lens[b] = n;
+      return;
+    }
     const uint32_t tok = argmax_index(A.row_key[r]);
     A.draft_out[(size_t)b * A.k + n] = tok < (uint32_t)A.vocab ? (int)tok : 0;
     A.n_prop[b] = n + 1;
+  }
+}
+
+// Softmax statistics of one row of logits (one CTA per row, fixed reduction
+// order): the argmax (lowest index on ties) and its probability
+// 1 / sum_v exp(l_v - l_max) (App. "Draft length and confidence threshold").
+__global__ void __launch_bounds__(256) draft_softmax_kernel(const float* __restrict__ logits, int V,
+                                                            const int* n_rows, unsigned long long* row_key,
+                                                            float* row_p) {
+  __shared__ float s_m[8], s_s[8];
+  __shared__ int s_i[8];
+  const int r = blockIdx.x;
+  if (r >= *n_rows) return;   // uniform over the CTA
+  const float* l = logits + (size_t)r * V;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  float m = -INFINITY;
+  int mi = 0x7fffffff;
+  for (int v = tid; v < V; v += 256) {
+    const float x = l[v];
+    if (x > m) {   // increasing v per thread: the first maximum is kept
+      m = x;
+      mi = v;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, m, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, mi, o);
+    if (om > m || (om == m && oi < mi)) {
+      m = om;
+      mi = oi;
+    }
+  }
+  if (lane == 0) {
+    s_m[warp] = m;
+    s_i[warp] = mi;
+  }
+  __syncthreads();
+  m = s_m[0];
+  mi = s_i[0];
+  for (int w = 1; w < 8; ++w)
+    if (s_m[w] > m || (s_m[w] == m && s_i[w] < mi)) {
+      m = s_m[w];
+      mi = s_i[w];
+    }
+  float sum = 0.f;
+  for (int v = tid; v < V; v += 256) sum += __expf(l[v] - m);
+  sum = warp_sum(sum);
+  if (lane == 0) s_s[warp] = sum;
+  __syncthreads();
+  if (tid == 0) {
+    float t = 0.f;
+    for (int w = 0; w < 8; ++w) t += s_s[w];
+    row_key[r] = argmax_key(m, (uint32_t)mi);
+    row_p[r] = 1.0f / t;
   }
 }
 
@@ -348,6 +409,10 @@ void launch_draft_take(const DraftArgs& a, cudaStream_t st) {
 }
 void launch_draft_finish(const DraftArgs& a, int* lens_out, cudaStream_t st) {
   draft_finish_kernel<<<(a.B + 255) / 256, 256, 0, st>>>(a, lens_out);
+}
+void launch_draft_softmax(const float* logits, int V, const int* n_rows, int rows_max, unsigned long long* row_key,
+                          float* row_p, cudaStream_t st) {
+  draft_softmax_kernel<<<std::max(1, rows_max), 256, 0, st>>>(logits, V, n_rows, row_key, row_p);
 }
 void launch_draft_attn(const DraftAttn& a, cudaStream_t st) {
   static bool configured = false;

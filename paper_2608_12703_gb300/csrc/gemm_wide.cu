@@ -30,7 +30,9 @@ void launch_bn(const WideGemm& g, const Epi& epi, int* status, cudaStream_t st) 
     case 32: launch_w<32, MODE, SPLIT>(g, epi, status, st); break;
     case 64: launch_w<64, MODE, SPLIT>(g, epi, status, st); break;
     case 96: launch_w<96, MODE, SPLIT>(g, epi, status, st); break;
-    default: launch_w<128, MODE, SPLIT>(g, epi, status, st); break;
+    default:
+      if constexpr (MODE != EPI_RESID) launch_w<128, MODE, SPLIT>(g, epi, status, st);
+      break;
   }
 }
 
@@ -38,9 +40,6 @@ template <int MODE>
 void launch_bn_wide(const WideGemm& g, const Epi& epi, int* status, cudaStream_t st) {
   switch (g.bn) {
     case 160: launch_w<160, MODE, 1>(g, epi, status, st); break;
-    case 192: launch_w<192, MODE, 1>(g, epi, status, st); break;
-    case 224: launch_w<224, MODE, 1>(g, epi, status, st); break;
-    case 256: launch_w<256, MODE, 1>(g, epi, status, st); break;
     default: launch_bn<MODE, 1>(g, epi, status, st); break;
   }
 }
@@ -48,8 +47,7 @@ void launch_bn_wide(const WideGemm& g, const Epi& epi, int* status, cudaStream_t
 }  // namespace
 
 // N tiles: as many as the SMs left per M tile allow (a tile per SM), rounded
-// to a tile width of the set; residual tiles at most 128 wide (their residual
-// tile shares the shared memory); long K (>= 48 k-blocks) split over a pair.
+// up to a tile width of the set; long K (>= 48 k-blocks) split over a pair.
 bool wide_pick(int M, int N, int K, int mode, int sms, int* bn, int* split) {
   if (M % 128 || K % 64 || N < 1 || sms < 1) return false;
   if (mode != EPI_QKV && mode != EPI_Q && mode != EPI_GELU && mode != EPI_RESID) return false;
@@ -58,8 +56,10 @@ bool wide_pick(int M, int N, int K, int mode, int sms, int* bn, int* split) {
   const int slots = sms / *split;
   const int nt = std::max(1, slots / mt);
   const int want = (N + nt - 1) / nt;
-  const int cap = mode == EPI_RESID ? 128 : 256;
-  static const int set[8] = {32, 64, 96, 128, 160, 192, 224, 256};
+  // tile widths whose accumulators fit tensor memory; a residual tile also
+  // keeps its residual tile in shared memory beside a ring of 2 stages per pipeline
+  const int cap = mode == EPI_RESID ? 96 : 160;
+  static const int set[5] = {32, 64, 96, 128, 160};
   *bn = cap;
   for (int c : set)
     if (c >= want && c <= cap) {

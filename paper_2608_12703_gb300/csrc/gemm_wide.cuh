@@ -3,17 +3,18 @@
 // streams with a deep pipeline and the weights are re-read as few times as the
 // SM count allows (BN is picked from the rows and the SM count).
 //
-//   two pipelines, each over every other k-block with its own ring of
-//   (A, B) stages and its own accumulators in tensor memory:
+//   P = WG_PIPES pipelines, each over every P-th k-block with its own ring of
+//   (A, B) stages and its own accumulator in tensor memory:
 //   warp 2p / lane 0     : TMA producer of pipeline p; pipeline 0 also loads
 //                          the tile of the residual stream x that a residual
 //                          projection adds to (one TMA box, during the main loop)
 //   warp 2p + 1 / lane 0 : issues pipeline p's tcgen05.mma (M = 128, N = BN,
 //                          K = 16), 4 per k-block, over its accumulators
-//   warps 4 - 7     : during the main loop, the tile's row data (the folded
-//                     LayerNorm's row statistics, the cache slots of the rows);
-//                     then the accumulators, summed in a fixed order, out of
-//                     tensor memory into shared memory
+//   warps 2 P .. 7  : during the main loop, the tile's per-feature operands
+//                     and row data (the folded LayerNorm's row statistics, the
+//                     cache slots of the rows)
+//   warps 4 - 7     : after the MMAs, the accumulators, summed in a fixed
+//                     order, out of tensor memory into shared memory
 //   warps 0 - 7     : the epilogue, one row per warp at a time, 4 features per lane
 //
 // Long K (at least 48 k-blocks) splits in two over a cluster pair: both CTAs
@@ -32,7 +33,8 @@ constexpr int WG_DYN_MAX = 220 * 1024;   // dynamic shared memory budget of one 
 // through an mbarrier pair takes a fixed ~380 cycles however deep the ring
 // (measured), so one pipeline moves one k-block per ~0.3 us; pipelines run
 // side by side
-constexpr int WG_PIPES = 2;
+constexpr int WG_PIPES = 3;
+static_assert(2 * WG_PIPES <= 6, "warps 0 .. 2 P - 1 hold the pipeline roles; at least two warps stay free");
 
 template <int BN, int MODE>
 struct WideCfg {
@@ -48,12 +50,13 @@ struct WideCfg {
   static constexpr int SMEM = 1024 + BAR_OFF + 256;
   // accumulators, split over the pipelines (within a pipeline the K = 16
   // steps of a k-block rotate over its share)
-  static constexpr int NACC = BN <= 128 ? 4 : 2;
+  static constexpr int NACC = WG_PIPES;
   static constexpr uint32_t TMEM_COLS = NACC * BN <= 128 ? 128 : NACC * BN <= 256 ? 256 : 512;
+  static constexpr int BN_MAX = 512 / WG_PIPES / 32 * 32;
   static_assert(STAGES >= 2 * WG_PIPES, "each pipeline needs two stages");
   static_assert(NACC % WG_PIPES == 0, "accumulators split over the pipelines");
   static_assert(BN * LDS * 4 <= STAGES * STAGE_BYTES, "the staged tile must fit the ring");
-  static_assert(BN % 32 == 0 && BN >= 32 && BN <= 256, "N tile");
+  static_assert(BN % 32 == 0 && BN >= 32 && NACC * BN <= 512, "N tile (the accumulators fill at most 512 columns)");
 };
 
 // GELU with erf from Abramowitz & Stegun, formula 7.1.28 (|error| <= 3e-7 in
@@ -196,21 +199,24 @@ gemm_wide_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant
   } else {
     pdl_wait();
     pdl_launch();
-    if (warp >= 4) {
-      const int t = threadIdx.x - 128;
+    if (warp >= 2 * WG_PIPES) {   // the warps without a pipeline role
+      constexpr int NT = WG_THREADS - 64 * WG_PIPES;
+      const int t = threadIdx.x - 64 * WG_PIPES;
       // the epilogue's per-feature operands of this tile
-      s_op[0][t] = __ldg(epi.bias + m0 + t);
-      if (epi.ln_part != nullptr && MODE != EPI_RESID) {
-        s_op[1][t] = __ldg(epi.ln_c1 + m0 + t);
-        s_op[2][t] = __ldg(epi.ln_c2 + m0 + t);
+      for (int f = t; f < 128; f += NT) {
+        s_op[0][f] = __ldg(epi.bias + m0 + f);
+        if (epi.ln_part != nullptr && MODE != EPI_RESID) {
+          s_op[1][f] = __ldg(epi.ln_c1 + m0 + f);
+          s_op[2][f] = __ldg(epi.ln_c2 + m0 + f);
+        }
+        if (MODE == EPI_RESID && epi.xg != nullptr) s_op[3][f] = __ldg(epi.xg_gain + m0 + f);
       }
-      if (MODE == EPI_RESID && epi.xg != nullptr) s_op[3][t] = __ldg(epi.xg_gain + m0 + t);
       // Folded LayerNorm: row statistics combined from the producer's equal
       // slices, one pass shifted by the first slice's mean:
       // mean = shift + E / S, M2 = sum M2_s + c (sum e_s^2 - E^2 / S)
       if (epi.ln_part != nullptr) {
         const int S = epi.ln_S;
-        for (int rl = t; rl < BN; rl += 128) {
+        for (int rl = t; rl < BN; rl += NT) {
           const int n = n0 + rl;
           const bool ok = n < n_valid;
           const float2* pr = epi.ln_part + (ok ? n : 0);
@@ -231,7 +237,7 @@ gemm_wide_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant
         }
       }
       if constexpr (MODE == EPI_QKV)
-        for (int rl = t; rl < BN; rl += 128) {
+        for (int rl = t; rl < BN; rl += NT) {
           const int n = n0 + rl;
           s_rb[rl] = n < n_valid ? epi.row_b[n] : 0;
           s_rp[rl] = n < n_valid ? epi.row_pos[n] : 0;

@@ -40,7 +40,7 @@ struct WideGemm {
   CUtensorMap mapB;   // rows [R][K], box 64 x bn
   CUtensorMap mapX;   // RESID: the residual stream [R][d] fp32, box 128 x bn (others: unused)
   int M, N, K;
-  int bn, split;      // N tile (32 .. 256, RESID <= 128); 1, or 2 = K split over a cluster pair
+  int bn, split;      // N tile (32 .. 160, RESID <= 96); 1, or 2 = K split over a cluster pair
   int stages = 0;     // stages per pipeline, at least 2 (0: as deep as shared memory allows)
   bool pdl = false;
 };
@@ -257,6 +257,8 @@ struct DraftArgs {
   int* draft_out;            // [B][k] proposals
   unsigned long long* row_key;   // [R_max] LM-head argmax keys of the pass
   __nv_bfloat16* x_in;       // [R_max][4 d] the pass's input representations
+  float threshold;           // confidence threshold on the proposal's probability (0 = off)
+  const float* row_p;        // [R_max] softmax probability of each row's argmax (threshold on)
 };
 struct DraftAttn {
   const float* q;            // [R][d] fp32
@@ -276,6 +278,10 @@ void launch_draft_embed(const DraftArgs& a, int rows_max, const void* tok_emb, c
 void launch_draft_take(const DraftArgs& a, cudaStream_t st);
 void launch_draft_finish(const DraftArgs& a, int* lens_out, cudaStream_t st);
 void launch_draft_attn(const DraftAttn& a, cudaStream_t st);
+// Per row of logits [rows][V] (fp32): the argmax key (as the LM-head epilogue
+// writes it: lowest index on ties) and the softmax probability of the argmax.
+void launch_draft_softmax(const float* logits, int V, const int* n_rows, int rows_max, unsigned long long* row_key,
+                          float* row_p, cudaStream_t st);
 
 // ---- Accept / commit ------------------------------------------------------------
 void launch_prefill_advance(int B, int c, const int* n_utt_rows, int* kv_len, cudaStream_t st);

@@ -217,10 +217,12 @@ class DraftModel:
     (catch-up of the last verification, restart, continuations) and leaves
     drafts and lens on the device, ready for ``Session.verify_device``."""
 
-    def __init__(self, sess: Session, blob: np.ndarray, total_lens, k: int, window="anchor"):
+    def __init__(self, sess: Session, blob: np.ndarray, total_lens, k: int, window="anchor", threshold: float = 0.0):
         if sess.B:
             raise A.AsrSpecError("attach the draft before encode_cache")
         A.asr_spec_draft_create(sess.h, blob)
+        if threshold > 0.0:
+            A.asr_spec_draft_set_threshold(sess.h, threshold)
         self.sess, self.k, self.window = sess, k, A.DRAFT_WIN[window]
         dev = sess.dev
         with torch.cuda.stream(sess.stream):

@@ -15,7 +15,8 @@ With no near-tie the GPU's emitted tokens are the target's greedy transcript
 
 Cases: batch 1 with k = 8 (nine verify rows, the few-row layers), a ragged
 batch of five under each window kind (anchor, shifted, random centres, none),
-a one-token prompt with k = 0 rounds and utterances that finish at once;
+a one-token prompt with k = 0 rounds and utterances that finish at once, the
+confidence threshold (blocks of varying length);
 and the device loop (propose -> verify, nothing read back between rounds)
 against the host-stepped loop, output for output.
 """
@@ -43,17 +44,41 @@ class DraftStats:
         self.max_gap = 0.0
         self.gaps = []          # oracle top-2 gap of every proposal
         self.flip_gaps = []
+        self.thr_decisions = 0  # threshold decisions checked, and those within THR_MARGIN that went the other way
+        self.thr_near = 0
+        self.cut = 0            # rounds the threshold ended early
 
 
-def _forced_round(dro, b, pending, P, feat, lens, props, win, ds, scale):
+THR_MARGIN = 0.05   # relative: the draft's top probability within this of the threshold decides either way
+
+
+def _forced_round(dro, b, pending, P, feat, lens, props, win, ds, scale, threshold=0.0, lens_max=None):
     """The oracle draft over the GPU's round for utterance b: the restart at P
-    and the continuations, each fed the GPU's previous proposal."""
-    if lens == 0:
+    and the continuations, each fed the GPU's previous proposal.  With a
+    confidence threshold the GPU proposes lens <= lens_max tokens; each
+    proposal's oracle probability must reach the threshold, and a block the
+    GPU ended early must end at a position the oracle also finds below it
+    (both unless the probability is within THR_MARGIN of the threshold)."""
+    lens_max = lens if lens_max is None else lens_max
+    if lens_max == 0:
         dro.step(b, int(pending), P, feat, win)
         return
     tok, f = int(pending), feat
-    for i in range(lens):
+    steps = lens + 1 if lens < lens_max else lens
+    for i in range(steps):
         logits, x = dro.step(b, tok, P + i, f, win)
+        if threshold > 0.0:
+            e = np.exp(logits - logits.max())
+            p_top = 1.0 / e.sum()
+            below = p_top < threshold
+            if below != (i == lens):
+                assert abs(p_top / threshold - 1.0) < THR_MARGIN, (
+                    f"utt {b}, position {i + 1}: oracle top probability {p_top} vs threshold {threshold}, "
+                    f"GPU {'ended' if i == lens else 'proposed'}")
+                ds.thr_near += 1
+            ds.thr_decisions += 1
+        if i == lens:
+            break
         a, g = int(np.argmax(logits)), int(props[i])
         ds.proposals += 1
         top2 = np.partition(logits, -2)[-2:]
@@ -67,7 +92,7 @@ def _forced_round(dro, b, pending, P, feat, lens, props, win, ds, scale):
         tok, f = g, np.tile(x, (4, 1))
 
 
-def run_lockstep(enc_lens, total, k, kind, prompt_len=W.PROMPT_LEN, k_sched=None, seed=0):
+def run_lockstep(enc_lens, total, k, kind, prompt_len=W.PROMPT_LEN, k_sched=None, seed=0, threshold=0.0):
     from paper_2608_12703_gb300.session import DraftModel, Session
     B = len(enc_lens)
     blob = W.make_weights(DIMS, std=STD)
@@ -86,7 +111,7 @@ def run_lockstep(enc_lens, total, k, kind, prompt_len=W.PROMPT_LEN, k_sched=None
     dro.encode()
     dro.prefill(prompt)
     sess = Session(DIMS, blob, max_batch=B, max_draft=k)
-    dm = DraftModel(sess, dblob, total, k, kind)
+    dm = DraftModel(sess, dblob, total, k, kind, threshold=threshold)
     sess.encode_cache(enc, enc_lens)
     sess.prefill(prompt)
     assert sess.status() == 0
@@ -107,7 +132,12 @@ def run_lockstep(enc_lens, total, k, kind, prompt_len=W.PROMPT_LEN, k_sched=None
             dm.set_centers(centers)
         dg, lg = dm.propose(kk)
         dg, lg = sess.host(dg).copy(), sess.host(lg).copy()
-        np.testing.assert_array_equal(lg, lens_o)
+        if threshold > 0.0:
+            np.testing.assert_array_equal(lg < 0, lens_o < 0)
+            assert np.all(lg <= lens_o)
+            ds.cut += int(np.sum((lg >= 0) & (lg < lens_o)))
+        else:
+            np.testing.assert_array_equal(lg, lens_o)
         for b in range(B):
             if lens_o[b] < 0:
                 continue
@@ -117,8 +147,8 @@ def run_lockstep(enc_lens, total, k, kind, prompt_len=W.PROMPT_LEN, k_sched=None
             else:
                 c = centers[b] if kind == "random" else window_center(kind, anchor[b], T)
                 win = window(c, T)
-            _forced_round(dro, b, orc.pending[b], int(orc.kv_len[b]), feat[b], int(lens_o[b]), dg[b], win, ds,
-                          scale)
+            _forced_round(dro, b, orc.pending[b], int(orc.kv_len[b]), feat[b], int(lg[b]), dg[b], win, ds,
+                          scale, threshold, int(lens_o[b]))
         P_old = orc.kv_len.copy()
         draft = dg if kk > 0 else np.zeros((B, 0), dtype=np.int32)
         ro, rg = compare_round(orc, sess, draft, lg, st, scale=scale)
@@ -186,6 +216,19 @@ def test_draft_edges(built_lib, cuda):
     sched = lambda r: [5, 0, 2, 5, 1][r % 5]
     st, ds, seqs, truth, _ = run_lockstep(enc_lens, total, 5, "anchor", prompt_len=1, k_sched=sched)
     _check("edges", st, ds, seqs, truth, total)
+
+
+def test_draft_confidence_threshold(built_lib, cuda):
+    """Variable block lengths from the confidence threshold (App. "Draft length
+    and confidence threshold"), set between the draft's typical top
+    probabilities so that some blocks end early and others run to k."""
+    enc_lens = [300, 57, 181]
+    total = [W.PROMPT_LEN + n for n in (30, 21, 26)]
+    st, ds, seqs, truth, _ = run_lockstep(enc_lens, total, 6, "anchor", threshold=0.009)
+    _check("threshold 0.009", st, ds, seqs, truth, total)
+    print(f"  threshold decisions {ds.thr_decisions}, near-threshold {ds.thr_near}, blocks cut {ds.cut}")
+    assert ds.cut > 3
+    assert ds.thr_near <= near_tie_bound(ds.thr_decisions)
 
 
 def test_device_loop_matches_host_stepped(built_lib, cuda):
