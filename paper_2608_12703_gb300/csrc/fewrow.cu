@@ -102,14 +102,22 @@ __device__ void fr_ln(const float* x, const float* g, const float* bta, uint8_t*
   }
 }
 
-// Thread 0: the first R rows of a row-major [rows][ld] array (element size
-// es, `bytes` of each row from column col0) into shared memory at dst with a
-// row pitch, one bulk copy per row, counted on bar.
+// Warp 0 (all lanes): the first R rows of a row-major [rows][ld] array
+// (element size es, `bytes` of each row from column col0) into shared memory
+// at dst with a row pitch, counted on bar: one bulk copy when source and
+// destination rows are both contiguous, else one per row, issued by R lanes
+// side by side (a bulk copy takes tens of ns to issue).
 __device__ __forceinline__ void fr_rows_async(const void* src, int ld, int col0, int es, uint32_t bytes, int R,
                                               uint8_t* dst, uint32_t pitch, uint64_t* bar) {
-  mbar_arrive_expect_tx(bar, (uint32_t)R * bytes);
-  for (int r = 0; r < R; ++r)
-    bulk_load(dst + r * pitch, static_cast<const char*>(src) + ((size_t)r * ld + col0) * es, bytes, bar);
+  const int lane = threadIdx.x & 31;
+  const char* s0 = static_cast<const char*>(src) + (size_t)col0 * es;
+  if (lane == 0) mbar_arrive_expect_tx(bar, (uint32_t)R * bytes);
+  __syncwarp();
+  if (pitch == bytes && (size_t)ld * es == bytes) {
+    if (lane == 0) bulk_load(dst, s0, (uint32_t)R * bytes, bar);
+  } else {
+    for (int r = lane; r < R; r += 32) bulk_load(dst + r * pitch, s0 + (size_t)r * ld * es, bytes, bar);
+  }
 }
 
 // Weight tiles of the few-row kernels are packed (at create) so that one
@@ -242,15 +250,17 @@ __global__ void __launch_bounds__(FR_T) fr_gemv_kernel(const __grid_constant__ F
   const int R = *A.n_rows;   // uniform over the grid
   const bool live = R > 0;
   if (live) {
-    if (tid == 0) {   // the input rows: written by the previous launch
+    if (tid < 32) {   // the input rows: written by the previous launch
       if constexpr (MODE == FR_GELU) {
         fr_rows_async(A.x, D, 0, 4, 4u * D, R, reinterpret_cast<uint8_t*>(xs), 4u * D, &abar);
-      } else {
-        mbar_arrive_expect_tx(&abar, (uint32_t)(R * np) * 2u * D);
-        for (int p = 0; p < np; ++p)
-          for (int r = 0; r < R; ++r)
-            bulk_load(act + (p * FR_R + r) * P, A.a + (size_t)r * A.K + (size_t)ks * Kc + (size_t)p * D, 2u * D,
-                      &abar);
+      } else {   // panel p, row r: one bulk copy each, issued by the warp's lanes side by side
+        if (tid == 0) mbar_arrive_expect_tx(&abar, (uint32_t)(R * np) * 2u * D);
+        __syncwarp();
+        for (int q = tid; q < R * np; q += 32) {
+          const int p = q / R, r = q - p * R;
+          bulk_load(act + (p * FR_R + r) * P, A.a + (size_t)r * A.K + (size_t)ks * Kc + (size_t)p * D, 2u * D,
+                    &abar);
+        }
       }
     }
     mbar_wait(&abar, 0, A.status);
@@ -455,7 +465,7 @@ __global__ void __launch_bounds__(FR_T) fr_self_kernel(const __grid_constant__ C
   const int R = *A.plan.n_rows;
   const bool live = R > 0;
   if (live) {
-    if (tid == 0) fr_rows_async(A.x, d, 0, 4, 4u * d, R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
+    if (tid < 32) fr_rows_async(A.x, d, 0, 4, 4u * d, R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
     mbar_wait(&lbar, 0, A.status);
     mbar_wait(&xbar, 0, A.status);
     fr_ln<KSW>(xs, lnp, lnp + d, act, R);
@@ -655,7 +665,7 @@ __global__ void __launch_bounds__(FR_T) fr_cross_kernel(const __grid_constant__ 
   const int R = *A.plan.n_rows;
   const bool live = R > 0;
   if (live) {
-    if (tid == 0) fr_rows_async(A.x, d, 0, 4, 4u * d, R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
+    if (tid < 32) fr_rows_async(A.x, d, 0, 4, 4u * d, R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
     mbar_wait(&lbar, 0, A.status);
     mbar_wait(&xbar, 0, A.status);
     fr_ln<KSW>(xs, lnp, lnp + d, act, R);

@@ -11,7 +11,7 @@ Record a capture (reads the CSV that ``ncu -i <report> --page raw --csv``
 printed):
 
   python -m paper_2608_12703_gb300.ncu_traffic record --csv <file> \
-      --kernel '<regex>' --workload <name> --cls <class> --group <gemm_tc|fewrow|attn_tc|rows> \
+      --kernel '<regex>' --workload <name> --cls <class> --group <gemm_tc|gemm_wide|fewrow|attn_tc|rows> \
       --summary profiles/<summary>.md [--scale <factor>]
 """
 from __future__ import annotations
@@ -32,6 +32,7 @@ TRAFFIC_FILE = os.path.join(ROOT, "profiles", "ncu_traffic.json")
 # the sources a kernel's code comes from (its own file, the headers it includes)
 SOURCE_GROUPS: Dict[str, List[str]] = {
     "gemm_tc": ["csrc/gemm_tc.cu", "csrc/kernels.h", "csrc/epilogue.cuh", "csrc/common.cuh"],
+    "gemm_wide": ["csrc/gemm_wide.cuh", "csrc/gemm_wide.cu", "csrc/kernels.h", "csrc/epilogue.cuh", "csrc/common.cuh"],
     "fewrow": ["csrc/fewrow.cu", "csrc/rowmma.cuh", "csrc/kernels.h", "csrc/epilogue.cuh", "csrc/common.cuh"],
     "attn_tc": ["csrc/attention_tc.cu", "csrc/kernels.h", "csrc/epilogue.cuh", "csrc/common.cuh"],
     "rows": ["csrc/rows.cu", "csrc/kernels.h", "csrc/epilogue.cuh", "csrc/common.cuh"],
