@@ -247,27 +247,28 @@ __global__ void __launch_bounds__(FR_T) fr_gemv_kernel(const __grid_constant__ F
   tl_mark(A.tl, TL_WORK);
   fr_stamp(A.trace, 1);
   pdl_launch();
-  const int R = *A.n_rows;   // uniform over the grid
-  const bool live = R > 0;
-  if (live) {
-    if (tid < 32) {   // the input rows: written by the previous launch
-      if constexpr (MODE == FR_GELU) {
-        fr_rows_async(A.x, D, 0, 4, 4u * D, R, reinterpret_cast<uint8_t*>(xs), 4u * D, &abar);
-      } else {   // panel p, row r: one bulk copy each, issued by the warp's lanes side by side
-        if (tid == 0) mbar_arrive_expect_tx(&abar, (uint32_t)(R * np) * 2u * D);
-        __syncwarp();
-        for (int q = tid; q < R * np; q += 32) {
-          const int p = q / R, r = q - p * R;
-          bulk_load(act + (p * FR_R + r) * P, A.a + (size_t)r * A.K + (size_t)ks * Kc + (size_t)p * D, 2u * D,
-                    &abar);
-        }
+  // The input rows (written by the previous launch): all FR_R row slots,
+  // issued at once without waiting to read how many are live (rows past them
+  // are not used)
+  if (tid < 32) {
+    if constexpr (MODE == FR_GELU) {
+      fr_rows_async(A.x, D, 0, 4, 4u * D, FR_R, reinterpret_cast<uint8_t*>(xs), 4u * D, &abar);
+    } else {   // panel p, row r: one bulk copy each, issued by the warp's lanes side by side
+      if (tid == 0) mbar_arrive_expect_tx(&abar, (uint32_t)(FR_R * np) * 2u * D);
+      __syncwarp();
+      for (int q = tid; q < FR_R * np; q += 32) {
+        const int p = q / FR_R, r = q - p * FR_R;
+        bulk_load(act + (p * FR_R + r) * P, A.a + (size_t)r * A.K + (size_t)ks * Kc + (size_t)p * D, 2u * D,
+                  &abar);
       }
     }
-    mbar_wait(&abar, 0, A.status);
-    if constexpr (MODE == FR_GELU) {
-      mbar_wait(&lbar, 0, A.status);
-      fr_ln<KSW>(xs, lnp, lnp + D, act, R);
-    }
+  }
+  const int R = *A.n_rows;   // uniform over the grid
+  const bool live = R > 0;
+  mbar_wait(&abar, 0, A.status);
+  if constexpr (MODE == FR_GELU) {
+    mbar_wait(&lbar, 0, A.status);
+    if (live) fr_ln<KSW>(xs, lnp, lnp + D, act, R);
   }
   fr_stamp(A.trace, 2);
   mbar_wait(&wbar, 0, A.status);
@@ -462,14 +463,13 @@ __global__ void __launch_bounds__(FR_T) fr_self_kernel(const __grid_constant__ C
   tl_mark(A.tl, TL_WORK);
   fr_stamp(A.trace, 1);
   pdl_launch();
+  // the residual rows: all FR_R slots at once (rows past the live ones are not used)
+  if (tid < 32) fr_rows_async(A.x, d, 0, 4, 4u * d, FR_R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
   const int R = *A.plan.n_rows;
   const bool live = R > 0;
-  if (live) {
-    if (tid < 32) fr_rows_async(A.x, d, 0, 4, 4u * d, R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
-    mbar_wait(&lbar, 0, A.status);
-    mbar_wait(&xbar, 0, A.status);
-    fr_ln<KSW>(xs, lnp, lnp + d, act, R);
-  }
+  mbar_wait(&lbar, 0, A.status);
+  mbar_wait(&xbar, 0, A.status);
+  if (live) fr_ln<KSW>(xs, lnp, lnp + d, act, R);
   fr_stamp(A.trace, 2);
   mbar_wait(&wbar, 0, A.status);
   fr_stamp(A.trace, 3);
@@ -662,14 +662,13 @@ __global__ void __launch_bounds__(FR_T) fr_cross_kernel(const __grid_constant__ 
   tl_mark(A.tl, TL_WORK);
   fr_stamp(A.trace, 1);
   pdl_launch();
+  // the residual rows: all FR_R slots at once (rows past the live ones are not used)
+  if (tid < 32) fr_rows_async(A.x, d, 0, 4, 4u * d, FR_R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
   const int R = *A.plan.n_rows;
   const bool live = R > 0;
-  if (live) {
-    if (tid < 32) fr_rows_async(A.x, d, 0, 4, 4u * d, R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
-    mbar_wait(&lbar, 0, A.status);
-    mbar_wait(&xbar, 0, A.status);
-    fr_ln<KSW>(xs, lnp, lnp + d, act, R);
-  }
+  mbar_wait(&lbar, 0, A.status);
+  mbar_wait(&xbar, 0, A.status);
+  if (live) fr_ln<KSW>(xs, lnp, lnp + d, act, R);
   fr_stamp(A.trace, 2);
   mbar_wait(&wbar, 0, A.status);
   fr_stamp(A.trace, 3);
