@@ -337,8 +337,9 @@ int asr_spec_timeline_read(asr_spec_handle h, uint64_t* ns, int32_t* kind, int32
  * its 6 L layer launches, the GPU global timer (ns) at 12 phases: entry, past
  * the wait on the previous launch, input rows ready, weights landed,
  * projection reduced, exchange landed, attention done, exit, first K/V chunk
- * landed, first chunk combined, merge inputs landed, (unused) (0 where a
- * launch has no such phase); verify then launches directly (no graph).  A
+ * landed, first chunk combined, merge inputs landed, bf16 input rows landed
+ * (GEMVs without a LayerNorm) (0 where a launch has no such phase); verify
+ * then launches directly (no graph).  A
  * verify of more rows records its 6 L tensor-core projections instead (in
  * layer order: QKV, self out, cross query, cross out, MLP up, MLP down), for
  * their first 320 CTAs: 0 entry, 1 set-up done, 2 first k-block landed,

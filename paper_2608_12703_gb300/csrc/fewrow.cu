@@ -56,67 +56,85 @@ __device__ __forceinline__ void fr_stamp(unsigned long long* tr, int phase) {
   if (tr != nullptr && threadIdx.x == 0) tr[(size_t)blockIdx.x * FR_TRACE_PHASES + phase] = global_ns();
 }
 
-// act[r] = bf16(LayerNorm(x_r) * g + b) for r < R, fp32 statistics; warp w
-// takes rows w and w + 8.  x (rows of D fp32), g, b: staged in shared memory.
+// LayerNorm of the step's rows in registers.  Lane l of every warp holds the
+// gain and bias of columns 4 (l + 32 i) .. + 3 (i < KSW), loaded before the
+// kernel waits on its predecessor (they are constants); after the wait, warp
+// w reads rows w and w + 8 of the residual stream straight from L2 into
+// registers (all FR_R row slots exist; the ones past the live rows are read
+// and not used), and writes bf16(LayerNorm(x_r) * g + b), fp32 statistics,
+// into the MMA operand rows.
 template <int KSW>
-__device__ void fr_ln(const float* x, const float* g, const float* bta, uint8_t* act, int R) {
-  constexpr int D = KSW * 128;
+struct LnRegs {
+  float4 g[KSW], b[KSW];
+};
+template <int KSW>
+__device__ __forceinline__ void fr_ln_params(LnRegs<KSW>& p, const float* g, const float* b) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int i = 0; i < KSW; ++i) {
+    p.g[i] = __ldg(reinterpret_cast<const float4*>(g) + lane + 32 * i);
+    p.b[i] = __ldg(reinterpret_cast<const float4*>(b) + lane + 32 * i);
+  }
+}
+template <int KSW>
+__device__ __forceinline__ void fr_ln_fetch(float4 (&v)[2][KSW], const float* x) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float4 v[2][KSW];
 #pragma unroll
   for (int j = 0; j < 2; ++j) {
     const int r = warp + 8 * j;
-    if (r < R) {
-      const float4* xr = reinterpret_cast<const float4*>(x + (size_t)r * D);
+    const float4* xr = reinterpret_cast<const float4*>(x + (size_t)r * KSW * 128);
 #pragma unroll
-      for (int i = 0; i < KSW; ++i) v[j][i] = xr[lane + 32 * i];
+    for (int i = 0; i < KSW; ++i) v[j][i] = r < FR_R ? __ldcg(xr + lane + 32 * i) : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+}
+template <int KSW>
+__device__ __forceinline__ void fr_ln_apply(const float4 (&v)[2][KSW], const LnRegs<KSW>& p, uint8_t* act, int R) {
+  constexpr int D = KSW * 128;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float mean[2], rstd[2];
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < KSW; ++i) s += (v[j][i].x + v[j][i].y) + (v[j][i].z + v[j][i].w);
+    mean[j] = s;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {   // the two rows' warp sums side by side
+    mean[0] += __shfl_xor_sync(0xffffffffu, mean[0], o);
+    mean[1] += __shfl_xor_sync(0xffffffffu, mean[1], o);
+  }
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    mean[j] = mean[j] / (float)D;
+    float q = 0.f;
+#pragma unroll
+    for (int i = 0; i < KSW; ++i) {
+      const float a = v[j][i].x - mean[j], b = v[j][i].y - mean[j], c = v[j][i].z - mean[j],
+                  e = v[j][i].w - mean[j];
+      q += (a * a + b * b) + (c * c + e * e);
     }
+    rstd[j] = q;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    rstd[0] += __shfl_xor_sync(0xffffffffu, rstd[0], o);
+    rstd[1] += __shfl_xor_sync(0xffffffffu, rstd[1], o);
   }
 #pragma unroll
   for (int j = 0; j < 2; ++j) {
     const int r = warp + 8 * j;
     if (r >= R) continue;
-    float s = 0.f;
-#pragma unroll
-    for (int i = 0; i < KSW; ++i) s += (v[j][i].x + v[j][i].y) + (v[j][i].z + v[j][i].w);
-    const float mean = warp_sum(s) / (float)D;
-    float q = 0.f;
-#pragma unroll
-    for (int i = 0; i < KSW; ++i) {
-      const float a = v[j][i].x - mean, b = v[j][i].y - mean, c = v[j][i].z - mean, e = v[j][i].w - mean;
-      q += (a * a + b * b) + (c * c + e * e);
-    }
-    const float rstd = rsqrtf(warp_sum(q) / (float)D + 1e-5f);
+    const float rs = rsqrtf(rstd[j] / (float)D + 1e-5f), mu = mean[j];
     uint2* row = reinterpret_cast<uint2*>(act + (size_t)r * fr_pitch(D));
 #pragma unroll
     for (int i = 0; i < KSW; ++i) {
-      const int c4 = lane + 32 * i;
-      const float4 gg = reinterpret_cast<const float4*>(g)[c4];
-      const float4 bb = reinterpret_cast<const float4*>(bta)[c4];
-      const float4 w = v[j][i];
+      const float4 w = v[j][i], gg = p.g[i], bb = p.b[i];
       uint2 o;
-      o.x = bf2_bits((w.x - mean) * rstd * gg.x + bb.x, (w.y - mean) * rstd * gg.y + bb.y);
-      o.y = bf2_bits((w.z - mean) * rstd * gg.z + bb.z, (w.w - mean) * rstd * gg.w + bb.w);
-      row[c4] = o;
+      o.x = bf2_bits((w.x - mu) * rs * gg.x + bb.x, (w.y - mu) * rs * gg.y + bb.y);
+      o.y = bf2_bits((w.z - mu) * rs * gg.z + bb.z, (w.w - mu) * rs * gg.w + bb.w);
+      row[lane + 32 * i] = o;
     }
-  }
-}
-
-// Warp 0 (all lanes): the first R rows of a row-major [rows][ld] array
-// (element size es, `bytes` of each row from column col0) into shared memory
-// at dst with a row pitch, counted on bar: one bulk copy when source and
-// destination rows are both contiguous, else one per row, issued by R lanes
-// side by side (a bulk copy takes tens of ns to issue).
-__device__ __forceinline__ void fr_rows_async(const void* src, int ld, int col0, int es, uint32_t bytes, int R,
-                                              uint8_t* dst, uint32_t pitch, uint64_t* bar) {
-  const int lane = threadIdx.x & 31;
-  const char* s0 = static_cast<const char*>(src) + (size_t)col0 * es;
-  if (lane == 0) mbar_arrive_expect_tx(bar, (uint32_t)R * bytes);
-  __syncwarp();
-  if (pitch == bytes && (size_t)ld * es == bytes) {
-    if (lane == 0) bulk_load(dst, s0, (uint32_t)R * bytes, bar);
-  } else {
-    for (int r = lane; r < R; r += 32) bulk_load(dst + r * pitch, s0 + (size_t)r * ld * es, bytes, bar);
   }
 }
 
@@ -200,17 +218,17 @@ __device__ __forceinline__ Pair fr_reduce(const float (&acc)[FR_MAXT][4], float*
 // [q K / KS, (q + 1) K / KS); rank 0 adds the other ranks' partials after its
 // own, in rank order.
 // ---------------------------------------------------------------------------
-__host__ __device__ inline int gemv_ln_off(int D, int tiles_max, int np, int KS) {
+__host__ __device__ inline int gemv_smem_bytes(int D, int tiles_max, int np, int KS) {
   return align_up(tiles_max * 16 * np * D, 128) + np * FR_R * fr_pitch(D) + FR_RED +
          (KS - 1) * FR_MAXT * 4 * FR_R * 8;
 }
 
 template <int KSW, int MODE, int KS>
-__global__ void __launch_bounds__(FR_T) fr_gemv_kernel(const __grid_constant__ FrGemv A) {
+__global__ void __launch_bounds__(FR_T, 1) fr_gemv_kernel(const __grid_constant__ FrGemv A) {
   constexpr int D = KSW * 128;
   constexpr uint32_t P = fr_pitch(D);
   extern __shared__ __align__(128) uint8_t fr_smem[];
-  __shared__ __align__(8) uint64_t wbar, lbar, abar, rbar;
+  __shared__ __align__(8) uint64_t wbar, abar, rbar;
   const int tid = threadIdx.x;
   const int ks = KS > 1 ? (int)cluster_ctarank() : 0;
   const int Kc = A.K / KS, np = Kc / D;
@@ -221,26 +239,20 @@ __global__ void __launch_bounds__(FR_T) fr_gemv_kernel(const __grid_constant__ F
   uint8_t* act = wts + align_up(A.tiles_max * (int)wtile, 128);
   float* red = reinterpret_cast<float*>(act + np * FR_R * P);
   float2* recv = reinterpret_cast<float2*>(reinterpret_cast<uint8_t*>(red) + FR_RED);
-  float* lnp = reinterpret_cast<float*>(fr_smem + gemv_ln_off(D, A.tiles_max, np, KS));   // gain, bias
-  float* xs = lnp + 2 * D;   // FR_GELU: the residual rows, fp32
   tl_mark(A.tl, TL_ENTRY);
   fr_stamp(A.trace, 0);
   if (tid == 0) {
     mbar_init(&wbar, 1);
-    mbar_init(&lbar, 1);
     mbar_init(&abar, 1);
     mbar_init(&rbar, 1);
     fence_mbar_init();
     if (KS > 1 && ks == 0) mbar_arrive_expect_tx(&rbar, (uint32_t)((KS - 1) * ntile * 4 * FR_R * 8));
-    if (MODE == FR_GELU) {   // the LayerNorm's gain and bias (constants)
-      mbar_arrive_expect_tx(&lbar, 8u * D);
-      bulk_load(lnp, A.ln_g, 4u * D, &lbar);
-      bulk_load(lnp + D, A.ln_b, 4u * D, &lbar);
-    }
     mbar_arrive_expect_tx(&wbar, (uint32_t)ntile * wtile);
     for (int i = 0; i < ntile; ++i)
       bulk_load(wts + i * wtile, A.W + ((size_t)(t0 + i) * A.K + (size_t)ks * Kc) * 8, wtile, &wbar);
   }
+  LnRegs<KSW> lnr;
+  if constexpr (MODE == FR_GELU) fr_ln_params(lnr, A.ln_g, A.ln_b);
   __syncthreads();
   if (KS > 1) cluster_arrive_relaxed();
   pdl_wait();
@@ -248,27 +260,26 @@ __global__ void __launch_bounds__(FR_T) fr_gemv_kernel(const __grid_constant__ F
   fr_stamp(A.trace, 1);
   pdl_launch();
   // The input rows (written by the previous launch): all FR_R row slots,
-  // issued at once without waiting to read how many are live (rows past them
-  // are not used)
-  if (tid < 32) {
-    if constexpr (MODE == FR_GELU) {
-      fr_rows_async(A.x, D, 0, 4, 4u * D, FR_R, reinterpret_cast<uint8_t*>(xs), 4u * D, &abar);
-    } else {   // panel p, row r: one bulk copy each, issued by the warp's lanes side by side
-      if (tid == 0) mbar_arrive_expect_tx(&abar, (uint32_t)(FR_R * np) * 2u * D);
-      __syncwarp();
-      for (int q = tid; q < FR_R * np; q += 32) {
-        const int p = q / FR_R, r = q - p * FR_R;
-        bulk_load(act + (p * FR_R + r) * P, A.a + (size_t)r * A.K + (size_t)ks * Kc + (size_t)p * D, 2u * D,
-                  &abar);
-      }
+  // requested at once without waiting to read how many are live (rows past
+  // them are not used)
+  float4 xv[2][KSW];
+  if constexpr (MODE == FR_GELU) {
+    fr_ln_fetch<KSW>(xv, A.x);
+  } else if (tid < 32) {   // panel p, row r: one bulk copy each, issued by the warp's lanes side by side
+    if (tid == 0) mbar_arrive_expect_tx(&abar, (uint32_t)(FR_R * np) * 2u * D);
+    __syncwarp();
+    for (int q = tid; q < FR_R * np; q += 32) {
+      const int p = q / FR_R, r = q - p * FR_R;
+      bulk_load(act + (p * FR_R + r) * P, A.a + (size_t)r * A.K + (size_t)ks * Kc + (size_t)p * D, 2u * D, &abar);
     }
   }
   const int R = *A.n_rows;   // uniform over the grid
   const bool live = R > 0;
-  mbar_wait(&abar, 0, A.status);
   if constexpr (MODE == FR_GELU) {
-    mbar_wait(&lbar, 0, A.status);
-    if (live) fr_ln<KSW>(xs, lnp, lnp + D, act, R);
+    if (live) fr_ln_apply<KSW>(xv, lnr, act, R);
+  } else {
+    mbar_wait(&abar, 0, A.status);
+    fr_stamp(A.trace, 11);
   }
   fr_stamp(A.trace, 2);
   mbar_wait(&wbar, 0, A.status);
@@ -325,7 +336,7 @@ __global__ void __launch_bounds__(FR_T) fr_gemv_kernel(const __grid_constant__ F
 // Per-head cluster kernels: shared memory layout
 // ---------------------------------------------------------------------------
 struct HeadLayout {
-  int wts, act, kv, red, gat, mrg, part, ln, xs, total;
+  int wts, act, kv, red, gat, mrg, part, total;
 };
 // The merge buffer and this CTA's partial alias the reduction buffer: a peer
 // sends a partial only after this CTA's gather contribution, which follows
@@ -345,10 +356,6 @@ __host__ __device__ inline HeadLayout head_layout(int D, int tiles_max, int n_sl
   o += align_up(FR_RED > (mrg_slots + 1) * FR_PART ? FR_RED : (mrg_slots + 1) * FR_PART, 128);
   L.gat = o;                                      // gathered q (, k, v) pairs [3][FR_R][32]
   o += 3 * FR_R * 32 * 4;
-  L.ln = o;                                       // LayerNorm gain and bias
-  o += 2 * D * 4;
-  L.xs = o;                                       // the residual rows, fp32
-  o += FR_R * D * 4;
   L.total = o;
   return L;
 }
@@ -392,13 +399,13 @@ __device__ __forceinline__ void share_pieces(uint32_t* gat, int n, int C, uint32
 // LayerNorm 1 -> QKV of head h -> self-attention of head h, one cluster per head
 // ---------------------------------------------------------------------------
 template <int KSW>
-__global__ void __launch_bounds__(FR_T) fr_self_kernel(const __grid_constant__ CUtensorMap kmap,
+__global__ void __launch_bounds__(FR_T, 1) fr_self_kernel(const __grid_constant__ CUtensorMap kmap,
                                                        const __grid_constant__ CUtensorMap vmap,
                                                        const __grid_constant__ FrHead A) {
   constexpr int D = KSW * 128;
   extern __shared__ __align__(1024) uint8_t hs_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(hs_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t wbar, lbar, xbar, gbar, mbar, kvbar;
+  __shared__ __align__(8) uint64_t wbar, gbar, mbar, kvbar;
   __shared__ int s_pos[FR_R];
   const HeadLayout Lo = head_layout(D, A.tiles_max, 1, A.mrg_slots);
   const int tid = threadIdx.x;
@@ -411,8 +418,6 @@ __global__ void __launch_bounds__(FR_T) fr_self_kernel(const __grid_constant__ C
   uint32_t* gat = reinterpret_cast<uint32_t*>(sm + Lo.gat);   // [3][FR_R][32]: q / 8, k, v pairs
   uint8_t* mrg = sm + Lo.mrg;                                 // [chunk][FR_R][66]
   float* part = reinterpret_cast<float*>(sm + Lo.part);
-  float* lnp = reinterpret_cast<float*>(sm + Lo.ln);
-  float* xs = reinterpret_cast<float*>(sm + Lo.xs);
   // this CTA's QKV tiles: local tiles [24 c / C, 24 (c + 1) / C) of the head's
   // 24 (q 0-7, k 8-15, v 16-23)
   const int lt0 = 24 * c / C, lt1 = 24 * (c + 1) / C, ntile = lt1 - lt0;
@@ -424,8 +429,6 @@ __global__ void __launch_bounds__(FR_T) fr_self_kernel(const __grid_constant__ C
   // the merge of utterance b happens in the CTA holding item (b, 0)
   if (tid == 0) {
     mbar_init(&wbar, 1);
-    mbar_init(&lbar, 1);
-    mbar_init(&xbar, 1);
     mbar_init(&gbar, 1);
     mbar_init(&mbar, 1);
     mbar_init(&kvbar, 1);
@@ -450,13 +453,12 @@ __global__ void __launch_bounds__(FR_T) fr_self_kernel(const __grid_constant__ C
         }
     }
     mbar_arrive_expect_tx(&mbar, mrg_bytes);
-    mbar_arrive_expect_tx(&lbar, 8u * d);   // the LayerNorm's gain and bias (constants)
-    bulk_load(lnp, A.ln_g, 4u * d, &lbar);
-    bulk_load(lnp + d, A.ln_b, 4u * d, &lbar);
     mbar_arrive_expect_tx(&wbar, (uint32_t)ntile * wtile);
     for (int i = 0; i < ntile; ++i) bulk_load(wts + i * wtile, A.W + (size_t)gtile(lt0 + i) * 8 * d, wtile, &wbar);
   }
   if (tid < FR_R) s_pos[tid] = A.plan.row_pos[tid];
+  LnRegs<KSW> lnr;
+  fr_ln_params(lnr, A.ln_g, A.ln_b);
   __syncthreads();
   cluster_arrive_relaxed();
   pdl_wait();
@@ -464,12 +466,11 @@ __global__ void __launch_bounds__(FR_T) fr_self_kernel(const __grid_constant__ C
   fr_stamp(A.trace, 1);
   pdl_launch();
   // the residual rows: all FR_R slots at once (rows past the live ones are not used)
-  if (tid < 32) fr_rows_async(A.x, d, 0, 4, 4u * d, FR_R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
+  float4 xv[2][KSW];
+  fr_ln_fetch<KSW>(xv, A.x);
   const int R = *A.plan.n_rows;
   const bool live = R > 0;
-  mbar_wait(&lbar, 0, A.status);
-  mbar_wait(&xbar, 0, A.status);
-  if (live) fr_ln<KSW>(xs, lnp, lnp + d, act, R);
+  if (live) fr_ln_apply<KSW>(xv, lnr, act, R);
   fr_stamp(A.trace, 2);
   mbar_wait(&wbar, 0, A.status);
   fr_stamp(A.trace, 3);
@@ -592,12 +593,12 @@ __global__ void __launch_bounds__(FR_T) fr_self_kernel(const __grid_constant__ C
 // encoder frames, one cluster per head; CTA c takes key chunks c, c + C, ...
 // ---------------------------------------------------------------------------
 template <int KSW>
-__global__ void __launch_bounds__(FR_T) fr_cross_kernel(const __grid_constant__ CUtensorMap xmap,
+__global__ void __launch_bounds__(FR_T, 1) fr_cross_kernel(const __grid_constant__ CUtensorMap xmap,
                                                         const __grid_constant__ FrHead A) {
   constexpr int D = KSW * 128;
   extern __shared__ __align__(1024) uint8_t hs_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(hs_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t wbar, lbar, xbar, gbar, mbar, kvbar[2];
+  __shared__ __align__(8) uint64_t wbar, gbar, mbar, kvbar[2];
   const HeadLayout Lo = head_layout(D, A.tiles_max, 2, A.mrg_slots);
   const int tid = threadIdx.x;
   const int C = A.C, c = (int)cluster_ctarank(), hh = (int)blockIdx.x / C;
@@ -609,8 +610,6 @@ __global__ void __launch_bounds__(FR_T) fr_cross_kernel(const __grid_constant__ 
   uint32_t* gat = reinterpret_cast<uint32_t*>(sm + Lo.gat);   // [FR_R][32] q / 8 pairs
   uint8_t* mrg = sm + Lo.mrg;                                 // [split][FR_R][66]
   float* part = reinterpret_cast<float*>(sm + Lo.part);
-  float* lnp = reinterpret_cast<float*>(sm + Lo.ln);
-  float* xs = reinterpret_cast<float*>(sm + Lo.xs);
   const int lt0 = 8 * c / C, lt1 = 8 * (c + 1) / C, ntile = lt1 - lt0;
   const uint32_t wtile = 16u * (uint32_t)D;
   const long long vofs = A.vofs;
@@ -623,8 +622,6 @@ __global__ void __launch_bounds__(FR_T) fr_cross_kernel(const __grid_constant__ 
   fr_stamp(A.trace, 0);
   if (tid == 0) {
     mbar_init(&wbar, 1);
-    mbar_init(&lbar, 1);
-    mbar_init(&xbar, 1);
     mbar_init(&gbar, 1);
     mbar_init(&mbar, 1);
     mbar_init(&kvbar[0], 1);
@@ -649,13 +646,12 @@ __global__ void __launch_bounds__(FR_T) fr_cross_kernel(const __grid_constant__ 
         tma_load_2d(dst, &xmap, &kvbar[issued], 0, (int)row);
         tma_load_2d(dst + FR_TILE, &xmap, &kvbar[issued], 0, (int)(row + vofs));
       }
-    mbar_arrive_expect_tx(&lbar, 8u * d);   // the LayerNorm's gain and bias (constants)
-    bulk_load(lnp, A.ln_g, 4u * d, &lbar);
-    bulk_load(lnp + d, A.ln_b, 4u * d, &lbar);
     mbar_arrive_expect_tx(&wbar, (uint32_t)ntile * wtile);
     for (int i = 0; i < ntile; ++i)
       bulk_load(wts + i * wtile, A.W + (size_t)(8 * hh + lt0 + i) * 8 * d, wtile, &wbar);
   }
+  LnRegs<KSW> lnr;
+  fr_ln_params(lnr, A.ln_g, A.ln_b);
   __syncthreads();
   cluster_arrive_relaxed();
   pdl_wait();
@@ -663,12 +659,11 @@ __global__ void __launch_bounds__(FR_T) fr_cross_kernel(const __grid_constant__ 
   fr_stamp(A.trace, 1);
   pdl_launch();
   // the residual rows: all FR_R slots at once (rows past the live ones are not used)
-  if (tid < 32) fr_rows_async(A.x, d, 0, 4, 4u * d, FR_R, reinterpret_cast<uint8_t*>(xs), 4u * d, &xbar);
+  float4 xv[2][KSW];
+  fr_ln_fetch<KSW>(xv, A.x);
   const int R = *A.plan.n_rows;
   const bool live = R > 0;
-  mbar_wait(&lbar, 0, A.status);
-  mbar_wait(&xbar, 0, A.status);
-  if (live) fr_ln<KSW>(xs, lnp, lnp + d, act, R);
+  if (live) fr_ln_apply<KSW>(xv, lnr, act, R);
   fr_stamp(A.trace, 2);
   mbar_wait(&wbar, 0, A.status);
   fr_stamp(A.trace, 3);
@@ -835,9 +830,8 @@ cudaError_t launch_fr_pack(const void* src, void* dst, int N, int K, cudaStream_
   return cudaGetLastError();
 }
 
-size_t fr_gemv_smem(int d, int K, int tiles_max, int ks, int mode) {
-  return (size_t)gemv_ln_off(d, tiles_max, K / ks / d, ks) + 8 * (size_t)d +
-         (mode == FR_GELU ? (size_t)FR_R * d * 4 : 0);
+size_t fr_gemv_smem(int d, int K, int tiles_max, int ks) {
+  return (size_t)gemv_smem_bytes(d, tiles_max, K / ks / d, ks);
 }
 
 size_t fr_head_smem(int d, int tiles_max, bool self_attn, int mrg_slots) {
@@ -859,7 +853,7 @@ int fr_configure(int d, int F, int H, int max_pos, int* C_out, int* sms_out, int
   {
     const int t_d = (nt_o + g_d - 1) / g_d;
     void* k = pick(d, 2, FR_RESID, FR_KS);
-    const size_t smem = fr_gemv_smem(d, F, FR_MAXT, FR_KS, FR_RESID);
+    const size_t smem = fr_gemv_smem(d, F, FR_MAXT, FR_KS);
     if ((int)smem > max_smem || t_d > FR_MAXT ||
         cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
       return 0;
@@ -884,11 +878,11 @@ int fr_configure(int d, int F, int H, int max_pos, int* C_out, int* sms_out, int
                           {FR_GELU, 1, d, (nt_f + g_f - 1) / g_f},
                           {FR_RESID, FR_KS, F, (nt_o + g_d - 1) / g_d}};
   for (auto& g : gemv) {
-    const size_t smem = fr_gemv_smem(d, g[2], g[3], g[1], g[0]);
+    const size_t smem = fr_gemv_smem(d, g[2], g[3], g[1]);
     if (g[3] > FR_MAXT || (int)smem > max_smem) return 0;
     void* k = pick(d, 2, g[0], g[1]);
     if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)std::max(smem, g[1] == FR_KS ? fr_gemv_smem(d, F, FR_MAXT, FR_KS, FR_RESID) : smem)) !=
+                             (int)std::max(smem, g[1] == FR_KS ? fr_gemv_smem(d, F, FR_MAXT, FR_KS) : smem)) !=
         cudaSuccess)
       return 0;
   }
@@ -935,7 +929,7 @@ cudaError_t launch_fr_gemv(const FrGemv& a, int mode, int ks, int groups, int d,
   void* k = pick(d, 2, mode, ks);
   if (k == nullptr) return cudaErrorInvalidValue;
   void* args[] = {const_cast<FrGemv*>(&a)};
-  return launch_k(k, dim3(groups * ks), fr_gemv_smem(d, a.K, a.tiles_max, ks, mode), st, pdl, ks, args);
+  return launch_k(k, dim3(groups * ks), fr_gemv_smem(d, a.K, a.tiles_max, ks), st, pdl, ks, args);
 }
 
 cudaError_t launch_fr_self(const CUtensorMap* kmap, const CUtensorMap* vmap, const FrHead& a, cudaStream_t st,

@@ -19,9 +19,9 @@ void launch_w(const WideGemm& g, const Epi& epi, int* status, cudaStream_t st) {
   });
   const dim3 grid((unsigned)(g.M / 128 * SPLIT), (unsigned)((g.N + BN - 1) / BN));
   constexpr int S_MAX = C::STAGES / WG_PIPES;   // stages per pipeline
-  const int S = g.stages >= 2 && g.stages < S_MAX ? g.stages : S_MAX;
-  launch_ex(gemm_wide_kernel<BN, MODE, SPLIT>, grid, dim3(WG_THREADS), C::SMEM, st, g.pdl, SPLIT, g.mapA, g.mapB,
-            g.mapX, g.K, S, epi, status);
+  const int S = g.stages >= 1 && g.stages < S_MAX ? g.stages : S_MAX;
+  launch_ex(gemm_wide_kernel<BN, MODE, SPLIT>, grid, dim3(WG_THREADS), (size_t)C::smem_bytes(S), st, g.pdl, SPLIT,
+            g.mapA, g.mapB, g.mapX, g.K, S, epi, status);
 }
 
 template <int MODE, int SPLIT>

@@ -45,9 +45,9 @@ struct WideCfg {
   static constexpr int LDS = 128 + 4;                                     // staged tile row stride (floats)
   static constexpr int FIT = (WG_DYN_MAX - 1024 - 256 - XT_BYTES) / STAGE_BYTES;
   static constexpr int STAGES = FIT < 8 ? FIT : 8;
-  static constexpr int XT_OFF = STAGES * STAGE_BYTES;
-  static constexpr int BAR_OFF = XT_OFF + XT_BYTES;
-  static constexpr int SMEM = 1024 + BAR_OFF + 256;
+  // dynamic shared memory for s stages per pipeline (the staged tile reuses the ring)
+  static constexpr int smem_bytes(int s) { return 1024 + WG_PIPES * s * STAGE_BYTES + XT_BYTES + 256; }
+  static constexpr int SMEM = smem_bytes(STAGES / WG_PIPES);
   // accumulators, split over the pipelines (within a pipeline the K = 16
   // steps of a k-block rotate over its share)
   static constexpr int NACC = WG_PIPES;
@@ -55,7 +55,7 @@ struct WideCfg {
   static constexpr int BN_MAX = 512 / WG_PIPES / 32 * 32;
   static_assert(STAGES >= 2 * WG_PIPES, "each pipeline needs two stages");
   static_assert(NACC % WG_PIPES == 0, "accumulators split over the pipelines");
-  static_assert(BN * LDS * 4 <= STAGES * STAGE_BYTES, "the staged tile must fit the ring");
+  static_assert(BN * LDS * 4 <= WG_PIPES * STAGE_BYTES, "the staged tile must fit a one-stage ring");
   static_assert(BN % 32 == 0 && BN >= 32 && NACC * BN <= 512, "N tile (the accumulators fill at most 512 columns)");
 };
 
@@ -84,12 +84,14 @@ gemm_wide_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant
   using C = WideCfg<BN, MODE>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // layout for S stages per pipeline: A ring, B ring, residual tile, barriers
+  const int NS = WG_PIPES * S;
   uint8_t* sA = smem;
-  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
-  float* xt = reinterpret_cast<float*>(smem + C::XT_OFF);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::BAR_OFF);
-  uint64_t* empty = full + C::STAGES;
-  uint64_t* done = empty + C::STAGES;   // [WG_PIPES]
+  uint8_t* sB = smem + NS * C::A_BYTES;
+  float* xt = reinterpret_cast<float*>(smem + NS * C::STAGE_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + NS * C::STAGE_BYTES + C::XT_BYTES);
+  uint64_t* empty = full + NS;
+  uint64_t* done = empty + NS;   // [WG_PIPES]
   uint64_t* xbar = done + WG_PIPES;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xbar + 1);
   __shared__ float ln_mu[BN], ln_rs[BN];   // folded LayerNorm: statistics of the tile's rows
@@ -119,7 +121,7 @@ gemm_wide_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant
     tmem_relinquish();
   }
   if (threadIdx.x == 32) {
-    for (int s = 0; s < C::STAGES; ++s) {
+    for (int s = 0; s < NS; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }

@@ -41,7 +41,7 @@ struct WideGemm {
   CUtensorMap mapX;   // RESID: the residual stream [R][d] fp32, box 128 x bn (others: unused)
   int M, N, K;
   int bn, split;      // N tile (32 .. 160, RESID <= 96); 1, or 2 = K split over a cluster pair
-  int stages = 0;     // stages per pipeline, at least 2 (0: as deep as shared memory allows)
+  int stages = 0;     // stages per pipeline, at least 1 (0: as deep as shared memory allows)
   bool pdl = false;
 };
 bool wide_pick(int M, int N, int K, int mode, int sms, int* bn, int* split);
@@ -214,14 +214,15 @@ struct FrHead {
 // ready, 3 weights landed, 4 projection reduced, 5 exchange landed (head:
 // gathered q/k/v; K-split group: the other ranks' partials), 6 attention
 // done (head), 7 exit; head kernels also 8 first K/V chunk landed, 9 first
-// chunk's attention combined, 10 merge inputs landed.  Up to FR_TRACE_CTAS
+// chunk's attention combined, 10 merge inputs landed, 11 (GEMVs without a
+// LayerNorm) bf16 input rows landed.  Up to FR_TRACE_CTAS
 // CTAs per launch.
 constexpr int FR_TRACE_PHASES = 12;
 constexpr int FR_TRACE_CTAS = 320;
 // 1 and the cluster size per head when the kernels run for these dimensions on this device
 // (gd_out: the MLP down-projection's groups of F / d CTAs)
 int fr_configure(int d, int F, int H, int max_pos, int* C_out, int* sms_out, int* gd_out);
-size_t fr_gemv_smem(int d, int K, int tiles_max, int ks, int mode);
+size_t fr_gemv_smem(int d, int K, int tiles_max, int ks);
 size_t fr_head_smem(int d, int tiles_max, bool self_attn, int mrg_slots);
 // groups: CTA groups of ks (one cluster each); a.tiles_max = ceil(N / 8 / groups)
 // Pack a bf16 [N][K] weight matrix (N, K multiples of 8) into the few-row

@@ -67,7 +67,7 @@ def timeline_summary(ns, kinds, rounds):
 
 FEWROW_KINDS = ["qkv_self", "self_out", "query_cross", "cross_out", "mlp_up", "mlp_down"]
 FEWROW_PHASES = ["entry", "past_wait", "rows", "weights", "reduced", "exchange", "attention", "exit", "kv_in",
-                 "combined", "merge_in"]
+                 "combined", "merge_in", "inputs_in"]
 
 
 def fewrow_trace_summary(tr):
@@ -94,7 +94,7 @@ def fewrow_trace_summary(tr):
         med = np.nanmean([np.nanmedian(r, axis=0) for r in acc[k]], axis=0)
         mx = np.nanmean([np.nanmax(r, axis=0) for r in acc[k]], axis=0)
         cells = "".join(f"{a:>8.2f}/{b:<7.2f}" if np.isfinite(a) else f"{'-':>16}"
-                        for a, b in zip(med[:11], mx[:11]))
+                        for a, b in zip(med[:12], mx[:12]))
         lines.append(f"  {k:<12}{cells}{mx[7]:>9.2f}")
     return "\n".join(lines)
 
