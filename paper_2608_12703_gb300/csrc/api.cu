@@ -85,6 +85,7 @@ struct asr_spec {
   std::map<int, CUtensorMap> xmaps;                   // BN -> map of the residual stream (fp32, box 128 x BN)
   int n_sms = 0;
   bool use_wide = true;   // many-row projections on the one-tile-per-SM kernel (ASRSPEC_WIDE=0: the split-K chain)
+  int fr_prefetch = 3;    // few-row launches prefetch the weights of the launch this many ahead into L2 (0: none)
   int wide_stages = 0;    // its stages per pipeline (ASRSPEC_WIDE_STAGES; 0 = as deep as shared memory allows)
 
   // profiling: CUDA events around each kernel class (direct launches only)
@@ -578,6 +579,20 @@ int run_layers_few(asr_spec* h) {
                  nullptr, nullptr, nullptr, h->V, h->maxpos, h->status);
   }
   auto bf = [](void* p) { return static_cast<const __nv_bfloat16*>(p); };
+  // the packed weights of the layers' six launches in launch order, for the
+  // L2 prefetch of a later launch's weights
+  auto later = [&](int l, int slot, const void** pf, uint32_t* bytes) {
+    const int g = 6 * l + slot + h->fr_prefetch;
+    *pf = nullptr;
+    *bytes = 0;
+    if (h->fr_prefetch <= 0 || g >= 6 * h->L) return;
+    const LayerW& n = h->lw[g / 6];
+    const uint32_t dd = (uint32_t)d * d * 2, fd = (uint32_t)F * d * 2;
+    const void* p[6] = {n.p_qkv, n.p_wo, n.p_wcq, n.p_wco, n.p_w1, n.p_w2};
+    const uint32_t b[6] = {3 * dd, dd, dd, dd, fd, fd};
+    *pf = p[g % 6];
+    *bytes = b[g % 6];
+  };
   for (int l = 0; l < h->L; ++l) {
     LayerW& w = h->lw[l];
     FrHead hd{};
@@ -604,6 +619,7 @@ int run_layers_few(asr_spec* h) {
     hs.vs = static_cast<__nv_bfloat16*>(h->vself) + l * self_layer;
     hs.row0 = (long long)l * h->Bmax * H * h->maxpos;
     hs.t_alloc = h->maxpos;
+    later(l, 0, &hs.pf, &hs.pf_bytes);
     {
       Prof p(h, ASR_PROF_QKV_SELF, 1);
       Tl t(h, ASR_TL_QKV_SELF);
@@ -624,6 +640,7 @@ int run_layers_few(asr_spec* h) {
     go.K = d;
     go.tiles_max = (nt_o + g_o - 1) / g_o;
     go.a = static_cast<const __nv_bfloat16*>(h->att);
+    later(l, 1, &go.pf, &go.pf_bytes);
     {
       Prof p(h, ASR_PROF_RESID, 1);
       Tl t(h, ASR_TL_GEMM + EPI_RESID);
@@ -644,6 +661,7 @@ int run_layers_few(asr_spec* h) {
     hc.t_alloc = h->Tmax;
     hc.q_anchor = l == h->anchor ? h->q_anchor : nullptr;
     hc.ml = l == h->anchor ? h->ml : nullptr;
+    later(l, 2, &hc.pf, &hc.pf_bytes);
     {
       Prof p(h, ASR_PROF_QUERY_CROSS, 1);
       Tl t(h, ASR_TL_QUERY_CROSS);
@@ -655,6 +673,7 @@ int run_layers_few(asr_spec* h) {
     FrGemv gc = go;
     gc.W = bf(w.p_wco);
     gc.bias = w.bco;
+    later(l, 3, &gc.pf, &gc.pf_bytes);
     {
       Prof p(h, ASR_PROF_RESID, 1);
       Tl t(h, ASR_TL_GEMM + EPI_RESID);
@@ -672,6 +691,7 @@ int run_layers_few(asr_spec* h) {
     gu.ln_g = w.ln3g;
     gu.ln_b = w.ln3b;
     gu.h_out = static_cast<__nv_bfloat16*>(h->hbuf);
+    later(l, 4, &gu.pf, &gu.pf_bytes);
     {
       Prof p(h, ASR_PROF_UP, 1);
       Tl t(h, ASR_TL_GEMM + EPI_GELU);
@@ -687,6 +707,7 @@ int run_layers_few(asr_spec* h) {
     gd.K = F;
     gd.tiles_max = (nt_o + g_d - 1) / g_d;
     gd.a = static_cast<const __nv_bfloat16*>(h->hbuf);
+    later(l, 5, &gd.pf, &gd.pf_bytes);
     {
       Prof p(h, ASR_PROF_RESID, 1);
       Tl t(h, ASR_TL_GEMM + EPI_RESID);
@@ -927,6 +948,7 @@ int asr_spec_create(const asr_model_dims* dims, const asr_weights* weights, void
     if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&h->n_sms, cudaDevAttrMultiProcessorCount, dev);
   }
   if (const char* e = std::getenv("ASRSPEC_WIDE")) h->use_wide = std::atoi(e) != 0;
+  if (const char* e = std::getenv("ASRSPEC_FR_PREFETCH")) h->fr_prefetch = std::max(0, std::atoi(e));
   if (const char* e = std::getenv("ASRSPEC_WIDE_STAGES")) h->wide_stages = std::max(0, std::atoi(e));
   {   // bounds-check mode: process-wide (each kernel module's constant), set by every create
     const char* e = std::getenv("ASRSPEC_CHECK");

@@ -138,6 +138,15 @@ __device__ __forceinline__ void fr_ln_apply(const float4 (&v)[2][KSW], const LnR
   }
 }
 
+// Thread 0: this CTA's share of a later launch's weights into L2 (that
+// launch's CTAs become resident only as this one's leave).
+__device__ __forceinline__ void fr_prefetch(const void* pf, uint32_t pf_bytes) {
+  if (pf == nullptr || pf_bytes == 0) return;
+  const uint32_t per = ((pf_bytes / gridDim.x) + 15u) & ~15u;
+  const uint32_t s0 = blockIdx.x * per;
+  if (s0 < pf_bytes) l2_prefetch(static_cast<const char*>(pf) + s0, per < pf_bytes - s0 ? per : pf_bytes - s0);
+}
+
 // Weight tiles of the few-row kernels are packed (at create) so that one
 // 8-row tile is contiguous and its 16-byte pieces run piece-major: piece c of
 // row r (columns 8 c .. 8 c + 7) at byte 16 (8 c + r).  A tile then lands
@@ -250,6 +259,7 @@ __global__ void __launch_bounds__(FR_T, 1) fr_gemv_kernel(const __grid_constant_
     mbar_arrive_expect_tx(&wbar, (uint32_t)ntile * wtile);
     for (int i = 0; i < ntile; ++i)
       bulk_load(wts + i * wtile, A.W + ((size_t)(t0 + i) * A.K + (size_t)ks * Kc) * 8, wtile, &wbar);
+    fr_prefetch(A.pf, A.pf_bytes);
   }
   LnRegs<KSW> lnr;
   if constexpr (MODE == FR_GELU) fr_ln_params(lnr, A.ln_g, A.ln_b);
@@ -455,6 +465,7 @@ __global__ void __launch_bounds__(FR_T, 1) fr_self_kernel(const __grid_constant_
     mbar_arrive_expect_tx(&mbar, mrg_bytes);
     mbar_arrive_expect_tx(&wbar, (uint32_t)ntile * wtile);
     for (int i = 0; i < ntile; ++i) bulk_load(wts + i * wtile, A.W + (size_t)gtile(lt0 + i) * 8 * d, wtile, &wbar);
+    fr_prefetch(A.pf, A.pf_bytes);
   }
   if (tid < FR_R) s_pos[tid] = A.plan.row_pos[tid];
   LnRegs<KSW> lnr;
@@ -649,6 +660,7 @@ __global__ void __launch_bounds__(FR_T, 1) fr_cross_kernel(const __grid_constant
     mbar_arrive_expect_tx(&wbar, (uint32_t)ntile * wtile);
     for (int i = 0; i < ntile; ++i)
       bulk_load(wts + i * wtile, A.W + (size_t)(8 * hh + lt0 + i) * 8 * d, wtile, &wbar);
+    fr_prefetch(A.pf, A.pf_bytes);
   }
   LnRegs<KSW> lnr;
   fr_ln_params(lnr, A.ln_g, A.ln_b);

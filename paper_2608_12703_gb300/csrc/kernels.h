@@ -187,6 +187,8 @@ struct FrGemv {
   int* status;
   unsigned long long* tl;
   unsigned long long* trace;   // per-CTA phase stamps [CTA][FR_TRACE_PHASES] (diagnostics), or null
+  const void* pf;              // a later launch's weights, prefetched into L2 (or null)
+  uint32_t pf_bytes;
 };
 struct FrHead {
   const __nv_bfloat16* W;   // self: fused QKV weights [3d][d]; cross: query weights [d][d]
@@ -208,6 +210,8 @@ struct FrHead {
   int* status;
   unsigned long long* tl;
   unsigned long long* trace;   // per-CTA phase stamps [CTA][FR_TRACE_PHASES] (diagnostics), or null
+  const void* pf;              // a later launch's weights, prefetched into L2 (or null)
+  uint32_t pf_bytes;
 };
 // Phase stamps of a traced few-row launch, GPU global timer (ns), thread 0 of
 // each CTA: 0 entry, 1 past the wait on the previous launch, 2 input rows
