@@ -392,6 +392,8 @@ static void configure_one() {
 void configure_attention_tc() {
   static std::once_flag once;
   std::call_once(once, [] {
+    configure_one<1, 1, false>();
+    configure_one<2, 1, false>();
     configure_one<1, 2, false>();
     configure_one<2, 2, false>();
     configure_one<1, 2, true>();
@@ -425,7 +427,12 @@ void launch_attention_tc(const AttnArgs& a, int* status, cudaStream_t st) {
     }
     return;
   }
-  if (a.splits == 1) {   // one CTA per (utterance, head): 2-deep ring, three CTAs per SM (54 vs 56 us at batch 64)
+  if (a.splits == 1 && a.causal) {   // self-attention, one CTA per (utterance, head): a one-chunk ring,
+    // five CTAs per SM (a few chunks per utterance; 636 vs 721 us per batch-64 round)
+    if (a.rows_max > 16) launch_one<2, 1, false, false>(a, a.splits, status, st);
+    else launch_one<1, 1, false, false>(a, a.splits, status, st);
+  } else if (a.splits == 1) {   // cross-attention, one CTA per (utterance, head): 2-deep ring, three CTAs per SM
+    // (54 vs 56 us at batch 64)
     if (a.rows_max > 16) launch_one<2, 2, false, false>(a, a.splits, status, st);
     else launch_one<1, 2, false, false>(a, a.splits, status, st);
   } else if (a.causal) {   // self-attention keys split over a cluster (at most max_pos keys)
