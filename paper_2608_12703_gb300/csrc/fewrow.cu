@@ -16,17 +16,18 @@
 //              frames split over the cluster, merged in split order;
 //   out        cross-attention output projection + residual (GEMV);
 //   up         LayerNorm 3 -> MLP up-projection + GELU (GEMV);
-//   down       MLP down-projection + residual (GEMV, K split over a pair of
-//              CTAs).
+//   down       MLP down-projection + residual (GEMV, K split over a cluster
+//              of 4 CTAs).
 // Every CTA computes whole 8-feature output tiles over its K range (mma.sync
 // m16n8k16, the rows padded to 16 as M, 8 weight rows as N; the K range
 // split over 8 warps and summed in warp order), so no split-K exchange is
-// needed except in the down-projection pair.  Weights (and the attention
+// needed except in the down-projection cluster.  Weights (and the attention
 // K/V, constant during a step) are requested before the wait on the previous
-// launch.  (Prefetching the weights of the launch two places later into L2,
-// at a CTA's start or at its end, was measured slower: 1470-1700 against
-// 1407 us per batch-1 round of the large decoder.)
-// The LayerNorm is computed by its consumers from the fp32 residual stream.
+// launch, and each launch prefetches into L2 the weights of a later launch
+// (the host picks which: three ahead by default).
+// The LayerNorm is computed by its consumers from the fp32 residual stream,
+// in registers: gain and bias before the wait, the rows straight from L2
+// after it.
 #include <algorithm>
 #include <mutex>
 
