@@ -42,11 +42,39 @@ UNIT = {"byte": 1.0, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "KB": 1e3, "MB": 
         "Kibyte": 1024.0, "Mibyte": 1024.0 ** 2, "Gibyte": 1024.0 ** 3}
 
 
+def code_text(src: str) -> str:
+    """The source with its comments removed and every run of whitespace made
+    one space: what the compiled code depends on (string and character
+    literals are kept as they are)."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if c in "\"'":                                     # a literal, up to its unescaped end
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        elif src.startswith("//", i):                     # to the end of the line
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+            out.append(" ")
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+            out.append(" ")
+        else:
+            out.append(c)
+            i += 1
+    return " ".join("".join(out).split())
+
+
 def source_hash(group: str) -> str:
+    """Hash of the code (comments and layout ignored) of a kernel's sources."""
     h = hashlib.sha256()
     for rel in SOURCE_GROUPS[group]:
-        with open(os.path.join(PKG, rel), "rb") as f:
-            h.update(rel.encode() + b"\0" + f.read())
+        with open(os.path.join(PKG, rel), encoding="utf-8") as f:
+            h.update(rel.encode() + b"\0" + code_text(f.read()).encode())
     return h.hexdigest()[:16]
 
 

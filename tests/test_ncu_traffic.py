@@ -48,3 +48,13 @@ def test_record_replaces_the_same_key(traffic):
     NT.record(str(traffic), "attn_tc", "w", "resid", "attn_tc", "b.md")
     ents = json.load(open(NT.TRAFFIC_FILE))["entries"]
     assert len(ents) == 1 and ents[0]["summary"] == "b.md"
+
+
+def test_code_text_ignores_comments_and_layout_only():
+    a = 'int f(int x) {  // the input\n  return x + 1; /* one more */\n}\nconst char* s = "// kept";\n'
+    b = 'int f(int x) {\n    return x + 1;\n}   // reworded note\nconst char* s = "// kept";'
+    c = 'int f(int x) { return x + 2; }\nconst char* s = "// kept";'
+    assert NT.code_text(a) == NT.code_text(b)
+    assert NT.code_text(a) != NT.code_text(c)
+    assert '"// kept"' in NT.code_text(a)
+    assert NT.code_text("char q = '\"'; /* x */ int y;") == "char q = '\"'; int y;"
